@@ -85,14 +85,22 @@ def dequantize_unit(b: int, codes: np.ndarray, scale: np.ndarray, zero: np.ndarr
 
 
 def dequantize_factor(layer: Dict, h: int, e: int) -> np.ndarray:
-    """P_hat_e^(h) as an I x n matrix whose column k is p_hat_{e,h,k}."""
+    """P_hat_e^(h) as an I x n matrix whose column k is p_hat_{e,h,k}: the
+    per-unit definition of dequantize_unit applied to all units at once."""
     I, n, group = layer["I"], layer["n"], layer["group"]
-    P = np.empty((I, n), dtype=np.float64)
-    bits = layer["bits"][h, e]
-    for k in range(n):
-        P[:, k] = dequantize_unit(int(bits[k]), layer["codes"][h, e, k],
-                                  layer["scale"][h, e, k], layer["zero"][h, e, k], group)
-    return P
+    bits = np.asarray(layer["bits"][h, e])
+    codes = layer["codes"][h, e]
+    P = np.zeros((n, I), dtype=np.float64)          # row k = unit k
+    q = (bits > 0) & (bits < 16)
+    if q.any():
+        g = np.arange(I) // group
+        s = f16_bits_to_f64(layer["scale"][h, e][q])[:, g]
+        z = f16_bits_to_f64(layer["zero"][h, e][q])[:, g]
+        P[q] = s * (codes[q].astype(np.float64) - z)
+    f = bits == 16
+    if f.any():
+        P[f] = f16_bits_to_f64(codes[f])
+    return P.T
 
 
 def basis(layer: Dict, h: int) -> np.ndarray:
@@ -172,18 +180,15 @@ def moe_forward_factored(layer: Dict, x_bits: np.ndarray, logits: np.ndarray,
     zu = x @ basis(layer, UP)
     s_acc = np.zeros((T, layer["n"]), dtype=np.float64)
     hidden = {}
-    cache = {}
-    for t in range(T):
-        for s in range(top_k):
-            e = int(idx[t, s])
-            if e not in cache:
-                cache[e] = tuple(dequantize_factor(layer, h, e) for h in (GATE, UP, DOWN))
-            Pg, Pu, Pd = cache[e]
+    for e in sorted(set(int(v) for v in idx.ravel())):   # one expert's factors at a time
+        Pg, Pu, Pd = (dequantize_factor(layer, h, e) for h in (GATE, UP, DOWN))
+        for t, s in zip(*np.nonzero(idx == e)):
             gate = Pg @ (alpha(layer, GATE, e) * zg[t])
             up = Pu @ (alpha(layer, UP, e) * zu[t])
             hvec = silu(gate) * up
-            hidden[(t, e)] = hvec
+            hidden[(int(t), e)] = hvec
             s_acc[t] += w[t, s] * alpha(layer, DOWN, e) * (Pd.T @ hvec)
+        del Pg, Pu, Pd
     y = s_acc @ basis(layer, DOWN).T
     if return_parts:
         return y, dict(idx=idx, w=w, zg=zg, zu=zu, s=s_acc, hidden=hidden)

@@ -346,3 +346,15 @@ def test_factored_equals_dense_tiny(alpha_scale):
     yd = oracle.moe_forward_dense(layer, x, logits, spec.top_k)
     yf = oracle.moe_forward_factored(layer, x, logits, spec.top_k)
     np.testing.assert_allclose(yf, yd, rtol=1e-9, atol=1e-11 * np.abs(yd).max())
+
+
+def test_factor_matrix_matches_per_unit_definition():
+    spec = _tiny_spec(n=40, I=96, group=32)
+    layer = synth.make_layer(spec, seed=21, bits_dist={0: .1, 1: .15, 2: .2, 3: .15, 4: .1, 6: .1, 8: .1, 16: .1})
+    for h in range(3):
+        for e in range(spec.E):
+            P = oracle.dequantize_factor(layer, h, e)
+            for k in range(spec.n):
+                col = oracle.dequantize_unit(int(layer["bits"][h, e, k]), layer["codes"][h, e, k],
+                                             layer["scale"][h, e, k], layer["zero"][h, e, k], spec.group)
+                np.testing.assert_array_equal(P[:, k], col)
