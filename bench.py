@@ -1,0 +1,389 @@
+#!/usr/bin/env python3
+"""Benchmark of the BitsMoE quantized MoE-layer forward on GB300.
+
+Default workload: the Qwen3-30B-A3B-shaped MoE layer (hidden 2048, 128 experts,
+top-8, intermediate 768, shared-basis rank 2048, 2.0 mean unit bits, group 128),
+batch-1 decode.  A step is one bitsmoe_moe_forward call (routing, shared-basis
+projection, gate/up factors + SwiGLU, down factor + weighted expert sum, output
+basis) on one synthetic token.
+
+  value   tokens/s with inputs resident in HBM: K forwards replayed from CUDA
+          graphs on one stream, timed with CUDA events; the layer rotates over
+          `--copies` packed copies (each step touches ~36 MB; the rotation set is
+          far larger than the 129 MB L2, so weights stream from HBM).
+  e2e     the same metric through bitsmoe_moe_forward_host: pinned host input
+          -> device, forward, y -> pinned host, synchronised, every step.
+  roofline  dominant phase (from bitsmoe_profile_forward, phases serialised and
+          timed with CUDA events), algorithmic bytes / its duration, against the
+          measured HBM copy bandwidth.
+  cpu_baseline  the fp64 oracle on the host cores, on a bounded sample.
+
+`--impl reference` times the oracle (the only reference for this path) on the
+host cores instead and prints the same JSON line with "impl": "reference".
+Multi-GPU: the forward does not shard, so `--gpus N` under torchrun runs N
+independent replicas (weak scaling, no collective in the data path).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "MoE-layer decode tokens/s at 2.0 avg bits; achieved HBM GB/s vs ~8 TB/s peak"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+PHASES = ["route", "basis_proj_gate_up", "gate_up_factors", "down_factor_sum", "out_basis"]
+KERNELS_PER_FORWARD = 5
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except Exception:
+        return {"hbm_gbs": FALLBACK_HBM_GBS}, "fallback"
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def host_route(logits, k):
+    """Experts each token is routed to (k largest logits, ties to the lower index):
+    used only to count the algorithmic bytes of a step."""
+    out = []
+    for row in logits:
+        order = np.lexsort((np.arange(row.size), -row.astype(np.float64)))[:k]
+        out.append(order)
+    return np.array(out)
+
+
+# --------------------------------------------------------------------------
+# clocks sampled during the timed region
+# --------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.file = None
+        self.t0 = self.t1 = None
+
+    def start(self):
+        try:
+            self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "20"], stdout=self.file, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+
+    def mark(self, which):
+        setattr(self, which, time.time())
+
+    def stop(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
+        time.sleep(0.1)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.file.flush()
+        self.file.seek(0)
+        rows = []
+        for line in self.file.read().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                ts = time.mktime(time.strptime(parts[0].split(".")[0], "%Y/%m/%d %H:%M:%S"))
+                frac = float("0." + parts[0].split(".")[1]) if "." in parts[0] else 0.0
+                rows.append((ts + frac, float(parts[1]), float(parts[2]), parts[5:9]))
+            except Exception:
+                continue
+        os.unlink(self.file.name)
+        window = [r for r in rows if self.t0 and self.t1 and self.t0 - 0.05 <= r[0] <= self.t1 + 0.05]
+        src = "timed_region"
+        if not window:
+            window, src = rows, "whole_run"
+        if not window:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no_samples"], "samples": 0}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in window for i, v in enumerate(r[3]) if v.lower().startswith("active")})
+        return {"sm_mhz": statistics.median(r[1] for r in window), "sm_max_mhz": max(r[2] for r in window),
+                "reasons": reasons, "samples": len(window), "window": src}
+
+
+# --------------------------------------------------------------------------
+# CPU baseline: the oracle on the host cores
+# --------------------------------------------------------------------------
+def oracle_tokens_per_s(spec, layer, T, budget_s=12.0, max_steps=None, seed=0):
+    import oracle
+    times, toks, steps = [], 0, 0
+    t_start = time.perf_counter()
+    while True:
+        x, logits = synth.make_inputs(spec, T, seed=seed, step=1000 + steps)
+        t = time.perf_counter()
+        oracle.moe_forward_factored(layer, x, logits, spec.top_k)
+        times.append(time.perf_counter() - t)
+        toks += T
+        steps += 1
+        if (max_steps and steps >= max_steps) or time.perf_counter() - t_start > budget_s:
+            break
+    return toks / sum(times), steps, sum(times)
+
+
+def cpu_cores():
+    try:
+        from threadpoolctl import threadpool_info
+        n = max((i.get("num_threads", 1) for i in threadpool_info()), default=None)
+        if n:
+            return int(n)
+    except Exception:
+        pass
+    return os.cpu_count() or 1
+
+
+# --------------------------------------------------------------------------
+def run_reference(args, spec, T):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    layer = synth.make_layer(spec, seed=0)
+    # warmup steps (bounded), then K steps each a bounded sample: one oracle forward of T tokens
+    oracle_tokens_per_s(spec, layer, T, budget_s=5.0, max_steps=max(1, min(args.warmup, 3)))
+    budget = float(os.environ.get("BITSMOE_REF_BUDGET_S", "90"))
+    v, steps, secs = oracle_tokens_per_s(spec, layer, T, budget_s=budget, max_steps=args.steps)
+    cores = cpu_cores()
+    line = {
+        "impl": "reference", "metric": METRIC, "value": v, "unit": "tokens/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * secs / steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": config_of(spec, T, args),
+        "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                         "sample": f"{steps} of {args.steps} steps timed ({secs:.1f} s), one fp64 numpy "
+                                   f"factored forward of {T} token(s) per step"},
+        "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def config_of(spec, T, args):
+    return {"workload": f"{spec.name}: Qwen3-30B-A3B-shaped MoE layer" if spec.name.startswith("qw3") else spec.name,
+            "hidden": spec.D, "experts": spec.E, "top_k": spec.top_k, "intermediate": spec.I,
+            "rank": spec.n, "group": spec.group, "mean_unit_bits": spec.mean_bits, "tokens_per_step": T,
+            "l2": f"rotating {args.copies} packed layer copies (>> 129 MB L2)", "seed": 0}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20000)
+    ap.add_argument("--warmup", type=int, default=200)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="qw3")
+    ap.add_argument("--tokens", type=int, default=None)
+    ap.add_argument("--copies", type=int, default=8)
+    ap.add_argument("--inputs", type=int, default=64)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--graph", type=int, default=256, help="forwards per captured CUDA graph")
+    args = ap.parse_args()
+    spec = synth.WORKLOADS[args.workload]
+    T = args.tokens or spec.tokens[0]
+    if args.impl == "reference":
+        run_reference(args, spec, T)
+        return
+
+    import torch
+    import paper_2606_00079_gb300 as bm
+    from paper_2606_00079_gb300 import build as bmbuild
+    bmbuild.build()
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    # ---- workload: one generated layer, packed once, uploaded as rotating copies
+    layer = synth.make_layer(spec, seed=0)
+    blob = bm.bitsmoe_pack_to_host(layer)
+    copies = [bm.bitsmoe_load_blob(blob, device=local) for _ in range(args.copies)]
+    L0 = copies[0]
+    moved = np.array([L0.expert_moved_bytes(e) for e in range(spec.E)], dtype=np.float64)  # E x 3
+    NI = args.inputs
+    xs, lgs, routes = [], [], []
+    for i in range(NI):
+        x, lg = synth.make_inputs(spec, T, seed=0, step=i)
+        xs.append(torch.from_numpy(x.view(np.int16)).to(dev))
+        lgs.append(torch.from_numpy(lg).to(dev))
+        routes.append(host_route(lg, spec.top_k))
+    ws = bm.Workspace(L0, T, spec.top_k, device=dev)
+    y = torch.empty((T, spec.D), dtype=torch.float32, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def step_args(i):
+        return xs[i % NI], lgs[i % NI], copies[i % args.copies]
+
+    def fwd(i, st):
+        x, lg, L = step_args(i)
+        bm.bitsmoe_moe_forward(x.data_ptr(), lg.data_ptr(), T, spec.top_k, L, y.data_ptr(), ws.ptr, ws.nbytes,
+                               st.cuda_stream)
+
+    # algorithmic bytes per step (bases, routed experts' factors, x, logits, y)
+    base_bytes = 3.0 * spec.D * spec.n * 2 + T * spec.D * 2 + T * spec.E * 4 + T * spec.D * 4
+
+    def step_bytes(i):
+        used = np.unique(routes[i % NI])
+        return base_bytes + moved[used].sum()
+
+    # ---- warmup (eager) then capture graphs of forwards
+    with torch.cuda.stream(stream):
+        for i in range(min(args.warmup, 8)):
+            fwd(i, stream)
+    stream.synchronize()
+    G = max(1, min(args.graph, args.steps))
+
+    def capture(n, offset):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for i in range(n):
+                fwd(offset + i, stream)
+        return g
+
+    nfull, rem = divmod(args.steps, G)
+    g_main = capture(G, 0)
+    g_rem = capture(rem, nfull * G) if rem else None
+    with torch.cuda.stream(stream):
+        for _ in range(max(1, args.warmup // G)):
+            g_main.replay()
+    stream.synchronize()
+
+    clk = ClockSampler(local)
+    clk.start()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clk.mark("t0")
+    e0.record(stream)
+    with torch.cuda.stream(stream):
+        for _ in range(nfull):
+            g_main.replay()
+        if g_rem is not None:
+            g_rem.replay()
+    e1.record(stream)
+    e1.synchronize()
+    clk.mark("t1")
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    clocks = clk.stop()
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+    total_bytes = sum(step_bytes(i) for i in range(args.steps))
+    value = world * args.steps * T / (ms / 1e3)
+    fwd_gbs = total_bytes / (ms / 1e3) / 1e9
+
+    # ---- per-phase roofline (phases serialised, CUDA events on the launch stream)
+    phase_ms = np.zeros(5)
+    nprof = 64
+    for i in range(nprof):
+        x, lg, L = step_args(i)
+        phase_ms += bm.bitsmoe_profile_forward(x.data_ptr(), lg.data_ptr(), T, spec.top_k, L, y.data_ptr(),
+                                               ws.ptr, ws.nbytes, stream.cuda_stream)
+    phase_ms /= nprof
+    mean_moved = np.mean([moved[np.unique(routes[i % NI])].sum(axis=0) for i in range(nprof)], axis=0)
+    P = T * spec.top_k
+    phase_bytes = [
+        T * spec.E * 4,
+        2.0 * spec.D * spec.n * 2 + T * spec.D * 2 + 2.0 * T * spec.n * 4,
+        mean_moved[0] + mean_moved[1] + 2.0 * T * spec.n * 4 + 2.0 * P * spec.I * 4,
+        mean_moved[2] + 2.0 * P * spec.I * 4 + T * spec.n * 4,
+        1.0 * spec.D * spec.n * 2 + T * spec.n * 4 + T * spec.D * 4,
+    ]
+    dom = int(np.argmax(phase_ms))
+    peaks, peak_src = measured_peaks()
+    peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    achieved = phase_bytes[dom] / (phase_ms[dom] / 1e3) / 1e9
+    roofline = {"bound": "hbm", "kernel": PHASES[dom], "achieved": achieved, "peak": peak,
+                "peak_source": peak_src, "unit": "GB/s", "frac": achieved / peak, "traffic": None,
+                "phase_ms": {PHASES[i]: float(phase_ms[i]) for i in range(5)},
+                "phase_bytes": {PHASES[i]: float(phase_bytes[i]) for i in range(5)},
+                "forward_gbs": fwd_gbs, "forward_frac_of_measured": fwd_gbs / peak,
+                "forward_frac_of_8tbs": fwd_gbs / NOMINAL_HBM_GBS}
+
+    # ---- e2e through the host-buffer entry point (pinned host memory)
+    xh = [torch.from_numpy(synth.make_inputs(spec, T, seed=0, step=i)[0].view(np.int16)).pin_memory()
+          for i in range(8)]
+    lh = [torch.from_numpy(synth.make_inputs(spec, T, seed=0, step=i)[1]).pin_memory() for i in range(8)]
+    yh = torch.empty((T, spec.D), dtype=torch.float32).pin_memory()
+    ne2e = max(10, min(args.steps, 2000))
+
+    def host_call(i):
+        L = copies[i % args.copies]
+        rc = bm._lib().bitsmoe_moe_forward_host(xh[i % 8].data_ptr(), lh[i % 8].data_ptr(), T, spec.top_k,
+                                                L.handle, yh.data_ptr(), ws.ptr, ws.nbytes, stream.cuda_stream)
+        if rc != 0:
+            raise bm.BitsMoEError(rc, "bitsmoe_moe_forward_host")
+
+    for i in range(5):
+        host_call(i)
+    t0 = time.perf_counter()
+    for i in range(ne2e):
+        host_call(i)
+    e2e_s = time.perf_counter() - t0
+    e2e = {"value": world * ne2e * T / e2e_s, "unit": "tokens/s", "steps": ne2e,
+           "h2d_bytes_per_step": T * spec.D * 2 + T * spec.E * 4, "d2h_bytes_per_step": T * spec.D * 4}
+
+    # ---- CPU baseline (rank 0, N = 1 only)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        v, steps, secs = oracle_tokens_per_s(spec, layer, T, budget_s=12.0)
+        cpu = {"value": v, "unit": "tokens/s", "cores": cpu_cores(), "kind": "oracle",
+               "sample": f"{steps} decode steps of {T} token(s), fp64 numpy factored forward ({secs:.1f} s)"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32",
+            "arith": "bf16 basis x f32 (f32 accumulate); u8 codes x i16 activations (dp2a, i32 accumulate)",
+            "data": "synthetic", "config": config_of(spec, T, args),
+            "hbm_gbs": fwd_gbs, "hbm_frac_of_8tbs": fwd_gbs / NOMINAL_HBM_GBS, "hbm_frac_of_measured": fwd_gbs / peak,
+            "bytes_per_step": total_bytes / args.steps,
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks,
+            "gpu_launches": args.steps * KERNELS_PER_FORWARD,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.barrier()
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

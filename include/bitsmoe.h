@@ -1,0 +1,189 @@
+/*
+ * bitsmoe.h - C ABI of libbitsmoe: the BitsMoE quantized MoE-layer forward
+ * (Stage 3 of the method) on one GB300 (sm_103a).
+ *
+ * The method (BitsMoE paper, Sec. "Shared-basis Spectral Decomposition" and
+ * Fig. 1 Stage 3; identity of Eq. app_normalized_decomposition) stores each
+ * routed expert e and projection h in {gate, up, down} as
+ *
+ *     W_e^(h) = P_e^(h) A_e^(h) Phi_h^T     (gate, up;  P: I x n,  Phi: D x n)
+ *     W_e^(h) = Phi_h A_e^(h) P_e^(h)^T     (down)
+ *
+ * with an unquantised shared basis Phi_h per projection type, spectral
+ * energies A = diag(alpha) and a normalised spectral factor P whose columns
+ * ("units", one rank-1 direction each, length I) are quantised with their own
+ * bit-width b in {0,1,2,3,4,6,8,16} (Eqs. quantized_spectral_vector,
+ * piecewise_error_surrogate).  At inference the activation is projected once
+ * onto the shared bases and the quantised factors are applied inside the
+ * kernels without rebuilding W ("Inference Efficiency", Sec. Experiments):
+ *
+ *     z_g = Phi_g^T x,  z_u = Phi_u^T x                          (once per layer)
+ *     h_e = SiLU(P_g,e (alpha_g,e * z_g)) * (P_u,e (alpha_u,e * z_u))
+ *     s   = sum_{e in topk} w_e * alpha_dn,e * (P_dn,e^T h_e)
+ *     y   = Phi_dn s                                              (once per token)
+ *
+ * Conventions for every entry point:
+ *   - return BITSMOE_OK (0) on success, a negative BITSMOE_ERR_* code otherwise;
+ *     no exception, abort, assert or device trap crosses the ABI;
+ *   - "device" pointers are CUDA device (or managed) memory of the device the
+ *     layer was packed on; "host" pointers are ordinary host memory;
+ *   - a stream is a cudaStream_t passed as void* (NULL = legacy default stream).
+ */
+#ifndef BITSMOE_H
+#define BITSMOE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define BITSMOE_OK                      0
+#define BITSMOE_ERR_INVALID_ARG        -1  /* null pointer, bad top_k, negative T ...            */
+#define BITSMOE_ERR_SHAPE              -2  /* unsupported dims / group size                      */
+#define BITSMOE_ERR_UNSUPPORTED_BITS   -3  /* a unit bit-width outside {0,1,2,3,4,6,8,16}         */
+#define BITSMOE_ERR_WORKSPACE_TOO_SMALL -4
+#define BITSMOE_ERR_ALIGNMENT          -5  /* device pointer not 16-byte aligned                 */
+#define BITSMOE_ERR_CUDA               -6  /* a CUDA runtime call failed (see bitsmoe_last_cuda_error) */
+#define BITSMOE_ERR_OOM                -7  /* host or device allocation failed                   */
+#define BITSMOE_ERR_TIMEOUT            -8  /* a bounded device-side wait ran out                  */
+#define BITSMOE_ERR_DEVICE_BOUNDS      -9  /* a device-side bounds check failed (access skipped) */
+#define BITSMOE_ERR_BLOB              -10  /* packed blob is malformed / wrong version           */
+
+/* Host description of one quantised MoE layer (all host pointers, read-only,
+ * owned by the caller; row-major, C order).
+ *
+ *   D      hidden size (>= 1)
+ *   E      routed experts (1 .. 1024)
+ *   I      expert intermediate size = length of a spectral unit; I % group == 0
+ *   n      shared-basis rank = units per (projection, expert), 1 .. 65535
+ *   group  quantisation group along the unit vector: 32, 64, 128 or 256
+ *   basis  [3] pointers, h = 0 gate, 1 up, 2 down; each D x n bf16 bit patterns,
+ *          element (d, j) at d * n + j, so column j is phi_{h,j}
+ *   bits   [3][E][n] unit bit-widths, each in {0,1,2,3,4,6,8,16}
+ *   alpha  [3][E][n] fp32 spectral energies alpha_{e,h,j}
+ *   codes  [3][E][n][I] uint16: for 0 < b < 16 the code q in [0, 2^b) of element i;
+ *          for b == 16 the fp16 bit pattern of p_hat[i]; ignored for b == 0
+ *   scale, zero  [3][E][n][I / group] fp16 bit patterns; a unit with
+ *          0 < b < 16 dequantises as p_hat[i] = scale[g] * (q[i] - zero[g]),
+ *          g = i / group; ignored for b in {0, 16}
+ */
+typedef struct bitsmoe_layer_host {
+  int32_t D, E, I, n, group;
+  const uint16_t* basis[3];
+  const uint8_t* bits;
+  const float* alpha;
+  const uint16_t* codes;
+  const uint16_t* scale;
+  const uint16_t* zero;
+} bitsmoe_layer_host;
+
+/* Writable destination of an unpack (same layout as bitsmoe_layer_host;
+ * every array allocated by the caller at its full size). */
+typedef struct bitsmoe_layer_host_out {
+  int32_t D, E, I, n, group;
+  uint16_t* basis[3];
+  uint8_t* bits;
+  float* alpha;
+  uint16_t* codes;
+  uint16_t* scale;
+  uint16_t* zero;
+} bitsmoe_layer_host_out;
+
+/* Sizes of the packed layer (bytes).  `moved_*` are the algorithmic bytes a
+ * forward must read per routed expert: codes of units with b > 0 at b bits per
+ * element, fp16 scale + zero per group of quantised units, fp32 alpha per unit
+ * with b > 0 (layout padding and index metadata not counted). */
+typedef struct bitsmoe_bytes {
+  uint64_t total;            /* device image size                               */
+  uint64_t basis;            /* 3 * D * n * 2                                   */
+  uint64_t codes_padded;     /* code streams as stored (tiles padded)           */
+  uint64_t meta;             /* unit indices, alpha, scale/zero, descriptors    */
+} bitsmoe_bytes;
+
+typedef struct bitsmoe_layer bitsmoe_layer;   /* opaque, library-owned, device-resident */
+
+/* Pack a host layer into the bucketed device layout and upload it to `device`.
+ * Allocates device memory (owned by the returned layer until bitsmoe_free),
+ * copies synchronously.  Errors: INVALID_ARG (null pointer, or a code >= 2^b in
+ * a unit of 0 < b < 16), SHAPE, UNSUPPORTED_BITS, OOM, CUDA. */
+int bitsmoe_pack(const bitsmoe_layer_host* src, int device, bitsmoe_layer** out);
+
+/* Same packing into a host blob (no GPU needed).  *blob is allocated by the
+ * library (free with bitsmoe_blob_free); *bytes is its size. */
+int bitsmoe_pack_to_host(const bitsmoe_layer_host* src, void** blob, size_t* bytes);
+void bitsmoe_blob_free(void* blob);
+
+/* Upload a blob made by bitsmoe_pack_to_host (validated on the host first). */
+int bitsmoe_load_blob(const void* blob, size_t bytes, int device, bitsmoe_layer** out);
+
+/* Inverse of packing: rebuild the host arrays bit-exactly from a blob or a
+ * device layer (dims must match; arrays preallocated by the caller).  Values
+ * not stored (codes/scale/zero of 0-bit units, scale/zero of 16-bit units) are
+ * written as 0. */
+int bitsmoe_unpack_blob(const void* blob, size_t bytes, bitsmoe_layer_host_out* dst);
+int bitsmoe_unpack(const bitsmoe_layer* layer, bitsmoe_layer_host_out* dst);
+
+/* Dims of a packed layer (D, E, I, n, group in that order). */
+int bitsmoe_layer_dims(const bitsmoe_layer* layer, int32_t dims[5]);
+int bitsmoe_layer_bytes(const bitsmoe_layer* layer, bitsmoe_bytes* out);
+/* Algorithmic bytes of expert e, per projection (out[0] gate, out[1] up,
+ * out[2] down): codes of units with b > 0 at b bits per element, fp16 scale and
+ * zero per group of the quantised units, fp32 alpha per unit with b > 0
+ * (layout padding and index metadata not counted). */
+int bitsmoe_expert_moved_bytes(const bitsmoe_layer* layer, int e, uint64_t out[3]);
+
+/* Workspace (device bytes) that bitsmoe_moe_forward needs for T tokens and
+ * top_k; 0 if the arguments are invalid. */
+size_t bitsmoe_workspace_bytes(const bitsmoe_layer* layer, int T, int top_k);
+
+/* The quantised MoE-layer forward, asynchronous on `stream`:
+ *   x       device, T x D bf16 bit patterns (row-major), 16-byte aligned
+ *   logits  device, T x E fp32 router logits (row-major), 16-byte aligned
+ *   T       tokens (T == 0 is a successful no-op)
+ *   top_k   1 .. min(E, 32): experts per token; the k largest logits are
+ *           selected (ties to the lower expert index) and weighted by a
+ *           softmax over the selected k
+ *   y       device, T x D fp32 output (row-major), 16-byte aligned, written
+ *   ws      device workspace of >= bitsmoe_workspace_bytes(layer, T, top_k)
+ *           bytes, 256-byte aligned, owned by the caller; must not be used by
+ *           another call in flight
+ * Host-side argument checks only: never allocates, never synchronises. */
+int bitsmoe_moe_forward(const void* x, const float* logits, int T, int top_k,
+                        const bitsmoe_layer* layer, float* y,
+                        void* ws, size_t ws_bytes, void* stream);
+
+/* Same forward from host buffers: copies x (T x D bf16) and logits (T x E fp32)
+ * from host memory into the workspace, runs the forward, copies y (T x D fp32)
+ * back to host memory and synchronises `stream`.  Pinned host memory gives
+ * asynchronous copies; pageable memory works but is slower. */
+int bitsmoe_moe_forward_host(const void* x_host, const float* logits_host, int T, int top_k,
+                             const bitsmoe_layer* layer, float* y_host,
+                             void* ws, size_t ws_bytes, void* stream);
+
+/* Profiling variant of bitsmoe_moe_forward (same arguments and results): the
+ * five phases run without overlap, each bracketed by CUDA events on `stream`,
+ * and the call synchronises.  phase_ms[0..4] receive the durations of
+ * routing, shared-basis projection (gate, up), gate/up factors + SwiGLU
+ * inputs, down factor + weighted expert sum, output basis. */
+int bitsmoe_profile_forward(const void* x, const float* logits, int T, int top_k,
+                            const bitsmoe_layer* layer, float* y,
+                            void* ws, size_t ws_bytes, void* stream, float phase_ms[5]);
+
+/* Synchronise `stream`, then read and clear the device status word kept in
+ * `ws`: BITSMOE_OK, or the first device-side error recorded by the last
+ * forward that used this workspace (each forward resets it when it starts). */
+int bitsmoe_last_device_status(void* ws, void* stream);
+
+/* Free a packed layer and its device memory (NULL is ignored). */
+void bitsmoe_free(bitsmoe_layer* layer);
+
+const char* bitsmoe_strerror(int code);
+/* The cudaError_t of the last BITSMOE_ERR_CUDA on this thread. */
+int bitsmoe_last_cuda_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* BITSMOE_H */

@@ -1,0 +1,289 @@
+"""Python binding of libbitsmoe, the GB300 BitsMoE quantized MoE-layer forward.
+
+Argument marshalling only: every step of the forward runs in the library's
+CUDA kernels.  The functions carry the C ABI's names (see include/bitsmoe.h);
+PyTorch is used only for device memory and streams by the convenience wrapper
+``moe_forward``.  There is no CPU fallback: if the compiled library is missing
+every entry point raises ``BitsMoEUnavailable``.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Dict, Optional
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libbitsmoe.so")
+
+OK = 0
+ERR = {
+    -1: "INVALID_ARG", -2: "SHAPE", -3: "UNSUPPORTED_BITS", -4: "WORKSPACE_TOO_SMALL",
+    -5: "ALIGNMENT", -6: "CUDA", -7: "OOM", -8: "TIMEOUT", -9: "DEVICE_BOUNDS", -10: "BLOB",
+}
+ERR_CODE = {v: k for k, v in ERR.items()}
+
+# Every C entry point declared in include/bitsmoe.h, with (restype, argtypes).
+_P = ctypes.c_void_p
+_I = ctypes.c_int
+_SZ = ctypes.c_size_t
+
+
+class _LayerHost(ctypes.Structure):
+    _fields_ = [("D", ctypes.c_int32), ("E", ctypes.c_int32), ("I", ctypes.c_int32),
+                ("n", ctypes.c_int32), ("group", ctypes.c_int32),
+                ("basis", _P * 3), ("bits", _P), ("alpha", _P), ("codes", _P),
+                ("scale", _P), ("zero", _P)]
+
+
+class _Bytes(ctypes.Structure):
+    _fields_ = [("total", ctypes.c_uint64), ("basis", ctypes.c_uint64),
+                ("codes_padded", ctypes.c_uint64), ("meta", ctypes.c_uint64)]
+
+
+SIGNATURES = {
+    "bitsmoe_pack": (_I, [ctypes.POINTER(_LayerHost), _I, ctypes.POINTER(_P)]),
+    "bitsmoe_pack_to_host": (_I, [ctypes.POINTER(_LayerHost), ctypes.POINTER(_P), ctypes.POINTER(_SZ)]),
+    "bitsmoe_blob_free": (None, [_P]),
+    "bitsmoe_load_blob": (_I, [_P, _SZ, _I, ctypes.POINTER(_P)]),
+    "bitsmoe_unpack_blob": (_I, [_P, _SZ, ctypes.POINTER(_LayerHost)]),
+    "bitsmoe_unpack": (_I, [_P, ctypes.POINTER(_LayerHost)]),
+    "bitsmoe_layer_dims": (_I, [_P, ctypes.POINTER(ctypes.c_int32)]),
+    "bitsmoe_layer_bytes": (_I, [_P, ctypes.POINTER(_Bytes)]),
+    "bitsmoe_expert_moved_bytes": (_I, [_P, _I, ctypes.POINTER(ctypes.c_uint64)]),
+    "bitsmoe_profile_forward": (_I, [_P, _P, _I, _I, _P, _P, _P, _SZ, _P, ctypes.POINTER(ctypes.c_float)]),
+    "bitsmoe_workspace_bytes": (_SZ, [_P, _I, _I]),
+    "bitsmoe_moe_forward": (_I, [_P, _P, _I, _I, _P, _P, _P, _SZ, _P]),
+    "bitsmoe_moe_forward_host": (_I, [_P, _P, _I, _I, _P, _P, _P, _SZ, _P]),
+    "bitsmoe_last_device_status": (_I, [_P, _P]),
+    "bitsmoe_free": (None, [_P]),
+    "bitsmoe_strerror": (ctypes.c_char_p, [_I]),
+    "bitsmoe_last_cuda_error": (_I, []),
+}
+
+
+class BitsMoEUnavailable(RuntimeError):
+    pass
+
+
+class BitsMoEError(RuntimeError):
+    def __init__(self, code: int, where: str = ""):
+        self.code = code
+        name = ERR.get(code, str(code))
+        extra = ""
+        if code == -6:
+            extra = f" (cudaError {_lib().bitsmoe_last_cuda_error()})"
+        super().__init__(f"{where}: BITSMOE_ERR_{name}{extra}")
+
+
+_lib_handle = None
+
+
+def _lib():
+    global _lib_handle
+    if _lib_handle is None:
+        if not os.path.exists(LIB_PATH):
+            raise BitsMoEUnavailable(
+                f"{LIB_PATH} is not built; build it with __graft_entry__.build() "
+                "(the BitsMoE forward has no CPU fallback)")
+        lib = ctypes.CDLL(LIB_PATH)
+        for name, (res, args) in SIGNATURES.items():
+            f = getattr(lib, name)
+            f.restype = res
+            f.argtypes = args
+        _lib_handle = lib
+    return _lib_handle
+
+
+def library_path() -> str:
+    _lib()
+    return LIB_PATH
+
+
+def _check(rc: int, where: str):
+    if rc != OK:
+        raise BitsMoEError(rc, where)
+
+
+def _ptr(a: np.ndarray) -> int:
+    return a.ctypes.data
+
+
+def _host_struct(layer: Dict):
+    """ctypes view of a host layer dict (see synth.make_layer); returns (struct, keepalive)."""
+    keep = {}
+    for k, dt in (("bits", np.uint8), ("alpha", np.float32), ("codes", np.uint16),
+                  ("scale", np.uint16), ("zero", np.uint16)):
+        keep[k] = np.ascontiguousarray(layer[k], dtype=dt)
+    bases = [np.ascontiguousarray(layer["basis"][h], dtype=np.uint16) for h in range(3)]
+    s = _LayerHost(int(layer["D"]), int(layer["E"]), int(layer["I"]), int(layer["n"]), int(layer["group"]))
+    s.basis = (_P * 3)(*[_ptr(b) for b in bases])
+    for k in ("bits", "alpha", "codes", "scale", "zero"):
+        setattr(s, k, _ptr(keep[k]))
+    keep["bases"] = bases
+    return s, keep
+
+
+def _empty_host(dims) -> Dict:
+    D, E, I, n, group = dims
+    ng = I // group
+    return dict(D=D, E=E, I=I, n=n, group=group,
+                basis=np.zeros((3, D, n), np.uint16), bits=np.zeros((3, E, n), np.uint8),
+                alpha=np.zeros((3, E, n), np.float32), codes=np.zeros((3, E, n, I), np.uint16),
+                scale=np.zeros((3, E, n, ng), np.uint16), zero=np.zeros((3, E, n, ng), np.uint16))
+
+
+def _out_struct(out: Dict):
+    s = _LayerHost(out["D"], out["E"], out["I"], out["n"], out["group"])
+    s.basis = (_P * 3)(*[_ptr(out["basis"][h]) for h in range(3)])
+    for k in ("bits", "alpha", "codes", "scale", "zero"):
+        setattr(s, k, _ptr(out[k]))
+    return s
+
+
+class Layer:
+    """A packed, device-resident layer (owns the library handle)."""
+
+    def __init__(self, handle: int):
+        self.handle = handle
+        dims = (ctypes.c_int32 * 5)()
+        _check(_lib().bitsmoe_layer_dims(handle, dims), "bitsmoe_layer_dims")
+        self.D, self.E, self.I, self.n, self.group = (int(v) for v in dims)
+
+    def free(self):
+        if self.handle:
+            _lib().bitsmoe_free(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass
+
+    def bytes(self) -> Dict[str, int]:
+        b = _Bytes()
+        _check(_lib().bitsmoe_layer_bytes(self.handle, ctypes.byref(b)), "bitsmoe_layer_bytes")
+        return dict(total=b.total, basis=b.basis, codes_padded=b.codes_padded, meta=b.meta)
+
+    def expert_moved_bytes(self, e: int):
+        """Algorithmic bytes of expert e per projection (gate, up, down)."""
+        v = (ctypes.c_uint64 * 3)()
+        _check(_lib().bitsmoe_expert_moved_bytes(self.handle, e, v), "bitsmoe_expert_moved_bytes")
+        return [int(a) for a in v]
+
+
+# --------------------------------------------------------------------------
+# C-ABI entry points
+# --------------------------------------------------------------------------
+def bitsmoe_pack(layer: Dict, device: int = 0) -> Layer:
+    s, keep = _host_struct(layer)
+    h = _P()
+    _check(_lib().bitsmoe_pack(ctypes.byref(s), device, ctypes.byref(h)), "bitsmoe_pack")
+    return Layer(h.value)
+
+
+def bitsmoe_pack_to_host(layer: Dict) -> np.ndarray:
+    s, keep = _host_struct(layer)
+    blob, nbytes = _P(), _SZ()
+    _check(_lib().bitsmoe_pack_to_host(ctypes.byref(s), ctypes.byref(blob), ctypes.byref(nbytes)),
+           "bitsmoe_pack_to_host")
+    try:
+        out = np.empty(nbytes.value, np.uint8)
+        ctypes.memmove(_ptr(out), blob.value, nbytes.value)
+    finally:
+        _lib().bitsmoe_blob_free(blob)
+    return out
+
+
+def bitsmoe_load_blob(blob: np.ndarray, device: int = 0) -> Layer:
+    blob = np.ascontiguousarray(blob, dtype=np.uint8)
+    h = _P()
+    _check(_lib().bitsmoe_load_blob(_ptr(blob), blob.nbytes, device, ctypes.byref(h)), "bitsmoe_load_blob")
+    return Layer(h.value)
+
+
+def bitsmoe_unpack_blob(blob: np.ndarray, dims) -> Dict:
+    blob = np.ascontiguousarray(blob, dtype=np.uint8)
+    out = _empty_host(dims)
+    s = _out_struct(out)
+    _check(_lib().bitsmoe_unpack_blob(_ptr(blob), blob.nbytes, ctypes.byref(s)), "bitsmoe_unpack_blob")
+    return out
+
+
+def bitsmoe_unpack(layer: Layer) -> Dict:
+    out = _empty_host((layer.D, layer.E, layer.I, layer.n, layer.group))
+    s = _out_struct(out)
+    _check(_lib().bitsmoe_unpack(layer.handle, ctypes.byref(s)), "bitsmoe_unpack")
+    return out
+
+
+def bitsmoe_workspace_bytes(layer: Layer, T: int, top_k: int) -> int:
+    return int(_lib().bitsmoe_workspace_bytes(layer.handle, T, top_k))
+
+
+def bitsmoe_moe_forward(x_ptr: int, logits_ptr: int, T: int, top_k: int, layer: Layer, y_ptr: int,
+                        ws_ptr: int, ws_bytes: int, stream: int = 0) -> None:
+    _check(_lib().bitsmoe_moe_forward(x_ptr, logits_ptr, T, top_k, layer.handle, y_ptr, ws_ptr,
+                                      ws_bytes, stream), "bitsmoe_moe_forward")
+
+
+def bitsmoe_moe_forward_host(x_bits: np.ndarray, logits: np.ndarray, top_k: int, layer: Layer,
+                             ws_ptr: int, ws_bytes: int, stream: int = 0,
+                             y_out: Optional[np.ndarray] = None) -> np.ndarray:
+    """Forward from host arrays (x bf16 bits T x D, logits fp32 T x E) -> y fp32 T x D."""
+    T = int(x_bits.shape[0])
+    y = y_out if y_out is not None else np.empty((T, layer.D), np.float32)
+    _check(_lib().bitsmoe_moe_forward_host(x_bits.ctypes.data, logits.ctypes.data, T, top_k, layer.handle,
+                                           y.ctypes.data, ws_ptr, ws_bytes, stream), "bitsmoe_moe_forward_host")
+    return y
+
+
+def bitsmoe_profile_forward(x_ptr: int, logits_ptr: int, T: int, top_k: int, layer: Layer, y_ptr: int,
+                            ws_ptr: int, ws_bytes: int, stream: int = 0):
+    """Forward with the five phases serialised and timed; returns their durations (ms)."""
+    ms = (ctypes.c_float * 5)()
+    _check(_lib().bitsmoe_profile_forward(x_ptr, logits_ptr, T, top_k, layer.handle, y_ptr, ws_ptr,
+                                          ws_bytes, stream, ms), "bitsmoe_profile_forward")
+    return [float(v) for v in ms]
+
+
+def bitsmoe_last_device_status(ws_ptr: int, stream: int = 0) -> int:
+    return int(_lib().bitsmoe_last_device_status(ws_ptr, stream))
+
+
+def bitsmoe_strerror(code: int) -> str:
+    return _lib().bitsmoe_strerror(code).decode()
+
+
+# --------------------------------------------------------------------------
+# torch convenience (device memory + streams only)
+# --------------------------------------------------------------------------
+class Workspace:
+    """Device workspace sized for (T, top_k) on a layer, allocated with torch."""
+
+    def __init__(self, layer: Layer, T: int, top_k: int, device=None):
+        import torch
+        self.nbytes = bitsmoe_workspace_bytes(layer, T, top_k)
+        if self.nbytes == 0:
+            raise BitsMoEError(ERR_CODE["INVALID_ARG"], "bitsmoe_workspace_bytes")
+        self.buf = torch.empty(self.nbytes + 256, dtype=torch.uint8,
+                               device=device if device is not None else f"cuda:{torch.cuda.current_device()}")
+        base = self.buf.data_ptr()
+        self.ptr = (base + 255) // 256 * 256
+
+
+def moe_forward(layer: Layer, x_bits, logits, top_k: int, ws: Optional[Workspace] = None, y=None, stream=None):
+    """y (fp32 T x D) = BitsMoE MoE-layer forward of x (int16/uint16 tensor of bf16 bits or a
+    torch.bfloat16 tensor, T x D) with router logits (fp32 T x E), all on the device."""
+    import torch
+    T = int(x_bits.shape[0])
+    if ws is None:
+        ws = Workspace(layer, T, top_k, device=x_bits.device)
+    if y is None:
+        y = torch.empty((T, layer.D), dtype=torch.float32, device=x_bits.device)
+    st = stream if stream is not None else torch.cuda.current_stream(x_bits.device)
+    bitsmoe_moe_forward(x_bits.data_ptr(), logits.data_ptr(), T, top_k, layer, y.data_ptr(),
+                        ws.ptr, ws.nbytes, st.cuda_stream)
+    return y

@@ -1,0 +1,164 @@
+"""Host-side checks of the C-ABI library (no GPU needed).
+
+* the library loads and exports every function include/bitsmoe.h declares;
+* packing into the bucketed layout and unpacking it round-trips bit-exactly,
+  for every bit-width, group size, ragged unit counts, padded rows and the
+  degenerate layers (an expert with every unit evicted, a single live unit);
+* malformed inputs and blobs are rejected with the documented error codes.
+"""
+import os
+import re
+
+import numpy as np
+import pytest
+
+import synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def bm():
+    import __graft_entry__
+    __graft_entry__.build_library()
+    import paper_2606_00079_gb300 as bm
+    return bm
+
+
+def _declared_functions():
+    src = open(os.path.join(ROOT, "include", "bitsmoe.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(bitsmoe_[a-z_]+)\s*\(", src)))
+
+
+def test_library_exports_every_declared_symbol(bm):
+    lib = bm._lib()
+    declared = _declared_functions()
+    assert len(declared) >= 15
+    for name in declared:
+        assert hasattr(lib, name), name
+    assert set(declared) == set(bm.SIGNATURES), "binding signatures differ from the header"
+
+
+def _spec(**kw):
+    base = dict(D=48, E=3, I=256, n=40, group=64, top_k=2)
+    base.update(kw)
+    return synth.scaled_spec(synth.WORKLOADS["tiny"], **base)
+
+
+def _expect_roundtrip(layer, out):
+    """Compare what is stored: every bit-width, basis, alpha of live units, codes of
+    live units, scale/zero of quantised units (evicted units unpack as zeros)."""
+    np.testing.assert_array_equal(out["basis"], layer["basis"])
+    np.testing.assert_array_equal(out["bits"], layer["bits"])
+    live = layer["bits"] > 0
+    np.testing.assert_array_equal(out["alpha"][live], layer["alpha"][live])
+    assert not out["alpha"][~live].any()
+    np.testing.assert_array_equal(out["codes"][live], layer["codes"][live])
+    assert not out["codes"][~live].any()
+    quant = live & (layer["bits"] < 16)
+    np.testing.assert_array_equal(out["scale"][quant], layer["scale"][quant])
+    np.testing.assert_array_equal(out["zero"][quant], layer["zero"][quant])
+    assert not out["scale"][~quant].any()
+
+
+ALL_BITS = {0: 0.1, 1: 0.15, 2: 0.2, 3: 0.15, 4: 0.1, 6: 0.1, 8: 0.1, 16: 0.1}
+
+
+@pytest.mark.parametrize("group,I", [(32, 96), (64, 256), (128, 384), (256, 512)])
+def test_pack_roundtrip_all_bit_widths(bm, group, I):
+    spec = _spec(group=group, I=I)
+    layer = synth.make_layer(spec, seed=group, bits_dist=ALL_BITS)
+    blob = bm.bitsmoe_pack_to_host(layer)
+    out = bm.bitsmoe_unpack_blob(blob, (spec.D, spec.E, spec.I, spec.n, spec.group))
+    _expect_roundtrip(layer, out)
+
+
+@pytest.mark.parametrize("b", [1, 2, 3, 4, 6, 8, 16])
+def test_pack_roundtrip_uniform_and_ragged(bm, b):
+    # n = 37 units: ragged against every tile width (2, 4, 8, 16, 32)
+    spec = _spec(n=37, D=40)
+    layer = synth.make_layer(spec, seed=b, bits_dist={b: 1.0})
+    out = bm.bitsmoe_unpack_blob(bm.bitsmoe_pack_to_host(layer), (spec.D, spec.E, spec.I, spec.n, spec.group))
+    _expect_roundtrip(layer, out)
+
+
+def test_pack_roundtrip_degenerate_layers(bm):
+    spec = _spec()
+    layer = synth.make_layer(spec, seed=1, bits_dist=ALL_BITS)
+    layer["bits"][0, 1, :] = 0            # gate of expert 1: every unit evicted
+    layer["bits"][2, 0, :] = 0            # down of expert 0: a single live unit
+    layer["bits"][2, 0, 17] = 3
+    layer["codes"][2, 0, 17] = np.arange(spec.I) % 8
+    layer["scale"][2, 0, 17] = 0x2C00
+    layer["zero"][2, 0, 17] = 0x4300
+    layer["bits"][:, 2, :] = 0            # expert 2 entirely evicted
+    out = bm.bitsmoe_unpack_blob(bm.bitsmoe_pack_to_host(layer), (spec.D, spec.E, spec.I, spec.n, spec.group))
+    _expect_roundtrip(layer, out)
+
+
+def test_pack_roundtrip_tiny_workload(bm):
+    spec = synth.WORKLOADS["tiny"]
+    layer = synth.make_layer(spec, seed=0)
+    blob = bm.bitsmoe_pack_to_host(layer)
+    out = bm.bitsmoe_unpack_blob(blob, (spec.D, spec.E, spec.I, spec.n, spec.group))
+    _expect_roundtrip(layer, out)
+    # packing is deterministic
+    np.testing.assert_array_equal(bm.bitsmoe_pack_to_host(layer), blob)
+
+
+def test_invalid_inputs_rejected(bm):
+    spec = _spec()
+    layer = synth.make_layer(spec, seed=2)
+    bad = dict(layer)
+    bad["bits"] = layer["bits"].copy()
+    bad["bits"][1, 0, 3] = 5
+    with pytest.raises(bm.BitsMoEError) as ei:
+        bm.bitsmoe_pack_to_host(bad)
+    assert ei.value.code == bm.ERR_CODE["UNSUPPORTED_BITS"]
+    bad = dict(layer)
+    bad["codes"] = layer["codes"].copy()
+    j = int(np.argmax(layer["bits"][0, 0] == 2))
+    assert layer["bits"][0, 0, j] == 2
+    bad["codes"][0, 0, j, 5] = 4               # code out of range for a 2-bit unit
+    with pytest.raises(bm.BitsMoEError) as ei:
+        bm.bitsmoe_pack_to_host(bad)
+    assert ei.value.code == bm.ERR_CODE["INVALID_ARG"]
+    bad = dict(layer, group=48)
+    with pytest.raises(bm.BitsMoEError) as ei:
+        bm.bitsmoe_pack_to_host(bad)
+    assert ei.value.code == bm.ERR_CODE["SHAPE"]
+    bad = dict(layer, I=250)                 # not a multiple of the group
+    with pytest.raises(bm.BitsMoEError) as ei:
+        bm.bitsmoe_pack_to_host(bad)
+    assert ei.value.code == bm.ERR_CODE["SHAPE"]
+
+
+def test_malformed_blob_rejected(bm):
+    spec = _spec()
+    layer = synth.make_layer(spec, seed=3)
+    blob = bm.bitsmoe_pack_to_host(layer)
+    dims = (spec.D, spec.E, spec.I, spec.n, spec.group)
+    for mutate in ("magic", "truncate", "offset", "unit"):
+        b = blob.copy()
+        if mutate == "magic":
+            b[0] ^= 0xFF
+        elif mutate == "truncate":
+            b = b[:-256]
+        elif mutate == "offset":
+            # ImageHeader: 2 u32 + 14 i32 = 64 bytes, then total_bytes, off_desc, ...
+            off = np.frombuffer(b[72:80].tobytes(), np.uint64)[0]
+            b[72:80] = np.frombuffer(np.uint64(off + 10 ** 9).tobytes(), np.uint8)
+        else:
+            # first unit index of the first (h, e) block: set it out of range
+            desc_off = int(np.frombuffer(b[72:80].tobytes(), np.uint64)[0])
+            unit_off = int(np.frombuffer(b[desc_off + 48:desc_off + 56].tobytes(), np.uint64)[0])
+            b[unit_off:unit_off + 4] = np.frombuffer(np.int32(10 ** 6).tobytes(), np.uint8)
+        with pytest.raises(bm.BitsMoEError) as ei:
+            bm.bitsmoe_unpack_blob(b, dims)
+        assert ei.value.code == bm.ERR_CODE["BLOB"], mutate
+
+
+def test_strerror(bm):
+    assert bm.bitsmoe_strerror(0) == "ok"
+    assert "workspace" in bm.bitsmoe_strerror(-4)
