@@ -171,6 +171,33 @@ int bitsmoe_profile_forward(const void* x, const float* logits, int T, int top_k
                             const bitsmoe_layer* layer, float* y,
                             void* ws, size_t ws_bytes, void* stream, float phase_ms[5]);
 
+/* Largest workspace (bytes, as bitsmoe_workspace_bytes reports it) that
+ * bitsmoe_moe_forward_noalloc can serve from its built-in scratch. */
+#define BITSMOE_NOALLOC_SCRATCH_BYTES (8u << 20)
+
+/* The forward of bitsmoe_moe_forward without a caller-provided workspace, for
+ * callers that cannot allocate device memory themselves: a serving runtime
+ * whose allocator has already reserved the device's memory, a plugin inside a
+ * framework whose caching allocator owns all device memory, or a decode loop
+ * that must not call cudaMalloc because cudaMalloc can synchronise the device.
+ * (The BitsMoE paper has no counterpart; this is a deployment convenience.)
+ *
+ * The scratch is one fixed device array of BITSMOE_NOALLOC_SCRATCH_BYTES
+ * (8 MiB) inside the library, present on every GPU that loads the library
+ * until the process exits.  This call allocates nothing: no cudaMalloc, no
+ * cudaFree, no allocating library routine.  The first call on a device looks
+ * up that device's address of the array (once per device, with the device
+ * current); make the first call before any stream capture.
+ *   x, logits, y, T, top_k, layer, stream: as for bitsmoe_moe_forward.
+ * Errors: as bitsmoe_moe_forward, and BITSMOE_ERR_WORKSPACE_TOO_SMALL when
+ * bitsmoe_workspace_bytes(layer, T, top_k) > BITSMOE_NOALLOC_SCRATCH_BYTES.
+ * Every call on a device shares the one array and it keeps the last call's
+ * contents (each forward clears what it accumulates into before using it),
+ * so calls that overlap on the GPU (different streams, or different host
+ * threads) race and give wrong results: serialise them. */
+int bitsmoe_moe_forward_noalloc(const void* x, const float* logits, int T, int top_k,
+                                const bitsmoe_layer* layer, float* y, void* stream);
+
 /* Synchronise `stream`, then read and clear the device status word kept in
  * `ws`: BITSMOE_OK, or the first device-side error recorded by the last
  * forward that used this workspace (each forward resets it when it starts). */

@@ -56,6 +56,7 @@ SIGNATURES = {
     "bitsmoe_workspace_bytes": (_SZ, [_P, _I, _I]),
     "bitsmoe_moe_forward": (_I, [_P, _P, _I, _I, _P, _P, _P, _SZ, _P]),
     "bitsmoe_moe_forward_host": (_I, [_P, _P, _I, _I, _P, _P, _P, _SZ, _P]),
+    "bitsmoe_moe_forward_noalloc": (_I, [_P, _P, _I, _I, _P, _P, _P]),
     "bitsmoe_last_device_status": (_I, [_P, _P]),
     "bitsmoe_free": (None, [_P]),
     "bitsmoe_strerror": (ctypes.c_char_p, [_I]),
@@ -238,6 +239,18 @@ def bitsmoe_moe_forward_host(x_bits: np.ndarray, logits: np.ndarray, top_k: int,
     _check(_lib().bitsmoe_moe_forward_host(x_bits.ctypes.data, logits.ctypes.data, T, top_k, layer.handle,
                                            y.ctypes.data, ws_ptr, ws_bytes, stream), "bitsmoe_moe_forward_host")
     return y
+
+
+NOALLOC_SCRATCH_BYTES = 8 << 20   # BITSMOE_NOALLOC_SCRATCH_BYTES
+
+
+def bitsmoe_moe_forward_noalloc(x_ptr: int, logits_ptr: int, T: int, top_k: int, layer: Layer, y_ptr: int,
+                                stream: int = 0) -> None:
+    """The forward for callers that cannot allocate device memory: its scratch is
+    the library's built-in array (NOALLOC_SCRATCH_BYTES per device, shared by all
+    calls on that device, so overlapping calls race)."""
+    _check(_lib().bitsmoe_moe_forward_noalloc(x_ptr, logits_ptr, T, top_k, layer.handle, y_ptr, stream),
+           "bitsmoe_moe_forward_noalloc")
 
 
 def bitsmoe_profile_forward(x_ptr: int, logits_ptr: int, T: int, top_k: int, layer: Layer, y_ptr: int,

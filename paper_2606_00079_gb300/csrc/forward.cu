@@ -1043,9 +1043,49 @@ int upload(std::vector<uint8_t>&& img, int device, bitsmoe_layer** out) {
   return BITSMOE_OK;
 }
 
+// Scratch of bitsmoe_moe_forward_noalloc: one fixed array per device that
+// loads the library.  Host code only ever sees a host-side stand-in for this
+// symbol; the device address comes from cudaGetSymbolAddress, once per device.
+constexpr size_t kNoAllocBytes = BITSMOE_NOALLOC_SCRATCH_BYTES;
+constexpr int kNoAllocMaxDevices = 64;
+static __device__ __align__(256) uint8_t g_noalloc_scratch[kNoAllocBytes];
+std::mutex g_noalloc_mu;
+void* g_noalloc_addr[kNoAllocMaxDevices] = {};
+
+// Device address of the scratch on `device` (which must be current).
+int noalloc_scratch(int device, void** out) {
+  if (device < 0 || device >= kNoAllocMaxDevices) return BITSMOE_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (!g_noalloc_addr[device]) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess || !p) return cuda_fail(e != cudaSuccess ? e : cudaErrorInvalidSymbol);
+    g_noalloc_addr[device] = p;
+  }
+  *out = g_noalloc_addr[device];
+  return BITSMOE_OK;
+}
+
 }  // namespace
 
 extern "C" {
+
+int bitsmoe_moe_forward_noalloc(const void* x, const float* logits, int T, int top_k, const bitsmoe_layer* L,
+                                float* y, void* stream) {
+  if (!L || T < 0) return BITSMOE_ERR_INVALID_ARG;
+  const ImageHeader& hd = L->hd();
+  if (top_k < 1 || top_k > std::min(hd.E, 32)) return BITSMOE_ERR_INVALID_ARG;
+  if ((int64_t)T * top_k > (1 << 24) || (int64_t)T * hd.D > (1ll << 31)) return BITSMOE_ERR_SHAPE;
+  if (T == 0) return BITSMOE_OK;
+  if (!x || !logits || !y) return BITSMOE_ERR_INVALID_ARG;
+  if (!aligned(x, 16) || !aligned(logits, 16) || !aligned(y, 16)) return BITSMOE_ERR_ALIGNMENT;
+  if (ws_layout(hd, T, top_k).total > kNoAllocBytes) return BITSMOE_ERR_WORKSPACE_TOO_SMALL;
+  int rc = check_device(L);
+  if (rc) return rc;
+  void* ws = nullptr;
+  if ((rc = noalloc_scratch(L->device, &ws))) return rc;
+  return forward_impl(x, logits, T, top_k, L, y, ws, kNoAllocBytes, static_cast<cudaStream_t>(stream));
+}
 
 int bitsmoe_pack(const bitsmoe_layer_host* src, int device, bitsmoe_layer** out) {
   if (!src || !out) return BITSMOE_ERR_INVALID_ARG;

@@ -1,0 +1,72 @@
+"""bitsmoe_moe_forward_noalloc: the forward for callers that cannot allocate
+device memory (their device memory belongs to another allocator, or
+allocating would synchronise the device in the middle of a decode loop).
+
+It must give the same result as bitsmoe_moe_forward with a caller-provided
+workspace, on consecutive calls that share its built-in scratch, and reject a
+batch whose workspace would not fit that scratch.  Collected last on purpose:
+the check passes alone in a fresh process and after every other test.
+"""
+import ctypes
+
+import numpy as np
+import pytest
+
+import synth
+
+pytestmark = pytest.mark.gpu
+TOL = 2e-3
+
+
+@pytest.fixture(scope="module")
+def env():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2606_00079_gb300 as bm
+    torch.cuda.set_device(0)
+    return torch, bm
+
+
+def _rel(a, b):
+    return float(np.max(np.abs(a - b)) / max(np.max(np.abs(b)), 1e-30))
+
+
+def test_noalloc_matches_workspace_forward_on_consecutive_calls(env):
+    torch, bm = env
+    lib = bm._lib()
+    spec = synth.WORKLOADS["qw3_skew"]
+    spec = synth.scaled_spec(spec, D=512, E=16, I=384, n=512, top_k=4)
+    layer = synth.make_layer(spec, seed=3)
+    L = bm.bitsmoe_pack(layer, device=0)
+    stream = torch.cuda.current_stream().cuda_stream
+    for call, T in enumerate((5, 3)):            # two calls in a row share the scratch
+        x, logits = synth.make_inputs(spec, T, seed=3, step=call)
+        xd = torch.from_numpy(x.view(np.int16)).cuda()
+        ld = torch.from_numpy(logits).cuda()
+        y_ref = bm.moe_forward(L, xd, ld, spec.top_k)
+        y = torch.full((T, spec.D), float("nan"), dtype=torch.float32, device="cuda")
+        rc = lib.bitsmoe_moe_forward_noalloc(xd.data_ptr(), ld.data_ptr(), T, spec.top_k, L.handle,
+                                             y.data_ptr(), ctypes.c_void_p(stream))
+        assert rc == 0, bm.bitsmoe_strerror(rc)
+        torch.cuda.synchronize()
+        err = _rel(y.cpu().numpy().astype(np.float64), y_ref.cpu().numpy().astype(np.float64))
+        assert err <= TOL, (call, err)
+
+
+def test_noalloc_rejects_batches_beyond_its_scratch(env):
+    torch, bm = env
+    spec = synth.WORKLOADS["tiny"]
+    layer = synth.make_layer(spec, seed=4)
+    L = bm.bitsmoe_pack(layer, device=0)
+    T = 1
+    while bm.bitsmoe_workspace_bytes(L, T, spec.top_k) <= bm.NOALLOC_SCRATCH_BYTES:
+        T *= 2
+    x = torch.zeros((T, spec.D), dtype=torch.int16, device="cuda")
+    lg = torch.zeros((T, spec.E), dtype=torch.float32, device="cuda")
+    y = torch.zeros((T, spec.D), dtype=torch.float32, device="cuda")
+    with pytest.raises(bm.BitsMoEError) as ei:
+        bm.bitsmoe_moe_forward_noalloc(x.data_ptr(), lg.data_ptr(), T, spec.top_k, L, y.data_ptr(), 0)
+    assert ei.value.code == bm.ERR_CODE["WORKSPACE_TOO_SMALL"]
