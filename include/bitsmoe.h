@@ -141,7 +141,7 @@ size_t bitsmoe_workspace_bytes(const bitsmoe_layer* layer, int T, int top_k);
 /* The quantised MoE-layer forward, asynchronous on `stream`:
  *   x       device, T x D bf16 bit patterns (row-major), 16-byte aligned
  *   logits  device, T x E fp32 router logits (row-major), 16-byte aligned
- *   T       tokens (T == 0 is a successful no-op)
+ *   T       tokens (T == 0 is a successful no-op; T * top_k <= 24576)
  *   top_k   1 .. min(E, 32): experts per token; the k largest logits are
  *           selected (ties to the lower expert index) and weighted by a
  *           softmax over the selected k

@@ -5,8 +5,9 @@
 //   [ImageHeader][ExpertDesc 3 x E][K2 segment table 2 x E x (nseg+1)]
 //   [basis_in  bf16 [2][n][D_pad]]  row j of projection h = phi_{h,j}  (gate, up)
 //   [basis_out bf16 [D][n_pad]]     row d = Phi_dn[d, :]
+//   [gate/up item table ItemRec 2 x E x nseg]
 //   per (h, e), contiguous: [unit index int32 [nslots]][alpha f32 [nslots]]
-//                           [scale/zero half2 per bucket [NG][nslots_b]][code stream]
+//                           [scale/zero half2 [NG][nslots] over all slots][code stream]
 //
 // Units of one (h, e) are bucketed by bit-width b in {1,2,3,4,6,8,16} (0-bit
 // units are dropped: they contribute nothing and move no bytes), stable in j.
@@ -21,7 +22,7 @@
 //     format), chunk 2 = high 1-bit plane of units 0-31 (1-bit format).
 //   b = 6: U = 16; chunks 0,1 = low 4-bit plane of units 0-7 / 8-15, chunk 2 =
 //     high 2-bit plane of units 0-15.
-//   b = 16: U = 2; word w = fp16(unit 0, row w) | fp16(unit 1, row w) << 16.
+//   b = 16: U = 4; chunk c, word w = fp16(unit 2c, row w) | fp16(unit 2c+1, row w) << 16.
 //   Stream order: [row block][bucket][tile][chunk][lane] x 16 bytes.
 //
 // down ("unit-lane" layout, UL): a lane owns one unit (slot) of a 32-slot
@@ -33,6 +34,9 @@
 //   b = 6: chunks 0..3 = low 4-bit plane rows 32c ..; chunks 4,5 = high 2-bit plane rows 64(c-4) ..
 //   b = 16: chunk c = rows 8c .. 8c+7, word w = fp16(row 2w) | fp16(row 2w+1) << 16.
 //   Stream order: [bucket][tile][row block][chunk][lane] x 16 bytes.
+//
+// Every tile holds a multiple of 4 units, so every slot range of a bucket, a
+// tile or a gate/up item starts on a 16-byte boundary of the slot arrays.
 //
 // Padding: slots beyond a bucket's unit count have alpha 0 and codes 0;
 // rows beyond I (up to I_pad) have code 0 and scale/zero 0, so padded
@@ -52,7 +56,7 @@
 namespace bmoe {
 
 constexpr uint32_t kMagic = 0x454F4D42u;   // "BMOE"
-constexpr uint32_t kVersion = 1;
+constexpr uint32_t kVersion = 2;
 constexpr int kNumBk = 7;
 constexpr int kRows = 128;                 // rows per row block
 constexpr int kChunkBytes = 512;           // one warp-wide 16-byte-per-lane load
@@ -65,9 +69,9 @@ __host__ __device__ constexpr int bk_of_bits(int b) {
 }
 // gate/up tiles: units per tile and 16-byte chunks per lane per tile
 __host__ __device__ constexpr int rl_units(int b) {
-  return b == 1 ? 32 : b == 2 ? 16 : b == 3 ? 32 : b == 4 ? 8 : b == 6 ? 16 : b == 8 ? 4 : 2;
+  return b == 1 ? 32 : b == 2 ? 16 : b == 3 ? 32 : b == 4 ? 8 : b == 6 ? 16 : 4;
 }
-__host__ __device__ constexpr int rl_chunks(int b) { return (b == 3 || b == 6) ? 3 : 1; }
+__host__ __device__ constexpr int rl_chunks(int b) { return (b == 3 || b == 6) ? 3 : b == 16 ? 2 : 1; }
 // down tiles: 32 units, chunks per lane per row block
 __host__ __device__ constexpr int ul_chunks(int b) { return b; }
 
@@ -79,7 +83,7 @@ struct BucketDesc {
   int32_t slot0;      // first slot of this bucket in the (h,e) slot arrays
   int32_t tile0;      // first flat tile index of this bucket within (h,e)
   uint64_t code_off;  // RL: byte offset inside one row-block stream; UL: inside the (h,e) stream
-  uint64_t sz_off;    // image offset of half2 [NG][nslots] scale/zero (0 when b == 16)
+  uint64_t sz_off;    // image offset of this bucket's column 0 in the (h,e) scale/zero matrix
 };
 
 struct ExpertDesc {
@@ -93,9 +97,27 @@ struct ExpertDesc {
   uint64_t rb_stride; // RL: bytes per row block (stream = NRB * rb_stride); UL: stream bytes
   uint64_t unit_off;  // image offset of int32 [nslots]
   uint64_t alpha_off; // image offset of float [nslots]
+  uint64_t sz_off;    // image offset of half2 (scale | zero << 16) [NG][nslots]; row stride nslots
   uint64_t moved;     // algorithmic bytes of this (h,e)
   BucketDesc bk[kNumBk];
 };
+
+// One gate/up work item: a segment of consecutive tiles of one (h, e) inside a
+// row block.  Its code bytes are one contiguous run of the row-block stream and
+// its slots one contiguous run of the slot arrays; its tiles cover nr
+// consecutive buckets.
+struct ItemRec {
+  uint32_t byte0;     // first code byte inside the row-block stream
+  uint32_t bytes;     // code bytes (16-byte multiple)
+  uint32_t slot0;     // first slot (multiple of 4)
+  uint16_t nslot;     // slots (multiple of 4)
+  uint8_t nr;         // buckets touched (0: empty item)
+  uint8_t bk0;        // index of the first one in ExpertDesc::bk
+  uint8_t bits[kNumBk + 1];
+  uint16_t ntl[kNumBk + 1];   // tiles per touched bucket
+  uint32_t pad_[2];
+};
+static_assert(sizeof(ItemRec) == 48, "ItemRec layout");
 
 struct ImageHeader {
   uint32_t magic, version;
@@ -112,6 +134,7 @@ struct ImageHeader {
   uint64_t off_basis_out; // bf16 [D][n_pad]
   uint64_t codes_bytes;   // code streams as stored
   uint64_t meta_bytes;    // unit/alpha/scale-zero arrays
+  uint64_t off_items;     // ItemRec [2][E][nseg]
 };
 
 inline uint64_t align_up(uint64_t v, uint64_t a) { return (v + a - 1) / a * a; }

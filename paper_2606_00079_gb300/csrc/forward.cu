@@ -43,6 +43,8 @@ struct bitsmoe_layer {
   uint8_t* d_img;
   uint64_t bytes;
   std::vector<uint8_t> meta;   // host copy of header + descriptors + segment table
+  int seg_bytes = 0;           // largest gate/up item: code bytes inside one row block
+  int ul_max_chunks = 1;       // largest 16-byte chunks per row block of any down unit
   const ImageHeader& hd() const { return *reinterpret_cast<const ImageHeader*>(meta.data()); }
   const ExpertDesc* desc() const {
     return reinterpret_cast<const ExpertDesc*>(meta.data() + hd().off_desc);
@@ -73,12 +75,16 @@ struct Fwd {
   const uint8_t* img;
   const ExpertDesc* desc;
   const int32_t* seg;
+  const ItemRec* items;
   const uint16_t* basis_in;
   const uint16_t* basis_out;
   int D, E, I, n, group, D_pad, n_pad, I_pad, NRB, NG, nseg, ul_max_tiles;
   int T, k, P;
   int s16;          // K2 smem row stride (int16 elements)
   int rbc;          // K3 row blocks per block
+  int decode;       // small-batch mode: routing computed in each kernel, prologue staging
+  int seg_bytes;    // largest gate/up item (bytes of codes in one row block)
+  int ul_bytes;     // largest down item (bytes of one tile over rbc row blocks)
   const uint16_t* x;
   const float* logits;
   float* y;
@@ -125,6 +131,56 @@ __device__ __forceinline__ void red_add_v4(float* addr, float a, float b, float 
   asm volatile("red.global.add.v4.f32 [%0], {%1,%2,%3,%4};" ::"l"(addr), "f"(a), "f"(b), "f"(c), "f"(d)
                : "memory");
 }
+__device__ __forceinline__ uint32_t smem_u32(const void* ptr) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(ptr));
+}
+__device__ __forceinline__ uint4 lds128(const void* p) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(smem_u32(p)));
+  return v;
+}
+template <bool SH>
+__device__ __forceinline__ uint4 ld128(const uint8_t* p) {
+  if (SH) return lds128(p);
+  return ldg_stream(p);
+}
+// mbarrier + bulk copy (global -> shared, completion counted in bytes on the mbarrier)
+__device__ __forceinline__ void mbar_init(uint64_t* bar) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(bar)) : "memory");
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+               ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile("{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+               : "=r"(ok) : "r"(smem_u32(bar)), "r"(parity) : "memory");
+  return ok != 0;
+}
+// Bounded wait on an mbarrier phase (about one second of SM clock at most).
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity))
+    if (clock64() - t0 > (2ll << 30)) return false;
+  return true;
+}
+// Copy `bytes` (16-byte multiple, 16-byte aligned ends) to shared memory on one
+// mbarrier; called by one lane.
+__device__ __forceinline__ void stage_bytes(void* dst, const uint8_t* src, uint32_t bytes, uint64_t* bar) {
+  mbar_init(bar);
+  mbar_expect_tx(bar, bytes);
+  uint32_t o = 0;
+  while (o < bytes) {
+    const uint32_t c = bytes - o < 32768u ? bytes - o : 32768u;
+    bulk_g2s(static_cast<uint8_t*>(dst) + o, src + o, c, bar);
+    o += c;
+  }
+}
 __device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 __device__ __forceinline__ float f16lo(uint32_t w) {
@@ -151,21 +207,135 @@ __device__ __forceinline__ uint32_t order_key(float f) {
 }
 
 // ---------------------------------------------------------------------------
+// Routing of all T tokens by one block into shared memory (small batches):
+// keys[T*E] | pe[P] | pw[P] | cnt[E] | start[E+1] | act[E+1] | plist[P].
+// Same rule as k_router.  Contains __syncthreads (call from the whole block).
+// ---------------------------------------------------------------------------
+__host__ __device__ constexpr int route_words(int T, int E, int P) { return T * E + 3 * P + 3 * E + 3; }
+
+struct RouteView {
+  const int* pe;
+  const float* pw;
+  const int* cnt;
+  const int* start;
+  const int* act;
+  const int* plist;
+};
+
+__device__ RouteView route_block(const Fwd& p, uint32_t* sm) {
+  const int E = p.E, k = p.k, T = p.T, P = p.P, tid = threadIdx.x, nt = blockDim.x;
+  uint32_t* keys = sm;
+  int* pe = reinterpret_cast<int*>(keys + T * E);
+  float* pw = reinterpret_cast<float*>(pe + P);
+  int* cnt = reinterpret_cast<int*>(pw + P);
+  int* start = cnt + E;
+  int* act = start + E + 1;
+  int* plist = act + E + 1;
+  for (int i = tid; i < T * E; i += nt) keys[i] = order_key(p.logits[i]);
+  for (int i = tid; i < E; i += nt) cnt[i] = 0;
+  __syncthreads();
+  // rank of each logit in its token's row (ties to the lower index)
+  for (int i = tid; i < T * E; i += nt) {
+    const int t = i / E, e = i - t * E;
+    const uint32_t key = keys[i];
+    const uint32_t* row = keys + t * E;
+    int rank = 0;
+    if ((E & 3) == 0 && ((t * E) & 3) == 0) {
+      const uint4* r4 = reinterpret_cast<const uint4*>(row);
+#pragma unroll 4
+      for (int f4 = 0; f4 < (E >> 2); ++f4) {
+        const uint4 o = r4[f4];
+        const int f = f4 << 2;
+        rank += (o.x > key) | ((o.x == key) & (f < e));
+        rank += (o.y > key) | ((o.y == key) & (f + 1 < e));
+        rank += (o.z > key) | ((o.z == key) & (f + 2 < e));
+        rank += (o.w > key) | ((o.w == key) & (f + 3 < e));
+      }
+    } else {
+      for (int f = 0; f < E; ++f) {
+        const uint32_t o = row[f];
+        rank += (o > key) | ((o == key) & (f < e));
+      }
+    }
+    if (rank < k) {
+      pe[t * k + rank] = e;
+      pw[t * k + rank] = p.logits[i];
+    }
+  }
+  __syncthreads();
+  for (int t = tid; t < T; t += nt) {
+    float* w = pw + t * k;
+    const float m = w[0];
+    float sum = 0.f;
+    for (int r = 0; r < k; ++r) sum += expf(w[r] - m);
+    const float inv = 1.f / sum;
+    for (int r = 0; r < k; ++r) w[r] = expf(w[r] - m) * inv;
+  }
+  for (int q = tid; q < P; q += nt) atomicAdd(&cnt[pe[q]], 1);
+  __syncthreads();
+  if (tid < 32) {   // exclusive scans of counts and of "routed" flags, one warp
+    const int lane = tid, per = (E + 31) >> 5, e0 = min(E, lane * per), e1 = min(E, e0 + per);
+    int c = 0, na = 0;
+    for (int e = e0; e < e1; ++e) {
+      c += cnt[e];
+      na += cnt[e] > 0;
+    }
+    int ci = c, ai = na;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int vc = __shfl_up_sync(0xFFFFFFFFu, ci, o), va = __shfl_up_sync(0xFFFFFFFFu, ai, o);
+      if (lane >= o) {
+        ci += vc;
+        ai += va;
+      }
+    }
+    int run = ci - c, ra = ai - na;
+    for (int e = e0; e < e1; ++e) {
+      start[e] = run;
+      run += cnt[e];
+      if (cnt[e] > 0) act[1 + ra++] = e;
+    }
+    if (lane == 31) {
+      start[E] = ci;
+      act[0] = ai;
+    }
+  }
+  __syncthreads();
+  for (int q = tid; q < P; q += nt) {   // stable order: pairs of one expert by increasing q
+    const int ex = pe[q];
+    int r = 0;
+    for (int q2 = 0; q2 < q; ++q2) r += pe[q2] == ex;
+    plist[start[ex] + r] = q;
+  }
+  __syncthreads();
+  return RouteView{pe, pw, cnt, start, act, plist};
+}
+
+// ---------------------------------------------------------------------------
 // K0: routing.  k largest logits per token (ties to the lower expert index),
 // gate weights = softmax over the selected k, then a stable grouping of the
 // (token, slot) pairs p = t * k + slot by expert.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(1024) k_router(Fwd p) {
   pdl_trigger();
+  // shared: keys [tpb][E] | pair expert [P] | pair logit/weight [P] | count [E] | start [E+1]
   extern __shared__ uint32_t keys[];
   const int E = p.E, k = p.k, T = p.T, P = p.P;
   const int tid = threadIdx.x;
-  if (tid == 0) *p.status = 0;
   const int tpb = max(1, (int)blockDim.x / E);
+  int* s_pe = reinterpret_cast<int*>(keys + tpb * E);
+  float* s_pw = reinterpret_cast<float*>(s_pe + P);
+  int* s_cnt = reinterpret_cast<int*>(s_pw + P);
+  int* s_start = s_cnt + E;
+  if (tid == 0) *p.status = 0;
   for (int t0 = 0; t0 < T; t0 += tpb) {
     const int tt = tid / E, e = tid - tt * E, t = t0 + tt;
     const bool valid = tt < tpb && t < T;
-    if (valid) keys[tt * E + e] = order_key(p.logits[(size_t)t * E + e]);
+    float lg = 0.f;
+    if (valid) {
+      lg = p.logits[(size_t)t * E + e];
+      keys[tt * E + e] = order_key(lg);
+    }
     __syncthreads();
     if (valid) {
       const uint32_t key = keys[tt * E + e];
@@ -176,43 +346,50 @@ __global__ void __launch_bounds__(1024) k_router(Fwd p) {
         rank += (o > key) | ((o == key) & (f < e));
       }
       if (rank < k) {
-        p.pair_expert[t * k + rank] = e;
-        p.pair_weight[t * k + rank] = p.logits[(size_t)t * E + e];
+        s_pe[t * k + rank] = e;
+        s_pw[t * k + rank] = lg;
       }
     }
     __syncthreads();
   }
   for (int t = tid; t < T; t += blockDim.x) {
-    float* w = p.pair_weight + (size_t)t * k;
+    float* w = s_pw + (size_t)t * k;
     const float m = w[0];
     float sum = 0.f;
     for (int r = 0; r < k; ++r) sum += expf(w[r] - m);
     const float inv = 1.f / sum;
-    for (int r = 0; r < k; ++r) w[r] = expf(w[r] - m) * inv;
+    for (int r = 0; r < k; ++r) {
+      const float v = expf(w[r] - m) * inv;
+      p.pair_weight[t * k + r] = v;
+      p.pair_expert[t * k + r] = s_pe[t * k + r];
+    }
   }
-  __syncthreads();
   const int warp = tid >> 5, lane = tid & 31, nw = blockDim.x >> 5;
   for (int e = warp; e < E; e += nw) {
     int c = 0;
     for (int q0 = 0; q0 < P; q0 += 32) {
       const int q = q0 + lane;
-      c += __popc(__ballot_sync(0xFFFFFFFFu, q < P && p.pair_expert[q] == e));
+      c += __popc(__ballot_sync(0xFFFFFFFFu, q < P && s_pe[q] == e));
     }
-    if (lane == 0) p.expert_count[e] = c;
+    if (lane == 0) s_cnt[e] = c;
   }
   __syncthreads();
   if (warp == 0) {
     int run = 0, act = 0;
     for (int e0 = 0; e0 < E; e0 += 32) {
       const int e = e0 + lane;
-      const int c = e < E ? p.expert_count[e] : 0;
+      const int c = e < E ? s_cnt[e] : 0;
       int incl = c;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
         const int v = __shfl_up_sync(0xFFFFFFFFu, incl, o);
         if (lane >= o) incl += v;
       }
-      if (e < E) p.expert_start[e] = run + incl - c;
+      if (e < E) {
+        s_start[e] = run + incl - c;
+        p.expert_start[e] = run + incl - c;
+        p.expert_count[e] = c;
+      }
       const unsigned nz = __ballot_sync(0xFFFFFFFFu, c > 0);
       if (c > 0) p.active[1 + act + __popc(nz & ((1u << lane) - 1u))] = e;
       act += __popc(nz);
@@ -225,10 +402,10 @@ __global__ void __launch_bounds__(1024) k_router(Fwd p) {
   }
   __syncthreads();
   for (int e = warp; e < E; e += nw) {
-    int base = p.expert_start[e];
+    int base = s_start[e];
     for (int q0 = 0; q0 < P; q0 += 32) {
       const int q = q0 + lane;
-      const bool m = q < P && p.pair_expert[q] == e;
+      const bool m = q < P && s_pe[q] == e;
       const unsigned b = __ballot_sync(0xFFFFFFFFu, m);
       if (m) p.pair_list[base + __popc(b & ((1u << lane) - 1u))] = q;
       base += __popc(b);
@@ -238,28 +415,44 @@ __global__ void __launch_bounds__(1024) k_router(Fwd p) {
 
 // ---------------------------------------------------------------------------
 // L2 prefetch of what the later phases read: gate/up then down factors of the
-// routed experts, then Phi_dn (warp 0 of every block, 16 KB pieces).
+// routed experts, then Phi_dn.  Range r goes to block r % gridDim (warp 0);
+// its 32 lanes split it into 16-byte-aligned pieces.
 // ---------------------------------------------------------------------------
+__device__ __forceinline__ void prefetch_range(const uint8_t* base, uint64_t beg, uint64_t end, int lane) {
+  uint64_t piece = (((end - beg) + 31) / 32 + 15) & ~15ull;   // 16-byte multiple
+  if (piece < 4096) piece = 4096;
+  uint64_t o = beg + (uint64_t)lane * piece;
+  const uint64_t stop = end < o + piece ? end : o + piece;
+  while (o < stop) {
+    const uint64_t c = stop - o < (1u << 19) ? stop - o : (1u << 19);
+    prefetch_l2(base + o, (uint32_t)c);
+    o += c;
+  }
+}
+
 __device__ void prefetch_for_experts(const Fwd& p) {
   if (threadIdx.x >= 32) return;
   const int lane = threadIdx.x;
   const int A = p.active[0];
-  const uint64_t slots = (uint64_t)gridDim.x * 32, me = (uint64_t)blockIdx.x * 32 + lane;
-  uint64_t gi = 0, budget = kPrefetchCap;
-  auto range = [&](uint64_t beg, uint64_t end) {
-    if (end > beg + budget) end = beg + budget;
-    budget -= end - beg;
-    for (uint64_t o = beg; o < end; o += kPrefetchPiece, ++gi)
-      if (gi % slots == me)
-        prefetch_l2(p.img + o, (uint32_t)(end - o < kPrefetchPiece ? end - o : kPrefetchPiece));
-  };
-  for (int h = 0; h < 3 && budget; ++h)
-    for (int a = 0; a < A && budget; ++a) {
-      const ExpertDesc& xd = p.desc[h * p.E + p.active[1 + a]];
-      range(xd.begin, xd.end);
-    }
+  const int nr = 3 * A + 1;
   const uint64_t bo = (uint64_t)((const uint8_t*)p.basis_out - p.img);
-  if (budget) range(bo, bo + (uint64_t)p.D * p.n_pad * 2);
+  uint64_t budget = kPrefetchCap;
+  for (int r = 0; r < nr; ++r) {
+    uint64_t beg, end;
+    if (r < 3 * A) {
+      const int h = r / A, a = r - h * A;
+      const ExpertDesc& xd = p.desc[h * p.E + p.active[1 + a]];
+      beg = xd.begin;
+      end = xd.end;
+    } else {
+      beg = bo;
+      end = bo + (uint64_t)p.D * p.n_pad * 2;
+    }
+    if (end - beg > budget) end = beg + budget;
+    budget -= end - beg;
+    if ((int)(r % gridDim.x) == (int)blockIdx.x && end > beg) prefetch_range(p.img, beg, end, lane);
+    if (!budget) break;
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -280,7 +473,18 @@ __global__ void __launch_bounds__(kThreads) k_gemv(Fwd p) {
   const int lane = threadIdx.x & 31;
   const int gw = blockIdx.x * kWarps + (threadIdx.x >> 5);
   const int nwt = gridDim.x * kWarps;
+  uint4 pre[8];
+  const bool have_pre = gw < nrows;
+  if (have_pre) {   // the warp's first row batch: issued before anything it waits on
+    const uint4* rp = reinterpret_cast<const uint4*>(mat + (size_t)gw * ld);
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int c = u * 32 + lane;
+      pre[u] = c < nch ? ldg_stream(rp + c) : make_uint4(0, 0, 0, 0);
+    }
+  }
   if (PROJ) {
+    if (p.decode && blockIdx.x == 0 && threadIdx.x == 0) *p.status = 0;
     const size_t ng = (size_t)p.P * 2 * p.I_pad / 4, ns = (size_t)p.T * p.n_pad / 4;
     const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
     for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < ng + ns;
@@ -314,10 +518,15 @@ __global__ void __launch_bounds__(kThreads) k_gemv(Fwd p) {
       for (int tt = 0; tt < TB; ++tt) acc[tt] = 0.f;
       for (int c0 = 0; c0 < nch; c0 += 32 * 8) {
         uint4 v[8];
+        if (have_pre && t0 == 0 && row == gw && c0 == 0) {
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          const int c = c0 + u * 32 + lane;
-          v[u] = c < nch ? ldg_stream(rp + c) : make_uint4(0, 0, 0, 0);
+          for (int u = 0; u < 8; ++u) v[u] = pre[u];
+        } else {
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const int c = c0 + u * 32 + lane;
+            v[u] = c < nch ? ldg_stream(rp + c) : make_uint4(0, 0, 0, 0);
+          }
         }
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
@@ -355,7 +564,136 @@ __global__ void __launch_bounds__(kThreads) k_gemv(Fwd p) {
       }
     }
   }
+  if (PROJ && !p.decode) {
+    pdl_wait();
+    prefetch_for_experts(p);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// K1 / K4, bulk-copy form: one block per SM owns a contiguous range of rows and
+// streams it through a two-stage shared-memory ring filled by cp.async.bulk
+// (one copy per stage), so few registers are held and the row bytes are in
+// flight from the block's first instructions (K4 issues its first stages before
+// waiting for the down kernel).  Warps take rows of a stage round-robin.
+// ---------------------------------------------------------------------------
+template <int TB, bool PROJ>
+__global__ void __launch_bounds__(kThreads) k_gemv_bulk(Fwd p, int stage_rows) {
+  pdl_trigger();
+  extern __shared__ int4 smem_gb[];
+  const int ld = PROJ ? p.D_pad : p.n_pad;
+  const int nrows = PROJ ? 2 * p.n : p.D;
+  const uint32_t row_bytes = (uint32_t)ld * 2;
+  const uint16_t* mat = PROJ ? p.basis_in : p.basis_out;
+  uint8_t* ring = reinterpret_cast<uint8_t*>(smem_gb);                          // [2][stage_rows][ld] bf16
+  float* vs = reinterpret_cast<float*>(ring + 2 * (size_t)stage_rows * row_bytes);   // [TB][ld]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(vs + (size_t)TB * ld);             // [2]
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  const int per = (nrows + gridDim.x - 1) / gridDim.x;
+  const int r0 = min(nrows, blockIdx.x * per), r1 = min(nrows, r0 + per);
+  const int nst = (r1 - r0 + stage_rows - 1) / stage_rows;
+  auto issue = [&](int st) {
+    const int a = r0 + st * stage_rows, b = min(r1, a + stage_rows);
+    uint64_t* bar = bars + (st & 1);
+    mbar_expect_tx(bar, (uint32_t)(b - a) * row_bytes);
+    bulk_g2s(ring + (size_t)(st & 1) * stage_rows * row_bytes, mat + (size_t)a * ld, (uint32_t)(b - a) * row_bytes, bar);
+  };
+  if (threadIdx.x == 0) {
+    mbar_init(bars);
+    mbar_init(bars + 1);
+    for (int st = 0; st < min(2, nst); ++st) issue(st);
+  }
   if (PROJ) {
+    if (p.decode && blockIdx.x == 0 && threadIdx.x == 0) *p.status = 0;
+    const size_t ng = (size_t)p.P * 2 * p.I_pad / 4, ns = (size_t)p.T * p.n_pad / 4;
+    const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < ng + ns; i += (size_t)gridDim.x * blockDim.x) {
+      if (i < ng) reinterpret_cast<float4*>(p.gu)[i] = z4;
+      else reinterpret_cast<float4*>(p.s)[i - ng] = z4;
+    }
+  } else {
+    pdl_wait();
+  }
+  bool ok = true;
+  int uses[2] = {0, 0};   // completed phases of each ring buffer (uniform across the block)
+  for (int t0 = 0; t0 < p.T; t0 += TB) {
+    const int tb = min(TB, p.T - t0);
+    __syncthreads();   // every stage of the previous token batch has been consumed
+    if (t0 > 0 && threadIdx.x == 0)
+      for (int st = 0; st < min(2, nst); ++st) issue(st);
+    // stage the vectors: 8 independent loads per thread in flight at a time
+    for (int i0 = threadIdx.x; i0 < TB * ld; i0 += 8 * blockDim.x) {
+      float v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int i = i0 + u * blockDim.x;
+        const int tt = i / ld, c = i - tt * ld;
+        v[u] = 0.f;
+        if (i < TB * ld && tt < tb) {
+          if (PROJ) {
+            if (c < p.D) v[u] = __uint_as_float((uint32_t)p.x[(size_t)(t0 + tt) * p.D + c] << 16);
+          } else {
+            if (c < p.n) v[u] = p.s[(size_t)(t0 + tt) * p.n_pad + c];
+          }
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        if (i0 + u * blockDim.x < TB * ld) vs[i0 + u * blockDim.x] = v[u];
+    }
+    __syncthreads();
+    for (int st = 0; st < nst; ++st) {
+      const uint32_t parity = (uint32_t)uses[st & 1] & 1u;
+      ++uses[st & 1];
+      if (!mbar_wait(bars + (st & 1), parity)) {
+        if (threadIdx.x == 0) atomicCAS(p.status, 0, BITSMOE_ERR_TIMEOUT);
+        ok = false;
+        break;
+      }
+      const int a = r0 + st * stage_rows, b = min(r1, a + stage_rows);
+      const uint8_t* buf = ring + (size_t)(st & 1) * stage_rows * row_bytes;
+      for (int row = a + wid; row < b; row += kWarps) {
+        const uint8_t* rp = buf + (size_t)(row - a) * row_bytes;
+        float acc[TB];
+#pragma unroll
+        for (int tt = 0; tt < TB; ++tt) acc[tt] = 0.f;
+        for (int c = lane; c < (ld >> 3); c += 32) {
+          const uint4 v = lds128(rp + (size_t)c * 16);
+          const float w0 = bf16lo(v.x), w1 = bf16hi(v.x), w2 = bf16lo(v.y), w3 = bf16hi(v.y);
+          const float w4 = bf16lo(v.z), w5 = bf16hi(v.z), w6 = bf16lo(v.w), w7 = bf16hi(v.w);
+#pragma unroll
+          for (int tt = 0; tt < TB; ++tt) {
+            const float4* xv = reinterpret_cast<const float4*>(vs + tt * ld + c * 8);
+            const float4 xa = xv[0], xb = xv[1];
+            float r = acc[tt];
+            r = fmaf(w0, xa.x, r); r = fmaf(w1, xa.y, r); r = fmaf(w2, xa.z, r); r = fmaf(w3, xa.w, r);
+            r = fmaf(w4, xb.x, r); r = fmaf(w5, xb.y, r); r = fmaf(w6, xb.z, r); r = fmaf(w7, xb.w, r);
+            acc[tt] = r;
+          }
+        }
+#pragma unroll
+        for (int tt = 0; tt < TB; ++tt) acc[tt] = warp_sum(acc[tt]);
+        if (lane == 0) {
+#pragma unroll
+          for (int tt = 0; tt < TB; ++tt) {
+            if (tt < tb) {
+              const int t = t0 + tt;
+              if (PROJ) {
+                const int h = row >= p.n, j = row - h * p.n;
+                p.z[((size_t)h * p.T + t) * p.n_pad + j] = acc[tt];
+              } else {
+                p.y[(size_t)t * p.D + row] = acc[tt];
+              }
+            }
+          }
+        }
+      }
+      __syncthreads();   // stage consumed: refill its buffer with stage st + 2
+      if (threadIdx.x == 0 && st + 2 < nst) issue(st + 2);
+    }
+    if (!ok) break;
+  }
+  if (PROJ && !p.decode) {
     pdl_wait();
     prefetch_for_experts(p);
   }
@@ -398,7 +736,7 @@ __device__ __forceinline__ void rl_dp(const uint4& v, const int* cp, int tstride
     }
 }
 
-template <int B, int TB>
+template <int B, int TB, bool SH = false>
 __device__ __forceinline__ void rl_range(const uint8_t* code, int ntl, const int* cq32, int tstride,
                                          float (&accf)[4][TB]) {
   constexpr int U = rl_units(B), C = rl_chunks(B);
@@ -411,7 +749,7 @@ __device__ __forceinline__ void rl_range(const uint8_t* code, int ntl, const int
   for (int t = 0; t < ntl; ++t) {
     uint4 v[C];
 #pragma unroll
-    for (int c = 0; c < C; ++c) v[c] = ldg_stream(code + (size_t)(t * C + c) * kChunkBytes);
+    for (int c = 0; c < C; ++c) v[c] = ld128<SH>(code + (size_t)(t * C + c) * kChunkBytes);
     const int* cp = cq32 + t * (U / 2);
     if (B == 3) {
       rl_dp<2, TB>(v[0], cp, tstride, acc);
@@ -439,19 +777,23 @@ __device__ __forceinline__ void rl_range(const uint8_t* code, int ntl, const int
   }
 }
 
-template <int TB>
+// 16-bit units: tile of 4 units in 2 chunks; chunk c, word w = fp16(unit 2c, row w) | fp16(unit 2c+1, row w)
+template <int TB, bool SH = false>
 __device__ __forceinline__ void rl_range16(const uint8_t* code, int ntl, const int32_t* unit, const float* alpha,
                                            const float* const (&zrow)[TB], float (&acc16)[4][TB]) {
   for (int t = 0; t < ntl; ++t) {
-    const uint4 v = ldg_stream(code + (size_t)t * kChunkBytes);
-    const int j0 = unit[2 * t], j1 = unit[2 * t + 1];
-    const float a0 = alpha[2 * t], a1 = alpha[2 * t + 1];
-    const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-    for (int tt = 0; tt < TB; ++tt) {
-      const float c0 = a0 * zrow[tt][j0], c1 = a1 * zrow[tt][j1];
+    for (int c = 0; c < 2; ++c) {
+      const uint4 v = ld128<SH>(code + (size_t)(2 * t + c) * kChunkBytes);
+      const int j0 = unit[4 * t + 2 * c], j1 = unit[4 * t + 2 * c + 1];
+      const float a0 = alpha[4 * t + 2 * c], a1 = alpha[4 * t + 2 * c + 1];
+      const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-      for (int w = 0; w < 4; ++w) acc16[w][tt] = fmaf(c0, f16lo(wv[w]), fmaf(c1, f16hi(wv[w]), acc16[w][tt]));
+      for (int tt = 0; tt < TB; ++tt) {
+        const float c0 = a0 * zrow[tt][j0], c1 = a1 * zrow[tt][j1];
+#pragma unroll
+        for (int w = 0; w < 4; ++w) acc16[w][tt] = fmaf(c0, f16lo(wv[w]), fmaf(c1, f16hi(wv[w]), acc16[w][tt]));
+      }
     }
   }
 }
@@ -518,7 +860,7 @@ __global__ void __launch_bounds__(kThreads) k_gateup(Fwd p) {
           const float al = alpha[gs];
 #pragma unroll
           for (int gl = 0; gl < G; ++gl) {
-            const float sc = __half2float(__ushort_as_half((unsigned short)(sz[(size_t)(g_base + gl) * bd.nslots + bs] & 0xFFFFu)));
+            const float sc = __half2float(__ushort_as_half((unsigned short)(sz[(size_t)(g_base + gl) * xd.nslots + bs] & 0xFFFFu)));
 #pragma unroll
             for (int tt = 0; tt < TB; ++tt) mx[tt] = fmaxf(mx[tt], fabsf(al * sc * zrow[tt][j]));
           }
@@ -548,7 +890,7 @@ __global__ void __launch_bounds__(kThreads) k_gateup(Fwd p) {
           const float al = alpha[gs];
 #pragma unroll
           for (int gl = 0; gl < G; ++gl) {
-            const uint32_t szw = sz[(size_t)(g_base + gl) * bd.nslots + bs];
+            const uint32_t szw = sz[(size_t)(g_base + gl) * xd.nslots + bs];
             const float sc = __half2float(__ushort_as_half((unsigned short)(szw & 0xFFFFu)));
             const float zp = __half2float(__ushort_as_half((unsigned short)(szw >> 16)));
 #pragma unroll
@@ -587,7 +929,7 @@ __global__ void __launch_bounds__(kThreads) k_gateup(Fwd p) {
           case 6: rl_range<6, TB>(code, ntl, cp, tstride, accf); break;
           case 8: rl_range<8, TB>(code, ntl, cp, tstride, accf); break;
           default: {
-            const int gs0 = bd.slot0 + rg[ri].lo * 2;
+            const int gs0 = bd.slot0 + rg[ri].lo * 4;
             rl_range16<TB>(code, ntl, unit + gs0, alpha + gs0, zrow, acc16);
           }
         }
@@ -656,10 +998,11 @@ __device__ __forceinline__ void ul_chunk(const uint4& v, int rbase, const int* h
   }
 }
 
-template <int B, int G, int TB>
+// scale/zero of group g of the lane's unit: sz[(g - szg0) * szstride + szcol]
+template <int B, int G, int TB, bool SH = false>
 __device__ __forceinline__ void ul_tile(const Fwd& p, const uint8_t* code, int rb0, int rb1, const int16_t* hq,
-                                        int hstride, const int* Hg, const uint32_t* sz, int nslots, int bs,
-                                        float (&accf)[TB]) {
+                                        int hstride, const int* Hg, const uint32_t* sz, int szstride, int szg0,
+                                        int szcol, float (&accf)[TB]) {
   constexpr int C = ul_chunks(B);
   const int gshift = 31 - __clz(p.group);
   const int tstride = hstride / 2;
@@ -669,7 +1012,7 @@ __device__ __forceinline__ void ul_tile(const Fwd& p, const uint8_t* code, int r
     if (B == 16) {
 #pragma unroll 4
       for (int c = 0; c < 16; ++c) {
-        const uint4 v = ldg_stream(cb + (size_t)c * kChunkBytes);
+        const uint4 v = ld128<SH>(cb + (size_t)c * kChunkBytes);
         const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
         for (int w = 0; w < 4; ++w) {
@@ -691,7 +1034,7 @@ __device__ __forceinline__ void ul_tile(const Fwd& p, const uint8_t* code, int r
       for (int tt = 0; tt < TB; ++tt) acc[g][tt] = acch[g][tt] = 0;
     uint4 v[C];
 #pragma unroll
-    for (int c = 0; c < C; ++c) v[c] = ldg_stream(cb + (size_t)c * kChunkBytes);
+    for (int c = 0; c < C; ++c) v[c] = ld128<SH>(cb + (size_t)c * kChunkBytes);
     if (B == 3) {
       ul_chunk<2, G, TB>(v[0], 0, hq32, tstride, gshift, acc);
       ul_chunk<2, G, TB>(v[1], 64, hq32, tstride, gshift, acc);
@@ -709,7 +1052,7 @@ __device__ __forceinline__ void ul_tile(const Fwd& p, const uint8_t* code, int r
     const int gfirst = (rb * kRows) >> gshift;
 #pragma unroll
     for (int g = 0; g < G; ++g) {
-      const uint32_t szw = sz[(size_t)(gfirst + g) * nslots + bs];
+      const uint32_t szw = sz[(size_t)(gfirst + g - szg0) * szstride + szcol];
       const float sc = __half2float(__ushort_as_half((unsigned short)(szw & 0xFFFFu)));
       const float zp = __half2float(__ushort_as_half((unsigned short)(szw >> 16)));
       const bool starts = G > 1 || ((rb * kRows) & (p.group - 1)) == 0;
@@ -825,13 +1168,13 @@ __global__ void __launch_bounds__(kThreads) k_down(Fwd p) {
 #pragma unroll
       for (int tt = 0; tt < TB; ++tt) accf[tt] = 0.f;
       switch (bd.bits) {
-        case 1: ul_tile<1, G, TB>(p, code, rb0, rb1, hq, nrows_max, Hg, sz, bd.nslots, bs, accf); break;
-        case 2: ul_tile<2, G, TB>(p, code, rb0, rb1, hq, nrows_max, Hg, sz, bd.nslots, bs, accf); break;
-        case 3: ul_tile<3, G, TB>(p, code, rb0, rb1, hq, nrows_max, Hg, sz, bd.nslots, bs, accf); break;
-        case 4: ul_tile<4, G, TB>(p, code, rb0, rb1, hq, nrows_max, Hg, sz, bd.nslots, bs, accf); break;
-        case 6: ul_tile<6, G, TB>(p, code, rb0, rb1, hq, nrows_max, Hg, sz, bd.nslots, bs, accf); break;
-        case 8: ul_tile<8, G, TB>(p, code, rb0, rb1, hq, nrows_max, Hg, sz, bd.nslots, bs, accf); break;
-        default: ul_tile<16, G, TB>(p, code, rb0, rb1, hq, nrows_max, Hg, sz, bd.nslots, bs, accf); break;
+        case 1: ul_tile<1, G, TB>(p, code, rb0, rb1, hq, nrows_max, Hg, sz, xd.nslots, 0, bs, accf); break;
+        case 2: ul_tile<2, G, TB>(p, code, rb0, rb1, hq, nrows_max, Hg, sz, xd.nslots, 0, bs, accf); break;
+        case 3: ul_tile<3, G, TB>(p, code, rb0, rb1, hq, nrows_max, Hg, sz, xd.nslots, 0, bs, accf); break;
+        case 4: ul_tile<4, G, TB>(p, code, rb0, rb1, hq, nrows_max, Hg, sz, xd.nslots, 0, bs, accf); break;
+        case 6: ul_tile<6, G, TB>(p, code, rb0, rb1, hq, nrows_max, Hg, sz, xd.nslots, 0, bs, accf); break;
+        case 8: ul_tile<8, G, TB>(p, code, rb0, rb1, hq, nrows_max, Hg, sz, xd.nslots, 0, bs, accf); break;
+        default: ul_tile<16, G, TB>(p, code, rb0, rb1, hq, nrows_max, Hg, sz, xd.nslots, 0, bs, accf); break;
       }
       if (al != 0.f) {
 #pragma unroll
@@ -841,6 +1184,405 @@ __global__ void __launch_bounds__(kThreads) k_down(Fwd p) {
             const float scale = shs[tt] * (1.f / 32767.f);
             atomicAdd(p.s + (size_t)(pr / p.k) * p.n_pad + j, p.pair_weight[pr] * al * scale * accf[tt]);
           }
+        }
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Decode mode (small T): the gate/up and down kernels compute the routing
+// themselves from the logits, then, in the PDL prologue that overlaps the
+// previous kernel, stage their packed codes into shared memory with bulk
+// copies and their per-unit metadata into registers.  After
+// griddepcontrol.wait only the data dependency (z, gate/up) remains.
+// ---------------------------------------------------------------------------
+constexpr int kK2DecWarps = 4;
+constexpr int kZ = 12;             // item slots per lane whose z values are gathered at once
+constexpr int kK3DecWarps = 4;
+
+template <int G, int TB>
+__global__ void __launch_bounds__(kK2DecWarps * 32) k_gateup_dec(Fwd p) {
+  pdl_trigger();
+  extern __shared__ int4 smem_k2d[];
+  uint32_t* rsm = reinterpret_cast<uint32_t*>(smem_k2d);
+  const int rwords = (route_words(p.T, p.E, p.P) + 3) & ~3;
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  const int smax = p.s16 - 8;                      // slots of the largest item, multiple of 8
+  const size_t per_warp = (size_t)p.seg_bytes + (size_t)smax * 4 * (2 + G) + (size_t)G * TB * p.s16 * 2 + 16;
+  uint8_t* codes = reinterpret_cast<uint8_t*>(rsm + rwords) + wid * per_warp;
+  int* su = reinterpret_cast<int*>(codes + p.seg_bytes);           // unit index per local slot
+  float* sa = reinterpret_cast<float*>(su + smax);                 // alpha
+  uint32_t* ssz = reinterpret_cast<uint32_t*>(sa + smax);          // [G][smax] scale | zero << 16
+  int16_t* cq = reinterpret_cast<int16_t*>(ssz + G * smax);        // [G][TB][s16]
+  uint64_t* bar = reinterpret_cast<uint64_t*>(codes + per_warp - 16);
+  const RouteView rv = route_block(p, rsm);
+  const int A = rv.act[0];
+  const int per_e = 2 * p.NRB * p.nseg;
+  const int item = blockIdx.x * kK2DecWarps + wid;
+  // every warp waits for the previous kernel before it exits, so that this
+  // grid completes only after it (PDL completion is then transitive)
+  if (item >= A * per_e) {
+    pdl_wait();
+    return;
+  }
+  const int a = item / per_e;
+  int r = item - a * per_e;
+  const int h = r / (p.NRB * p.nseg);
+  r -= h * p.NRB * p.nseg;
+  const int rb = r / p.nseg, sg = r - rb * p.nseg;
+  const int e = rv.act[1 + a];
+  const ExpertDesc& xd = p.desc[h * p.E + e];
+  const ItemRec it = p.items[((size_t)h * p.E + e) * p.nseg + sg];
+  if (it.nr == 0) {
+    pdl_wait();
+    return;
+  }
+  const int g_base = (rb * kRows) / p.group;
+  if (lane == 0) {
+    const uint32_t mb = (uint32_t)it.nslot * 4;
+    mbar_init(bar);
+    mbar_expect_tx(bar, it.bytes + (2 + G) * mb);
+    bulk_g2s(codes, p.img + xd.code_base + (size_t)rb * xd.rb_stride + it.byte0, it.bytes, bar);
+    bulk_g2s(su, p.img + xd.unit_off + (size_t)it.slot0 * 4, mb, bar);
+    bulk_g2s(sa, p.img + xd.alpha_off + (size_t)it.slot0 * 4, mb, bar);
+#pragma unroll
+    for (int gl = 0; gl < G; ++gl)
+      bulk_g2s(ssz + gl * smax, p.img + xd.sz_off + ((size_t)(g_base + gl) * xd.nslots + it.slot0) * 4, mb, bar);
+  }
+  pdl_wait();
+  // ranges: consecutive buckets, quantised ones first, 16-bit last
+  int nls = 0;
+  for (int q = 0; q < it.nr; ++q)
+    if (it.bits[q] < 16) nls += it.ntl[q] * rl_units(it.bits[q]);
+  const int gl_lane = G == 1 ? 0 : (4 * lane) / p.group;
+  const int ntok = rv.cnt[e], pst = rv.start[e];
+  const int tstride = p.s16 / 2;
+  if (!mbar_wait(bar, 0)) {
+    if (lane == 0) atomicCAS(p.status, 0, BITSMOE_ERR_TIMEOUT);
+    mbar_wait(bar, 0);
+    return;
+  }
+  for (int tb0 = 0; tb0 < ntok; tb0 += TB) {
+    const int tb = min(TB, ntok - tb0);
+    int pair[TB];
+    const float* zrow[TB];
+#pragma unroll
+    for (int tt = 0; tt < TB; ++tt) {
+      pair[tt] = rv.plist[pst + tb0 + min(tt, tb - 1)];
+      zrow[tt] = p.z + ((size_t)h * p.T + pair[tt] / p.k) * p.n_pad;
+    }
+    // c = alpha * z * scale per (slot, group, token): int16 with one scale per token.
+    // The z gathers are issued together (one L2 round trip): kZ slots per lane.
+    const bool fast = nls <= 32 * kZ;
+    float zr[kZ][TB];
+    if (fast) {
+#pragma unroll
+      for (int m = 0; m < kZ; ++m) {
+        const int i = lane + 32 * m;
+        const int j = i < nls ? su[i] : 0;
+#pragma unroll
+        for (int tt = 0; tt < TB; ++tt) zr[m][tt] = i < nls ? zrow[tt][j] : 0.f;
+      }
+#pragma unroll
+      for (int m = 0; m < kZ; ++m) {
+        const int i = lane + 32 * m;
+        const float al = i < nls ? sa[i] : 0.f;
+#pragma unroll
+        for (int tt = 0; tt < TB; ++tt) zr[m][tt] *= al;
+      }
+    }
+    float mx[TB];
+#pragma unroll
+    for (int tt = 0; tt < TB; ++tt) mx[tt] = 0.f;
+    if (fast) {
+#pragma unroll
+      for (int m = 0; m < kZ; ++m) {
+        const int i = lane + 32 * m;
+        if (i < nls) {
+#pragma unroll
+          for (int gl = 0; gl < G; ++gl) {
+            const float sc = __half2float(__ushort_as_half((unsigned short)(ssz[gl * smax + i] & 0xFFFFu)));
+#pragma unroll
+            for (int tt = 0; tt < TB; ++tt) mx[tt] = fmaxf(mx[tt], fabsf(zr[m][tt] * sc));
+          }
+        }
+      }
+    } else {
+      for (int i = lane; i < nls; i += 32) {
+        const int j = su[i];
+        const float al = sa[i];
+#pragma unroll
+        for (int tt = 0; tt < TB; ++tt) {
+          const float zv = al * zrow[tt][j];
+#pragma unroll
+          for (int gl = 0; gl < G; ++gl)
+            mx[tt] = fmaxf(mx[tt], fabsf(zv * __half2float(__ushort_as_half((unsigned short)(ssz[gl * smax + i] & 0xFFFFu)))));
+        }
+      }
+    }
+    float inv[TB], scl[TB];
+#pragma unroll
+    for (int tt = 0; tt < TB; ++tt) {
+      mx[tt] = warp_max(mx[tt]);
+      inv[tt] = mx[tt] > 0.f ? 32767.f / mx[tt] : 0.f;
+      scl[tt] = mx[tt] * (1.f / 32767.f);
+    }
+    float corr[G][TB];
+#pragma unroll
+    for (int gl = 0; gl < G; ++gl)
+#pragma unroll
+      for (int tt = 0; tt < TB; ++tt) corr[gl][tt] = 0.f;
+    if (fast) {
+#pragma unroll
+      for (int m = 0; m < kZ; ++m) {
+        const int i = lane + 32 * m;
+        if (i < nls) {
+#pragma unroll
+          for (int gl = 0; gl < G; ++gl) {
+            const uint32_t w = ssz[gl * smax + i];
+            const float sc = __half2float(__ushort_as_half((unsigned short)(w & 0xFFFFu)));
+            const float zp = __half2float(__ushort_as_half((unsigned short)(w >> 16)));
+#pragma unroll
+            for (int tt = 0; tt < TB; ++tt) {
+              const int ci = __float2int_rn(zr[m][tt] * sc * inv[tt]);
+              cq[(size_t)(gl * TB + tt) * p.s16 + i] = (int16_t)ci;
+              corr[gl][tt] = fmaf((float)ci, zp, corr[gl][tt]);
+            }
+          }
+        }
+      }
+    } else {
+      for (int i = lane; i < nls; i += 32) {
+        const int j = su[i];
+        const float al = sa[i];
+#pragma unroll
+        for (int tt = 0; tt < TB; ++tt) {
+          const float zv = al * zrow[tt][j];
+#pragma unroll
+          for (int gl = 0; gl < G; ++gl) {
+            const uint32_t w = ssz[gl * smax + i];
+            const float sc = __half2float(__ushort_as_half((unsigned short)(w & 0xFFFFu)));
+            const float zp = __half2float(__ushort_as_half((unsigned short)(w >> 16)));
+            const int ci = __float2int_rn(zv * sc * inv[tt]);
+            cq[(size_t)(gl * TB + tt) * p.s16 + i] = (int16_t)ci;
+            corr[gl][tt] = fmaf((float)ci, zp, corr[gl][tt]);
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int gl = 0; gl < G; ++gl)
+#pragma unroll
+      for (int tt = 0; tt < TB; ++tt) corr[gl][tt] = warp_sum(corr[gl][tt]);
+    __syncwarp();
+    float accf[4][TB], acc16[4][TB];
+#pragma unroll
+    for (int w = 0; w < 4; ++w)
+#pragma unroll
+      for (int tt = 0; tt < TB; ++tt) accf[w][tt] = acc16[w][tt] = 0.f;
+    const int* cq32 = reinterpret_cast<const int*>(cq + (size_t)gl_lane * TB * p.s16);
+    uint32_t boff = 0;
+    int ls = 0;
+    for (int q = 0; q < it.nr; ++q) {
+      const int b = it.bits[q], ntl = it.ntl[q];
+      const uint8_t* code = codes + boff + lane * 16;
+      const int* cp = cq32 + ls / 2;
+      switch (b) {
+        case 1: rl_range<1, TB, true>(code, ntl, cp, tstride, accf); break;
+        case 2: rl_range<2, TB, true>(code, ntl, cp, tstride, accf); break;
+        case 3: rl_range<3, TB, true>(code, ntl, cp, tstride, accf); break;
+        case 4: rl_range<4, TB, true>(code, ntl, cp, tstride, accf); break;
+        case 6: rl_range<6, TB, true>(code, ntl, cp, tstride, accf); break;
+        case 8: rl_range<8, TB, true>(code, ntl, cp, tstride, accf); break;
+        default: rl_range16<TB, true>(code, ntl, su + ls, sa + ls, zrow, acc16); break;
+      }
+      boff += (uint32_t)ntl * rl_chunks(b) * kChunkBytes;
+      ls += ntl * rl_units(b);
+    }
+    const int row = rb * kRows + 4 * lane;
+#pragma unroll
+    for (int tt = 0; tt < TB; ++tt) {
+      if (tt < tb) {
+        float cl = corr[0][tt];
+#pragma unroll
+        for (int gl = 1; gl < G; ++gl)
+          if (gl == gl_lane) cl = corr[gl][tt];
+        float o[4];
+#pragma unroll
+        for (int w = 0; w < 4; ++w) o[w] = fmaf(scl[tt], accf[w][tt] - cl, acc16[w][tt]);
+        red_add_v4(p.gu + ((size_t)pair[tt] * 2 + h) * p.I_pad + row, o[0], o[1], o[2], o[3]);
+      }
+    }
+    __syncwarp();
+  }
+}
+
+template <int G, int TB>
+__global__ void __launch_bounds__(kK3DecWarps * 32) k_down_dec(Fwd p) {
+  pdl_trigger();
+  extern __shared__ int4 smem_k3d[];
+  uint32_t* rsm = reinterpret_cast<uint32_t*>(smem_k3d);
+  const int rwords = (route_words(p.T, p.E, p.P) + 3) & ~3;
+  const int rbc = p.rbc;
+  const int nrows_max = rbc * kRows;
+  const int gshift = 31 - __clz(p.group);
+  const int ngc_max = max(1, nrows_max >> gshift);
+  float* hf = reinterpret_cast<float*>(rsm + rwords);                  // [TB][nrows_max]
+  int16_t* hq = reinterpret_cast<int16_t*>(hf + TB * nrows_max);       // [TB][nrows_max]
+  int* Hg = reinterpret_cast<int*>(hq + TB * nrows_max);               // [TB][64]
+  float* red = reinterpret_cast<float*>(Hg + TB * 64);                 // [warps][TB]
+  float* shs = red + kK3DecWarps * TB;                                 // [TB], padded to 4
+  const size_t per_warp = (size_t)p.ul_bytes + (size_t)ngc_max * 32 * 4 + 16;
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  uint8_t* codes = reinterpret_cast<uint8_t*>(shs + ((TB + 3) & ~3)) + wid * per_warp;
+  uint32_t* szs = reinterpret_cast<uint32_t*>(codes + p.ul_bytes);
+  uint64_t* bar = reinterpret_cast<uint64_t*>(codes + per_warp - 16);
+  const RouteView rv = route_block(p, rsm);
+  const int A = rv.act[0];
+  const int ntg = (p.ul_max_tiles + kK3DecWarps - 1) / kK3DecWarps;
+  const int nrc = (p.NRB + rbc - 1) / rbc;
+  const int item = blockIdx.x;
+  if (item >= A * ntg * nrc) {   // wait before exiting: keeps PDL completion transitive
+    pdl_wait();
+    return;
+  }
+  const int a = item / (ntg * nrc);
+  const int r = item - a * ntg * nrc;
+  const int tg = r / nrc, rc = r - tg * nrc;
+  const int e = rv.act[1 + a];
+  const ExpertDesc& xd = p.desc[2 * p.E + e];
+  if (tg * kK3DecWarps >= xd.ntiles) {
+    pdl_wait();
+    return;
+  }
+  const int rb0 = rc * rbc, rb1 = min(p.NRB, rb0 + rbc);
+  const int row0 = rb0 * kRows, nrows = (rb1 - rb0) * kRows;
+  const int tile = tg * kK3DecWarps + wid;
+  int bi = -1;
+  if (tile < xd.ntiles)
+    for (int q = 0; q < xd.nbk; ++q)
+      if (tile >= xd.bk[q].tile0 && tile < xd.bk[q].tile0 + xd.bk[q].ntiles) bi = q;
+  int j = 0, bs = 0, szg0 = 0;
+  float al = 0.f;
+  if (bi >= 0) {
+    const BucketDesc& bd = xd.bk[bi];
+    const uint32_t nb = (uint32_t)(rb1 - rb0) * ul_chunks(bd.bits) * kChunkBytes;
+    if (lane == 0)
+      stage_bytes(codes,
+                  p.img + xd.code_base + bd.code_off +
+                      ((size_t)(tile - bd.tile0) * p.NRB + rb0) * ul_chunks(bd.bits) * kChunkBytes,
+                  nb, bar);
+    bs = (tile - bd.tile0) * 32 + lane;
+    const int gs = bd.slot0 + bs;
+    j = reinterpret_cast<const int32_t*>(p.img + xd.unit_off)[gs];
+    al = reinterpret_cast<const float*>(p.img + xd.alpha_off)[gs];
+    szg0 = row0 >> gshift;
+    if (bd.bits < 16) {
+      const uint32_t* sz = reinterpret_cast<const uint32_t*>(p.img + bd.sz_off);
+      const int g1 = min(p.NG, ((rb1 * kRows - 1) >> gshift) + 1);
+      for (int g0 = szg0; g0 < g1; g0 += 8) {   // 8 loads in flight at a time
+        uint32_t v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) v[u] = g0 + u < g1 ? sz[(size_t)(g0 + u) * xd.nslots + bs] : 0u;
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          if (g0 + u < g1) szs[(g0 + u - szg0) * 32 + lane] = v[u];
+      }
+    }
+  }
+  pdl_wait();
+  const int ntok = rv.cnt[e], pst = rv.start[e];
+  bool staged = false;
+  constexpr int kMaxRowsPerThread = kK3MaxRB * kRows / (kK3DecWarps * 32);
+  for (int tb0 = 0; tb0 < ntok; tb0 += TB) {
+    const int tb = min(TB, ntok - tb0);
+    __syncthreads();   // previous batch finished with hq / Hg
+    for (int i = threadIdx.x; i < TB * 64; i += blockDim.x) Hg[i] = 0;
+    // h = SiLU(gate) * up for this block's rows, kept in registers
+    float hv[kMaxRowsPerThread][TB];
+    float mx[TB];
+#pragma unroll
+    for (int tt = 0; tt < TB; ++tt) mx[tt] = 0.f;
+#pragma unroll
+    for (int m = 0; m < kMaxRowsPerThread; ++m) {
+      const int i = threadIdx.x + m * kK3DecWarps * 32;
+#pragma unroll
+      for (int tt = 0; tt < TB; ++tt) {
+        float v = 0.f;
+        if (i < nrows && tt < tb) {
+          const int pr = rv.plist[pst + tb0 + tt];
+          const float g = p.gu[((size_t)pr * 2) * p.I_pad + row0 + i];
+          const float u = p.gu[((size_t)pr * 2 + 1) * p.I_pad + row0 + i];
+          v = g / (1.f + __expf(-g)) * u;
+        }
+        hv[m][tt] = v;
+        mx[tt] = fmaxf(mx[tt], fabsf(v));
+      }
+    }
+#pragma unroll
+    for (int tt = 0; tt < TB; ++tt) {
+      const float m = warp_max(mx[tt]);
+      if (lane == 0) red[wid * TB + tt] = m;
+    }
+    __syncthreads();
+    float scale[TB];
+#pragma unroll
+    for (int tt = 0; tt < TB; ++tt) {
+      float m = 0.f;
+#pragma unroll
+      for (int w = 0; w < kK3DecWarps; ++w) m = fmaxf(m, red[w * TB + tt]);
+      scale[tt] = m;
+      const float inv = m > 0.f ? 32767.f / m : 0.f;
+#pragma unroll
+      for (int mm = 0; mm < kMaxRowsPerThread; ++mm) {
+        const int i = threadIdx.x + mm * kK3DecWarps * 32;
+        if (i < nrows) {
+          const int q = __float2int_rn(hv[mm][tt] * inv);
+          hq[tt * nrows_max + i] = (int16_t)q;
+          // a warp's 32 consecutive rows lie in one group (group >= 32)
+          int sq = q;
+#pragma unroll
+          for (int o = 16; o; o >>= 1) sq += __shfl_xor_sync(0xFFFFFFFFu, sq, o);
+          if (lane == 0) atomicAdd(&Hg[tt * 64 + (i >> gshift)], sq);
+        }
+      }
+    }
+    if (threadIdx.x == 0)
+#pragma unroll
+      for (int tt = 0; tt < TB; ++tt) shs[tt] = scale[tt];
+    __syncthreads();
+    if (bi < 0) continue;
+    if (!staged) {
+      if (!mbar_wait(bar, 0)) {
+        if (lane == 0) atomicCAS(p.status, 0, BITSMOE_ERR_TIMEOUT);
+        mbar_wait(bar, 0);
+        bi = -1;
+        continue;
+      }
+      staged = true;
+    }
+    const BucketDesc& bd = xd.bk[bi];
+    const uint8_t* code = codes + lane * 16;
+    float accf[TB];
+#pragma unroll
+    for (int tt = 0; tt < TB; ++tt) accf[tt] = 0.f;
+    switch (bd.bits) {
+      case 1: ul_tile<1, G, TB, true>(p, code, rb0, rb1, hq, nrows_max, Hg, szs, 32, szg0, lane, accf); break;
+      case 2: ul_tile<2, G, TB, true>(p, code, rb0, rb1, hq, nrows_max, Hg, szs, 32, szg0, lane, accf); break;
+      case 3: ul_tile<3, G, TB, true>(p, code, rb0, rb1, hq, nrows_max, Hg, szs, 32, szg0, lane, accf); break;
+      case 4: ul_tile<4, G, TB, true>(p, code, rb0, rb1, hq, nrows_max, Hg, szs, 32, szg0, lane, accf); break;
+      case 6: ul_tile<6, G, TB, true>(p, code, rb0, rb1, hq, nrows_max, Hg, szs, 32, szg0, lane, accf); break;
+      case 8: ul_tile<8, G, TB, true>(p, code, rb0, rb1, hq, nrows_max, Hg, szs, 32, szg0, lane, accf); break;
+      default: ul_tile<16, G, TB, true>(p, code, rb0, rb1, hq, nrows_max, Hg, szs, 32, szg0, lane, accf); break;
+    }
+    if (al != 0.f) {
+#pragma unroll
+      for (int tt = 0; tt < TB; ++tt) {
+        if (tt < tb) {
+          const int pr = rv.plist[pst + tb0 + tt];
+          const float scale = shs[tt] * (1.f / 32767.f);
+          atomicAdd(p.s + (size_t)(pr / p.k) * p.n_pad + j, rv.pw[pr] * al * scale * accf[tt]);
         }
       }
     }
@@ -904,9 +1646,20 @@ int launch(K kernel, dim3 grid, dim3 block, size_t smem, cudaStream_t st, bool p
   return BITSMOE_OK;
 }
 
+// Every kernel asks for the largest shared-memory carveout, so that blocks of
+// consecutive kernels of the chain can be resident on one SM at the same time
+// (an SM cannot hold blocks configured with different L1/shared splits).
 template <class K>
 int set_smem(K kernel, size_t smem) {
+  static std::mutex mu;
+  static std::vector<std::pair<const void*, size_t>> done;
+  std::lock_guard<std::mutex> lock(mu);
+  const void* key = reinterpret_cast<const void*>(kernel);
+  for (auto& d : done)
+    if (d.first == key && d.second >= smem) return BITSMOE_OK;
+  BM_CK(cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared));
   if (smem > 48 * 1024) BM_CK(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+  done.emplace_back(key, std::max<size_t>(smem, 48 * 1024));
   return BITSMOE_OK;
 }
 
@@ -943,6 +1696,80 @@ int launch_k2k3(const Fwd& p, int sms, cudaStream_t st, bool pdl, const std::fun
   return launch(k_down<G, TB>, dim3(sms * 2), dim3(kThreads), sm3, st, pdl, p);
 }
 
+template <int TB>
+int launch_gemv_bulk_tb(bool proj, const Fwd& p, int sms, cudaStream_t st, bool pdl) {
+  const int ld = proj ? p.D_pad : p.n_pad;
+  const int nrows = proj ? 2 * p.n : p.D;
+  const size_t row_bytes = (size_t)ld * 2;
+  const size_t vec = (size_t)TB * ld * 4;
+  const size_t budget = vec < 150 * 1024 ? 200 * 1024 - vec : 48 * 1024;
+  const int grid = std::min(nrows, sms);
+  const int per = (nrows + grid - 1) / grid;
+  int stage_rows = (int)std::max<size_t>(1, std::min<size_t>((budget / 2) / row_bytes, (size_t)(per + 1) / 2));
+  const size_t smem = 2 * (size_t)stage_rows * row_bytes + vec + 16;
+  int rc;
+  if (proj) {
+    if ((rc = set_smem(k_gemv_bulk<TB, true>, smem))) return rc;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    BM_CK(cudaLaunchKernelEx(&cfg, k_gemv_bulk<TB, true>, p, stage_rows));
+    return BITSMOE_OK;
+  }
+  if ((rc = set_smem(k_gemv_bulk<TB, false>, smem))) return rc;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  BM_CK(cudaLaunchKernelEx(&cfg, k_gemv_bulk<TB, false>, p, stage_rows));
+  return BITSMOE_OK;
+}
+
+int launch_gemv_bulk(bool proj, const Fwd& p, int sms, cudaStream_t st, bool pdl) {
+  if (p.T <= 1) return launch_gemv_bulk_tb<1>(proj, p, sms, st, pdl);
+  if (p.T <= 2) return launch_gemv_bulk_tb<2>(proj, p, sms, st, pdl);
+  if (p.T <= 4) return launch_gemv_bulk_tb<4>(proj, p, sms, st, pdl);
+  return launch_gemv_bulk_tb<8>(proj, p, sms, st, pdl);
+}
+
+template <int G, int TB>
+int launch_k2k3_dec(const Fwd& p, int A_max, int sms, cudaStream_t st, bool pdl,
+                    const std::function<int()>& between) {
+  int rc;
+  const size_t rbytes = (size_t)((route_words(p.T, p.E, p.P) + 3) & ~3) * 4;
+  const size_t smax = (size_t)p.s16 - 8;
+  const size_t pw2 = (size_t)p.seg_bytes + smax * 4 * (2 + G) + (size_t)G * TB * p.s16 * 2 + 16;
+  const size_t sm2 = rbytes + kK2DecWarps * pw2;
+  const int items2 = A_max * 2 * p.NRB * p.nseg;
+  if ((rc = set_smem(k_gateup_dec<G, TB>, sm2))) return rc;
+  if ((rc = launch(k_gateup_dec<G, TB>, dim3((items2 + kK2DecWarps - 1) / kK2DecWarps), dim3(kK2DecWarps * 32), sm2,
+                   st, pdl, p)))
+    return rc;
+  if (between && (rc = between())) return rc;
+  const size_t nrm = (size_t)p.rbc * kRows;
+  const int ngc_max = std::max(1, (int)(nrm / p.group));
+  const size_t pw3 = (size_t)p.ul_bytes + (size_t)ngc_max * 32 * 4 + 16;
+  const size_t sm3 = rbytes + TB * nrm * 6 + TB * 64 * 4 + kK3DecWarps * TB * 4 + ((TB + 3) & ~3) * 4 +
+                     kK3DecWarps * pw3;
+  const int ntg = (p.ul_max_tiles + kK3DecWarps - 1) / kK3DecWarps;
+  const int nrc = (p.NRB + p.rbc - 1) / p.rbc;
+  if ((rc = set_smem(k_down_dec<G, TB>, sm3))) return rc;
+  return launch(k_down_dec<G, TB>, dim3(std::max(1, A_max * ntg * nrc)), dim3(kK3DecWarps * 32), sm3, st, pdl, p);
+}
+
 template <int G>
 int launch_k2k3_tb(const Fwd& p, int sms, cudaStream_t st, bool pdl, const std::function<int()>& between) {
   return p.T == 1 ? launch_k2k3<G, 1>(p, sms, st, pdl, between) : launch_k2k3<G, 4>(p, sms, st, pdl, between);
@@ -961,6 +1788,7 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
   p.img = L->d_img;
   p.desc = reinterpret_cast<const ExpertDesc*>(L->d_img + hd.off_desc);
   p.seg = reinterpret_cast<const int32_t*>(L->d_img + hd.off_seg);
+  p.items = reinterpret_cast<const ItemRec*>(L->d_img + hd.off_items);
   p.basis_in = reinterpret_cast<const uint16_t*>(L->d_img + hd.off_basis_in);
   p.basis_out = reinterpret_cast<const uint16_t*>(L->d_img + hd.off_basis_out);
   p.D = hd.D; p.E = hd.E; p.I = hd.I; p.n = hd.n; p.group = hd.group;
@@ -969,6 +1797,16 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
   p.T = T; p.k = top_k; p.P = T * top_k;
   p.s16 = (int)align_up(std::max(hd.seg_max_slots, 8), 64) + 8;
   p.rbc = k3_rbc(hd);
+  p.seg_bytes = L->seg_bytes;
+  // decode mode: every kernel can afford the routing of all tokens
+  p.decode = T <= 8 && T * hd.E <= 4096;
+  if (p.decode) {   // down staging: keep a warp's tile within ~48 KB of shared memory
+    const int need = std::max(1, hd.group / kRows);
+    int rbc = std::min(p.rbc, std::max(1, (48 * 1024) / (L->ul_max_chunks * kChunkBytes)));
+    rbc = std::max(need, rbc / need * need);
+    p.rbc = rbc;
+    p.ul_bytes = rbc * L->ul_max_chunks * kChunkBytes;
+  }
   p.x = static_cast<const uint16_t*>(x);
   p.logits = logits;
   p.y = y;
@@ -988,13 +1826,37 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
     if (ev) BM_CK(cudaEventRecord(ev[i], st));
     return BITSMOE_OK;
   };
+  const int G = std::max(1, kRows / hd.group);
+  if (p.decode) {
+    const int A_max = std::min(hd.E, p.P);
+    if ((rc = mark(0))) return rc;
+    if ((rc = mark(1))) return rc;
+    if ((rc = launch_gemv_bulk(true, p, sms, st, false))) return rc;
+    if ((rc = mark(2))) return rc;
+    std::function<int()> between = ev ? std::function<int()>([&]() { return mark(3); }) : std::function<int()>();
+    if (T == 1) {
+      if (G == 1) rc = launch_k2k3_dec<1, 1>(p, A_max, sms, st, pdl, between);
+      else if (G == 2) rc = launch_k2k3_dec<2, 1>(p, A_max, sms, st, pdl, between);
+      else rc = launch_k2k3_dec<4, 1>(p, A_max, sms, st, pdl, between);
+    } else {
+      if (G == 1) rc = launch_k2k3_dec<1, 4>(p, A_max, sms, st, pdl, between);
+      else if (G == 2) rc = launch_k2k3_dec<2, 4>(p, A_max, sms, st, pdl, between);
+      else rc = launch_k2k3_dec<4, 4>(p, A_max, sms, st, pdl, between);
+    }
+    if (rc) return rc;
+    if ((rc = mark(4))) return rc;
+    if ((rc = launch_gemv_bulk(false, p, sms, st, pdl))) return rc;
+    return mark(5);
+  }
   const int tpb = std::max(1, 1024 / hd.E);
+  const size_t router_smem = ((size_t)tpb * hd.E + 2 * (size_t)p.P + 2 * (size_t)hd.E + 1) * 4;
+  if (router_smem > 200 * 1024) return BITSMOE_ERR_SHAPE;
   if ((rc = mark(0))) return rc;
-  if ((rc = launch(k_router, dim3(1), dim3(1024), (size_t)tpb * hd.E * 4, st, false, p))) return rc;
+  if ((rc = set_smem(k_router, router_smem))) return rc;
+  if ((rc = launch(k_router, dim3(1), dim3(1024), router_smem, st, false, p))) return rc;
   if ((rc = mark(1))) return rc;
   if ((rc = launch_gemv_any(true, p, sms, st, pdl))) return rc;
   if ((rc = mark(2))) return rc;
-  const int G = std::max(1, kRows / hd.group);
   if (G == 1) rc = launch_k2k3_tb<1>(p, sms, st, pdl, ev ? [&]() { return mark(3); } : std::function<int()>());
   else if (G == 2) rc = launch_k2k3_tb<2>(p, sms, st, pdl, ev ? [&]() { return mark(3); } : std::function<int()>());
   else rc = launch_k2k3_tb<4>(p, sms, st, pdl, ev ? [&]() { return mark(3); } : std::function<int()>());
@@ -1039,6 +1901,24 @@ int upload(std::vector<uint8_t>&& img, int device, bitsmoe_layer** out) {
   L->d_img = d;
   L->bytes = img.size();
   L->meta.assign(img.begin(), img.begin() + meta_end);
+  {
+    const ExpertDesc* d = L->desc();
+    const int32_t* sg = reinterpret_cast<const int32_t*>(L->meta.data() + hd->off_seg);
+    for (int pi = 0; pi < 2 * hd->E; ++pi) {
+      const ExpertDesc& x = d[pi];
+      for (int q = 0; q < hd->nseg; ++q) {
+        const int t0 = sg[(size_t)pi * (hd->nseg + 1) + q], t1 = sg[(size_t)pi * (hd->nseg + 1) + q + 1];
+        int bytes = 0;
+        for (int k = 0; k < x.nbk; ++k) {
+          const int lo = std::max(t0, x.bk[k].tile0), hi = std::min(t1, x.bk[k].tile0 + x.bk[k].ntiles);
+          if (hi > lo) bytes += (hi - lo) * rl_chunks(x.bk[k].bits) * kChunkBytes;
+        }
+        L->seg_bytes = std::max(L->seg_bytes, bytes);
+      }
+    }
+    for (int pi = 2 * hd->E; pi < 3 * hd->E; ++pi)
+      for (int k = 0; k < d[pi].nbk; ++k) L->ul_max_chunks = std::max(L->ul_max_chunks, ul_chunks(d[pi].bk[k].bits));
+  }
   *out = L;
   return BITSMOE_OK;
 }

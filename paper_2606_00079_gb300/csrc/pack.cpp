@@ -55,8 +55,8 @@ void visit_rl(int b, int ntiles, int NRB, uint64_t rb_stride_words, uint64_t buc
                                   ((uint64_t)(tile * C + c) * 32 + lane) * 4 + w;
             const int row = rb * kRows + 4 * lane + w;
             if (b == 16) {
-              f(word, 0, 16, 0, tile * 2, row);
-              f(word, 16, 16, 0, tile * 2 + 1, row);
+              f(word, 0, 16, 0, tile * U + 2 * c, row);
+              f(word, 16, 16, 0, tile * U + 2 * c + 1, row);
               continue;
             }
             const Plane p = rl_plane(b, c);
@@ -253,6 +253,7 @@ int build_image(const bitsmoe_layer_host* src, std::vector<uint8_t>& img) {
   uint64_t off = align_up(sizeof(ImageHeader), 256);
   hd.off_desc = off;      off = align_up(off + desc.size() * sizeof(ExpertDesc), 256);
   hd.off_seg = off;       off = align_up(off + seg.size() * sizeof(int32_t), 256);
+  hd.off_items = off;     off = align_up(off + 2ull * E * nseg * sizeof(ItemRec), 256);
   hd.off_basis_in = off;  off = align_up(off + 2ull * n * d.D_pad * 2, 256);
   hd.off_basis_out = off; off = align_up(off + (uint64_t)d.D * d.n_pad * 2, 256);
   for (size_t pi = 0; pi < desc.size(); ++pi) {
@@ -260,13 +261,8 @@ int build_image(const bitsmoe_layer_host* src, std::vector<uint8_t>& img) {
     x.begin = off;
     x.unit_off = off;  off = align_up(off + (uint64_t)x.nslots * 4, 16);
     x.alpha_off = off; off = align_up(off + (uint64_t)x.nslots * 4, 16);
-    for (int k = 0; k < x.nbk; ++k) {
-      BucketDesc& bd = x.bk[k];
-      if (bd.bits < 16) {
-        bd.sz_off = off;
-        off = align_up(off + (uint64_t)d.NG * bd.nslots * 4, 16);
-      }
-    }
+    x.sz_off = off;    off = align_up(off + (uint64_t)d.NG * x.nslots * 4, 16);
+    for (int k = 0; k < x.nbk; ++k) x.bk[k].sz_off = x.sz_off + (uint64_t)x.bk[k].slot0 * 4;
     hd.meta_bytes += off - x.begin;
     off = align_up(off, 256);
     x.code_base = off;
@@ -286,6 +282,34 @@ int build_image(const bitsmoe_layer_host* src, std::vector<uint8_t>& img) {
   std::memcpy(base, &hd, sizeof(hd));
   std::memcpy(base + hd.off_desc, desc.data(), desc.size() * sizeof(ExpertDesc));
   std::memcpy(base + hd.off_seg, seg.data(), seg.size() * sizeof(int32_t));
+  // gate/up item table
+  {
+    ItemRec* items = reinterpret_cast<ItemRec*>(base + hd.off_items);
+    for (int pi = 0; pi < 2 * E; ++pi) {
+      const ExpertDesc& x = desc[pi];
+      const int32_t* sg = &seg[(size_t)pi * (nseg + 1)];
+      for (int q = 0; q < nseg; ++q) {
+        ItemRec& it = items[(size_t)pi * nseg + q];
+        std::memset(&it, 0, sizeof(it));
+        const int t0 = sg[q], t1 = sg[q + 1];
+        for (int k = 0; k < x.nbk; ++k) {
+          const BucketDesc& bd = x.bk[k];
+          const int lo = std::max(t0, bd.tile0) - bd.tile0, hi = std::min(t1, bd.tile0 + bd.ntiles) - bd.tile0;
+          if (lo >= hi) continue;
+          if (it.nr == 0) {
+            it.bk0 = (uint8_t)k;
+            it.byte0 = (uint32_t)(bd.code_off + (uint64_t)lo * rl_chunks(bd.bits) * kChunkBytes);
+            it.slot0 = (uint32_t)(bd.slot0 + lo * rl_units(bd.bits));
+          }
+          it.bits[it.nr] = (uint8_t)bd.bits;
+          it.ntl[it.nr] = (uint16_t)(hi - lo);
+          it.bytes += (uint32_t)((hi - lo) * rl_chunks(bd.bits) * kChunkBytes);
+          it.nslot = (uint16_t)(it.nslot + (hi - lo) * rl_units(bd.bits));
+          ++it.nr;
+        }
+      }
+    }
+  }
 
   // 4. bases
   uint16_t* bin = reinterpret_cast<uint16_t*>(base + hd.off_basis_in);
@@ -320,7 +344,7 @@ int build_image(const bitsmoe_layer_host* src, std::vector<uint8_t>& img) {
         for (int g = 0; g < ngroups_real; ++g)
           for (int s = 0; s < bd.count; ++s) {
             const size_t q = (he * n + us[s]) * ngroups_real + g;
-            sz[(size_t)g * bd.nslots + s] = (uint32_t)src->scale[q] | ((uint32_t)src->zero[q] << 16);
+            sz[(size_t)g * x.nslots + s] = (uint32_t)src->scale[q] | ((uint32_t)src->zero[q] << 16);
           }
       }
       auto put = [&](uint64_t word, int bitpos, int pb, int pshift, int slot, int row) {
@@ -353,6 +377,7 @@ int validate_image(const uint8_t* img, size_t bytes) {
   auto in = [&](uint64_t off, uint64_t len) { return off <= bytes && len <= bytes - off; };
   if (!in(hd->off_desc, 3ull * E * sizeof(ExpertDesc)) ||
       !in(hd->off_seg, 2ull * E * (hd->nseg + 1) * 4) ||
+      !in(hd->off_items, 2ull * E * hd->nseg * sizeof(ItemRec)) || hd->off_items % 16 ||
       !in(hd->off_basis_in, 2ull * n * hd->D_pad * 2) ||
       !in(hd->off_basis_out, (uint64_t)hd->D * hd->n_pad * 2))
     return BITSMOE_ERR_BLOB;
@@ -365,7 +390,8 @@ int validate_image(const uint8_t* img, size_t bytes) {
     const bool rl = pi < 2 * E;
     if (x.nbk < 0 || x.nbk > kNumBk) return BITSMOE_ERR_BLOB;
     if (!in(x.unit_off, (uint64_t)x.nslots * 4) || !in(x.alpha_off, (uint64_t)x.nslots * 4) ||
-        x.unit_off % 4 || x.alpha_off % 4 || x.code_base % 16)
+        !in(x.sz_off, (uint64_t)hd->NG * x.nslots * 4) || x.unit_off % 16 || x.alpha_off % 16 ||
+        x.sz_off % 16 || x.code_base % 16 || x.nslots % 4)
       return BITSMOE_ERR_BLOB;
     const uint64_t stream = rl ? x.rb_stride * hd->NRB : x.rb_stride;
     if (!in(x.code_base, stream)) return BITSMOE_ERR_BLOB;
@@ -381,8 +407,7 @@ int validate_image(const uint8_t* img, size_t bytes) {
           bd.nslots != bd.ntiles * per_tile || bd.slot0 != slot || bd.tile0 != tile ||
           bd.code_off != off)
         return BITSMOE_ERR_BLOB;
-      if (bd.bits < 16 && (!in(bd.sz_off, (uint64_t)hd->NG * bd.nslots * 4) || bd.sz_off % 4))
-        return BITSMOE_ERR_BLOB;
+      if (bd.sz_off != x.sz_off + (uint64_t)bd.slot0 * 4) return BITSMOE_ERR_BLOB;
       off += rl ? (uint64_t)bd.ntiles * rl_chunks(bd.bits) * kChunkBytes
                 : (uint64_t)bd.ntiles * hd->NRB * ul_chunks(bd.bits) * kChunkBytes;
       slot += bd.nslots;
@@ -395,7 +420,26 @@ int validate_image(const uint8_t* img, size_t bytes) {
     for (int s = 0; s < x.nslots; ++s)
       if (unit[s] < 0 || unit[s] >= n) return BITSMOE_ERR_BLOB;
     if (rl) {
+      const ItemRec* items = reinterpret_cast<const ItemRec*>(img + hd->off_items) + (size_t)pi * hd->nseg;
       const int32_t* sg = seg + (size_t)pi * (hd->nseg + 1);
+      for (int q = 0; q < hd->nseg; ++q) {   // item records must match the segment table
+        const ItemRec& it = items[q];
+        int nr = 0, slots = 0;
+        uint64_t bytes = 0;
+        for (int k = 0; k < x.nbk; ++k) {
+          const BucketDesc& bd = x.bk[k];
+          const int lo = std::max(sg[q], bd.tile0) - bd.tile0, hi = std::min(sg[q + 1], bd.tile0 + bd.ntiles) - bd.tile0;
+          if (lo >= hi) continue;
+          if (nr == 0 && (it.bk0 != k || it.byte0 != bd.code_off + (uint64_t)lo * rl_chunks(bd.bits) * kChunkBytes ||
+                          it.slot0 != (uint32_t)(bd.slot0 + lo * rl_units(bd.bits))))
+            return BITSMOE_ERR_BLOB;
+          if (nr >= kNumBk || it.bits[nr] != bd.bits || it.ntl[nr] != hi - lo) return BITSMOE_ERR_BLOB;
+          bytes += (uint64_t)(hi - lo) * rl_chunks(bd.bits) * kChunkBytes;
+          slots += (hi - lo) * rl_units(bd.bits);
+          ++nr;
+        }
+        if (it.nr != nr || it.bytes != bytes || it.nslot != slots) return BITSMOE_ERR_BLOB;
+      }
       if (sg[0] != 0 || sg[hd->nseg] != x.ntiles) return BITSMOE_ERR_BLOB;
       for (int s = 0; s < hd->nseg; ++s)
         if (sg[s + 1] < sg[s]) return BITSMOE_ERR_BLOB;
@@ -459,7 +503,7 @@ int unpack_image(const uint8_t* img, size_t bytes, bitsmoe_layer_host_out* dst) 
         for (int g = 0; g < ng; ++g)
           for (int s = 0; s < bd.count; ++s) {
             const int j = unit[bd.slot0 + s];
-            const uint32_t v = sz[(size_t)g * bd.nslots + s];
+            const uint32_t v = sz[(size_t)g * x.nslots + s];
             dst->scale[(he * n + j) * ng + g] = (uint16_t)(v & 0xFFFF);
             dst->zero[(he * n + j) * ng + g] = (uint16_t)(v >> 16);
           }
