@@ -82,13 +82,15 @@ struct Fwd {
   int T, k, P;
   int s16;          // K2 smem row stride (int16 elements)
   int rbc;          // K3 row blocks per block
-  int decode;       // small-batch mode: routing computed in each kernel, prologue staging
+  int decode;       // small-batch mode: routing published once, prologue staging
+  int accum;        // output basis adds into y (residual) instead of writing it
   int seg_bytes;    // largest gate/up item (bytes of codes in one row block)
   int ul_bytes;     // largest down item (bytes of one tile over rbc row blocks)
   const uint16_t* x;
   const float* logits;
   float* y;
   int* status;
+  int* route_flag;  // decode mode: set once the routing below is published
   int* pair_expert;
   float* pair_weight;
   int* expert_count;
@@ -181,6 +183,23 @@ __device__ __forceinline__ void stage_bytes(void* dst, const uint8_t* src, uint3
     o += c;
   }
 }
+__device__ __forceinline__ int ld_acquire(const int* ptr) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(ptr) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_release(int* ptr, int v) {
+  asm volatile("st.release.gpu.global.b32 [%0], %1;" ::"l"(ptr), "r"(v) : "memory");
+}
+// Bounded wait (about one second of SM clock) for a flag published by another block.
+__device__ __forceinline__ bool wait_flag(const int* flag) {
+  const long long t0 = clock64();
+  while (ld_acquire(flag) == 0) {
+    if (clock64() - t0 > (2ll << 30)) return false;
+    __nanosleep(64);
+  }
+  return true;
+}
 __device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 __device__ __forceinline__ float f16lo(uint32_t w) {
@@ -238,6 +257,8 @@ __device__ RouteView route_block(const Fwd& p, uint32_t* sm) {
   for (int i = tid; i < T * E; i += nt) {
     const int t = i / E, e = i - t * E;
     const uint32_t key = keys[i];
+    // the logit back from its key (the key map is a bijection on non-NaN floats)
+    const float logit = __uint_as_float((key & 0x80000000u) ? (key & 0x7FFFFFFFu) : ~key);
     const uint32_t* row = keys + t * E;
     int rank = 0;
     if ((E & 3) == 0 && ((t * E) & 3) == 0) {
@@ -259,7 +280,7 @@ __device__ RouteView route_block(const Fwd& p, uint32_t* sm) {
     }
     if (rank < k) {
       pe[t * k + rank] = e;
-      pw[t * k + rank] = p.logits[i];
+      pw[t * k + rank] = key ? logit : __int_as_float(0x7FC00000);   // key 0: NaN logit
     }
   }
   __syncthreads();
@@ -309,6 +330,165 @@ __device__ RouteView route_block(const Fwd& p, uint32_t* sm) {
   }
   __syncthreads();
   return RouteView{pe, pw, cnt, start, act, plist};
+}
+
+// ---------------------------------------------------------------------------
+// Pre-norm of a stacked MoE block: r = h / sqrt(mean(h^2) + eps) (unit weight),
+// x = bf16(r), router logits = W_r x (fp32 accumulate).  Each block computes a
+// slice of the experts' logits; its warps load their router rows in the PDL
+// prologue, before waiting for the kernel that produced h.  It lets the next
+// kernel launch only once x and the logits are written.
+// ---------------------------------------------------------------------------
+struct NormArgs {
+  const float* h;
+  const uint16_t* w;
+  float eps;
+  int T, D, E, D_pad8;
+  uint16_t* x;
+  float* logits;
+};
+
+template <int TB>
+__global__ void __launch_bounds__(kThreads) k_norm_router(NormArgs a) {
+  extern __shared__ float4 smem_nr[];
+  float* xs = reinterpret_cast<float*>(smem_nr);          // [TB][D_pad8] bf16-rounded r
+  float* red = xs + (size_t)TB * a.D_pad8;                 // [kWarps][TB]
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  const int nch = a.D >> 3;                                // 16-byte chunks of a row (D % 8 == 0)
+  const int row0 = blockIdx.x * kWarps + wid;
+  const int nrw = gridDim.x * kWarps;
+  uint4 pre[8];
+  if (row0 < a.E) {
+    const uint4* rp = reinterpret_cast<const uint4*>(a.w + (size_t)row0 * a.D);
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int c = u * 32 + lane;
+      pre[u] = c < nch ? ldg_stream(rp + c) : make_uint4(0, 0, 0, 0);
+    }
+  }
+  pdl_wait();
+  for (int t0 = 0; t0 < a.T; t0 += TB) {
+    const int tb = min(TB, a.T - t0);
+    __syncthreads();
+    float ss[TB];
+#pragma unroll
+    for (int tt = 0; tt < TB; ++tt) ss[tt] = 0.f;
+    for (int d = threadIdx.x; d < a.D; d += blockDim.x)
+#pragma unroll
+      for (int tt = 0; tt < TB; ++tt)
+        if (tt < tb) {
+          const float v = a.h[(size_t)(t0 + tt) * a.D + d];
+          ss[tt] = fmaf(v, v, ss[tt]);
+        }
+#pragma unroll
+    for (int tt = 0; tt < TB; ++tt) {
+      const float v = warp_sum(ss[tt]);
+      if (lane == 0) red[wid * TB + tt] = v;
+    }
+    __syncthreads();
+    float inv[TB];
+#pragma unroll
+    for (int tt = 0; tt < TB; ++tt) {
+      float sum = 0.f;
+      for (int w = 0; w < kWarps; ++w) sum += red[w * TB + tt];
+      inv[tt] = rsqrtf(sum / (float)a.D + a.eps);
+    }
+    for (int i = threadIdx.x; i < TB * a.D; i += blockDim.x) {
+      const int tt = i / a.D, d = i - tt * a.D;
+      float r = 0.f;
+      if (tt < tb) {
+        float iv = inv[0];
+#pragma unroll
+        for (int u = 1; u < TB; ++u)
+          if (u == tt) iv = inv[u];
+        // round to bf16 (nearest even): both the MoE input and the router use it
+        uint32_t u32 = __float_as_uint(a.h[(size_t)(t0 + tt) * a.D + d] * iv);
+        u32 = (u32 + 0x7FFFu + ((u32 >> 16) & 1u)) & 0xFFFF0000u;
+        r = __uint_as_float(u32);
+        if (blockIdx.x == 0) a.x[(size_t)(t0 + tt) * a.D + d] = (uint16_t)(u32 >> 16);
+      }
+      xs[tt * a.D_pad8 + d] = r;
+    }
+    __syncthreads();
+    for (int row = row0; row < a.E; row += nrw) {
+      const uint4* rp = reinterpret_cast<const uint4*>(a.w + (size_t)row * a.D);
+      float acc[TB];
+#pragma unroll
+      for (int tt = 0; tt < TB; ++tt) acc[tt] = 0.f;
+      for (int c0 = 0; c0 < nch; c0 += 256) {
+        uint4 v[8];
+        if (row == row0 && c0 == 0 && t0 == 0) {
+#pragma unroll
+          for (int u = 0; u < 8; ++u) v[u] = pre[u];
+        } else {
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const int c = c0 + u * 32 + lane;
+            v[u] = c < nch ? ldg_stream(rp + c) : make_uint4(0, 0, 0, 0);
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int c = c0 + u * 32 + lane;
+          if (c < nch) {
+            const float w0 = bf16lo(v[u].x), w1 = bf16hi(v[u].x), w2 = bf16lo(v[u].y), w3 = bf16hi(v[u].y);
+            const float w4 = bf16lo(v[u].z), w5 = bf16hi(v[u].z), w6 = bf16lo(v[u].w), w7 = bf16hi(v[u].w);
+#pragma unroll
+            for (int tt = 0; tt < TB; ++tt) {
+              const float4* xv = reinterpret_cast<const float4*>(xs + tt * a.D_pad8 + c * 8);
+              const float4 xa = xv[0], xb = xv[1];
+              float r = acc[tt];
+              r = fmaf(w0, xa.x, r); r = fmaf(w1, xa.y, r); r = fmaf(w2, xa.z, r); r = fmaf(w3, xa.w, r);
+              r = fmaf(w4, xb.x, r); r = fmaf(w5, xb.y, r); r = fmaf(w6, xb.z, r); r = fmaf(w7, xb.w, r);
+              acc[tt] = r;
+            }
+          }
+        }
+      }
+#pragma unroll
+      for (int tt = 0; tt < TB; ++tt) acc[tt] = warp_sum(acc[tt]);
+      if (lane == 0)
+#pragma unroll
+        for (int tt = 0; tt < TB; ++tt)
+          if (tt < tb) a.logits[(size_t)(t0 + tt) * a.E + row] = acc[tt];
+    }
+  }
+  __syncthreads();
+  __threadfence();
+  pdl_trigger();   // only now: the next kernels read x and the logits in their prologues
+}
+
+// ---------------------------------------------------------------------------
+// Decode-mode router: first kernel of the chain.  It lets the projection
+// kernel launch at once, then routes while the memory system is still idle
+// (the logits load is not queued behind the basis streams) and publishes the
+// routing with a release flag that the gate/up and down kernels wait on.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads) k_route_publish(Fwd p) {
+  if (threadIdx.x == 0) {   // before the trigger: no later kernel may see the previous call's flag
+    p.status[0] = 0;
+    p.route_flag[0] = 0;
+    __threadfence();
+  }
+  __syncthreads();
+  pdl_trigger();
+  extern __shared__ uint32_t smem_rp[];
+  const RouteView rv = route_block(p, smem_rp);
+  for (int i = threadIdx.x; i < p.P; i += blockDim.x) {
+    p.pair_expert[i] = rv.pe[i];
+    p.pair_weight[i] = rv.pw[i];
+    p.pair_list[i] = rv.plist[i];
+  }
+  for (int i = threadIdx.x; i <= p.E; i += blockDim.x) {
+    if (i < p.E) p.expert_count[i] = rv.cnt[i];
+    p.expert_start[i] = rv.start[i];
+    p.active[i] = rv.act[i];
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    st_release(p.route_flag, 1);
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -557,7 +737,7 @@ __global__ void __launch_bounds__(kThreads) k_gemv(Fwd p) {
               const int h = row >= p.n, j = row - h * p.n;
               p.z[((size_t)h * p.T + t) * p.n_pad + j] = acc[tt];
             } else {
-              p.y[(size_t)t * p.D + row] = acc[tt];
+              p.y[(size_t)t * p.D + row] = p.accum ? p.y[(size_t)t * p.D + row] + acc[tt] : acc[tt];
             }
           }
         }
@@ -604,7 +784,6 @@ __global__ void __launch_bounds__(kThreads) k_gemv_bulk(Fwd p, int stage_rows) {
     for (int st = 0; st < min(2, nst); ++st) issue(st);
   }
   if (PROJ) {
-    if (p.decode && blockIdx.x == 0 && threadIdx.x == 0) *p.status = 0;
     const size_t ng = (size_t)p.P * 2 * p.I_pad / 4, ns = (size_t)p.T * p.n_pad / 4;
     const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
     for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < ng + ns; i += (size_t)gridDim.x * blockDim.x) {
@@ -682,7 +861,7 @@ __global__ void __launch_bounds__(kThreads) k_gemv_bulk(Fwd p, int stage_rows) {
                 const int h = row >= p.n, j = row - h * p.n;
                 p.z[((size_t)h * p.T + t) * p.n_pad + j] = acc[tt];
               } else {
-                p.y[(size_t)t * p.D + row] = acc[tt];
+                p.y[(size_t)t * p.D + row] = p.accum ? p.y[(size_t)t * p.D + row] + acc[tt] : acc[tt];
               }
             }
           }
@@ -697,6 +876,7 @@ __global__ void __launch_bounds__(kThreads) k_gemv_bulk(Fwd p, int stage_rows) {
     pdl_wait();
     prefetch_for_experts(p);
   }
+  if (PROJ && p.decode) pdl_wait();   // (a preceding kernel, if any, completes before this grid)
 }
 
 // ---------------------------------------------------------------------------
@@ -1198,6 +1378,7 @@ __global__ void __launch_bounds__(kThreads) k_down(Fwd p) {
 // griddepcontrol.wait only the data dependency (z, gate/up) remains.
 // ---------------------------------------------------------------------------
 constexpr int kK2DecWarps = 4;
+constexpr int kDecMaxT = 8;        // decode mode: at most this many tokens
 constexpr int kZ = 12;             // item slots per lane whose z values are gathered at once
 constexpr int kK3DecWarps = 4;
 
@@ -1205,35 +1386,40 @@ template <int G, int TB>
 __global__ void __launch_bounds__(kK2DecWarps * 32) k_gateup_dec(Fwd p) {
   pdl_trigger();
   extern __shared__ int4 smem_k2d[];
-  uint32_t* rsm = reinterpret_cast<uint32_t*>(smem_k2d);
-  const int rwords = (route_words(p.T, p.E, p.P) + 3) & ~3;
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
   const int smax = p.s16 - 8;                      // slots of the largest item, multiple of 8
   const size_t per_warp = (size_t)p.seg_bytes + (size_t)smax * 4 * (2 + G) + (size_t)G * TB * p.s16 * 2 + 16;
-  uint8_t* codes = reinterpret_cast<uint8_t*>(rsm + rwords) + wid * per_warp;
+  uint8_t* codes = reinterpret_cast<uint8_t*>(smem_k2d) + wid * per_warp;
   int* su = reinterpret_cast<int*>(codes + p.seg_bytes);           // unit index per local slot
   float* sa = reinterpret_cast<float*>(su + smax);                 // alpha
   uint32_t* ssz = reinterpret_cast<uint32_t*>(sa + smax);          // [G][smax] scale | zero << 16
   int16_t* cq = reinterpret_cast<int16_t*>(ssz + G * smax);        // [G][TB][s16]
   uint64_t* bar = reinterpret_cast<uint64_t*>(codes + per_warp - 16);
-  const RouteView rv = route_block(p, rsm);
-  const int A = rv.act[0];
   const int per_e = 2 * p.NRB * p.nseg;
   const int item = blockIdx.x * kK2DecWarps + wid;
+  const int a = item / per_e;
+  // the routing, published by the projection kernel's first block
+  if (!wait_flag(p.route_flag)) {
+    if (lane == 0) atomicCAS(p.status, 0, BITSMOE_ERR_TIMEOUT);
+    pdl_wait();
+    return;
+  }
+  const int A = p.active[0];
+  const int e_raw = p.active[1 + min(a, p.E - 1)];
   // every warp waits for the previous kernel before it exits, so that this
   // grid completes only after it (PDL completion is then transitive)
   if (item >= A * per_e) {
     pdl_wait();
     return;
   }
-  const int a = item / per_e;
   int r = item - a * per_e;
   const int h = r / (p.NRB * p.nseg);
   r -= h * p.NRB * p.nseg;
   const int rb = r / p.nseg, sg = r - rb * p.nseg;
-  const int e = rv.act[1 + a];
+  const int e = e_raw;
   const ExpertDesc& xd = p.desc[h * p.E + e];
   const ItemRec it = p.items[((size_t)h * p.E + e) * p.nseg + sg];
+  const int ntok = p.expert_count[e], pst = p.expert_start[e];
   if (it.nr == 0) {
     pdl_wait();
     return;
@@ -1250,13 +1436,15 @@ __global__ void __launch_bounds__(kK2DecWarps * 32) k_gateup_dec(Fwd p) {
     for (int gl = 0; gl < G; ++gl)
       bulk_g2s(ssz + gl * smax, p.img + xd.sz_off + ((size_t)(g_base + gl) * xd.nslots + it.slot0) * 4, mb, bar);
   }
+  int plist[kDecMaxT];   // the expert's (token, slot) pairs
+#pragma unroll
+  for (int q = 0; q < kDecMaxT; ++q) plist[q] = q < ntok ? p.pair_list[pst + q] : 0;
   pdl_wait();
   // ranges: consecutive buckets, quantised ones first, 16-bit last
   int nls = 0;
   for (int q = 0; q < it.nr; ++q)
     if (it.bits[q] < 16) nls += it.ntl[q] * rl_units(it.bits[q]);
   const int gl_lane = G == 1 ? 0 : (4 * lane) / p.group;
-  const int ntok = rv.cnt[e], pst = rv.start[e];
   const int tstride = p.s16 / 2;
   if (!mbar_wait(bar, 0)) {
     if (lane == 0) atomicCAS(p.status, 0, BITSMOE_ERR_TIMEOUT);
@@ -1269,7 +1457,12 @@ __global__ void __launch_bounds__(kK2DecWarps * 32) k_gateup_dec(Fwd p) {
     const float* zrow[TB];
 #pragma unroll
     for (int tt = 0; tt < TB; ++tt) {
-      pair[tt] = rv.plist[pst + tb0 + min(tt, tb - 1)];
+      const int q = tb0 + min(tt, tb - 1);
+      int pv = plist[0];
+#pragma unroll
+      for (int u = 1; u < kDecMaxT; ++u)
+        if (u == q) pv = plist[u];
+      pair[tt] = pv;
       zrow[tt] = p.z + ((size_t)h * p.T + pair[tt] / p.k) * p.n_pad;
     }
     // c = alpha * z * scale per (slot, group, token): int16 with one scale per token.
@@ -1422,13 +1615,11 @@ template <int G, int TB>
 __global__ void __launch_bounds__(kK3DecWarps * 32) k_down_dec(Fwd p) {
   pdl_trigger();
   extern __shared__ int4 smem_k3d[];
-  uint32_t* rsm = reinterpret_cast<uint32_t*>(smem_k3d);
-  const int rwords = (route_words(p.T, p.E, p.P) + 3) & ~3;
   const int rbc = p.rbc;
   const int nrows_max = rbc * kRows;
   const int gshift = 31 - __clz(p.group);
   const int ngc_max = max(1, nrows_max >> gshift);
-  float* hf = reinterpret_cast<float*>(rsm + rwords);                  // [TB][nrows_max]
+  float* hf = reinterpret_cast<float*>(smem_k3d);                      // [TB][nrows_max]
   int16_t* hq = reinterpret_cast<int16_t*>(hf + TB * nrows_max);       // [TB][nrows_max]
   int* Hg = reinterpret_cast<int*>(hq + TB * nrows_max);               // [TB][64]
   float* red = reinterpret_cast<float*>(Hg + TB * 64);                 // [warps][TB]
@@ -1438,19 +1629,23 @@ __global__ void __launch_bounds__(kK3DecWarps * 32) k_down_dec(Fwd p) {
   uint8_t* codes = reinterpret_cast<uint8_t*>(shs + ((TB + 3) & ~3)) + wid * per_warp;
   uint32_t* szs = reinterpret_cast<uint32_t*>(codes + p.ul_bytes);
   uint64_t* bar = reinterpret_cast<uint64_t*>(codes + per_warp - 16);
-  const RouteView rv = route_block(p, rsm);
-  const int A = rv.act[0];
   const int ntg = (p.ul_max_tiles + kK3DecWarps - 1) / kK3DecWarps;
   const int nrc = (p.NRB + rbc - 1) / rbc;
   const int item = blockIdx.x;
+  const int a = item / (ntg * nrc);
+  if (!wait_flag(p.route_flag)) {   // the routing, published by the projection kernel
+    if (threadIdx.x == 0) atomicCAS(p.status, 0, BITSMOE_ERR_TIMEOUT);
+    pdl_wait();
+    return;
+  }
+  const int A = p.active[0];
+  const int e = p.active[1 + min(a, p.E - 1)];
   if (item >= A * ntg * nrc) {   // wait before exiting: keeps PDL completion transitive
     pdl_wait();
     return;
   }
-  const int a = item / (ntg * nrc);
   const int r = item - a * ntg * nrc;
   const int tg = r / nrc, rc = r - tg * nrc;
-  const int e = rv.act[1 + a];
   const ExpertDesc& xd = p.desc[2 * p.E + e];
   if (tg * kK3DecWarps >= xd.ntiles) {
     pdl_wait();
@@ -1491,8 +1686,14 @@ __global__ void __launch_bounds__(kK3DecWarps * 32) k_down_dec(Fwd p) {
       }
     }
   }
+  const int ntok = p.expert_count[e], pst = p.expert_start[e];
+  int plist[kDecMaxT];
+  float pwt[kDecMaxT];
+#pragma unroll
+  for (int q = 0; q < kDecMaxT; ++q) plist[q] = q < ntok ? p.pair_list[pst + q] : 0;
+#pragma unroll
+  for (int q = 0; q < kDecMaxT; ++q) pwt[q] = q < ntok ? p.pair_weight[plist[q]] : 0.f;
   pdl_wait();
-  const int ntok = rv.cnt[e], pst = rv.start[e];
   bool staged = false;
   constexpr int kMaxRowsPerThread = kK3MaxRB * kRows / (kK3DecWarps * 32);
   for (int tb0 = 0; tb0 < ntok; tb0 += TB) {
@@ -1511,7 +1712,10 @@ __global__ void __launch_bounds__(kK3DecWarps * 32) k_down_dec(Fwd p) {
       for (int tt = 0; tt < TB; ++tt) {
         float v = 0.f;
         if (i < nrows && tt < tb) {
-          const int pr = rv.plist[pst + tb0 + tt];
+          int pr = plist[0];
+#pragma unroll
+          for (int u = 1; u < kDecMaxT; ++u)
+            if (u == tb0 + tt) pr = plist[u];
           const float g = p.gu[((size_t)pr * 2) * p.I_pad + row0 + i];
           const float u = p.gu[((size_t)pr * 2 + 1) * p.I_pad + row0 + i];
           v = g / (1.f + __expf(-g)) * u;
@@ -1580,9 +1784,16 @@ __global__ void __launch_bounds__(kK3DecWarps * 32) k_down_dec(Fwd p) {
 #pragma unroll
       for (int tt = 0; tt < TB; ++tt) {
         if (tt < tb) {
-          const int pr = rv.plist[pst + tb0 + tt];
+          int pr = plist[0];
+          float wv = pwt[0];
+#pragma unroll
+          for (int u = 1; u < kDecMaxT; ++u)
+            if (u == tb0 + tt) {
+              pr = plist[u];
+              wv = pwt[u];
+            }
           const float scale = shs[tt] * (1.f / 32767.f);
-          atomicAdd(p.s + (size_t)(pr / p.k) * p.n_pad + j, rv.pw[pr] * al * scale * accf[tt]);
+          atomicAdd(p.s + (size_t)(pr / p.k) * p.n_pad + j, wv * al * scale * accf[tt]);
         }
       }
     }
@@ -1702,7 +1913,7 @@ int launch_gemv_bulk_tb(bool proj, const Fwd& p, int sms, cudaStream_t st, bool 
   const int nrows = proj ? 2 * p.n : p.D;
   const size_t row_bytes = (size_t)ld * 2;
   const size_t vec = (size_t)TB * ld * 4;
-  const size_t budget = vec < 150 * 1024 ? 200 * 1024 - vec : 48 * 1024;
+  const size_t budget = proj ? 64 * 1024 : (vec < 150 * 1024 ? 200 * 1024 - vec : 48 * 1024);
   const int grid = std::min(nrows, sms);
   const int per = (nrows + grid - 1) / grid;
   int stage_rows = (int)std::max<size_t>(1, std::min<size_t>((budget / 2) / row_bytes, (size_t)(per + 1) / 2));
@@ -1749,7 +1960,7 @@ template <int G, int TB>
 int launch_k2k3_dec(const Fwd& p, int A_max, int sms, cudaStream_t st, bool pdl,
                     const std::function<int()>& between) {
   int rc;
-  const size_t rbytes = (size_t)((route_words(p.T, p.E, p.P) + 3) & ~3) * 4;
+  const size_t rbytes = 0;
   const size_t smax = (size_t)p.s16 - 8;
   const size_t pw2 = (size_t)p.seg_bytes + smax * 4 * (2 + G) + (size_t)G * TB * p.s16 * 2 + 16;
   const size_t sm2 = rbytes + kK2DecWarps * pw2;
@@ -1777,8 +1988,42 @@ int launch_k2k3_tb(const Fwd& p, int sms, cudaStream_t st, bool pdl, const std::
 
 bool aligned(const void* ptr, size_t a) { return ((uintptr_t)ptr % a) == 0; }
 
+template <int TB>
+int launch_norm_router_tb(const NormArgs& a, int sms, cudaStream_t st) {
+  const size_t smem = (size_t)TB * a.D_pad8 * 4 + kWarps * TB * 4;
+  int rc;
+  if ((rc = set_smem(k_norm_router<TB>, smem))) return rc;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(std::max(1, std::min((a.E + kWarps - 1) / kWarps, sms)));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  BM_CK(cudaLaunchKernelEx(&cfg, k_norm_router<TB>, a));
+  return BITSMOE_OK;
+}
+
+int launch_norm_router(const NormArgs& a, int sms, cudaStream_t st) {
+  if (a.T <= 1) return launch_norm_router_tb<1>(a, sms, st);
+  if (a.T <= 2) return launch_norm_router_tb<2>(a, sms, st);
+  if (a.T <= 4) return launch_norm_router_tb<4>(a, sms, st);
+  return launch_norm_router_tb<8>(a, sms, st);
+}
+
+int num_sms_current(int* sms) {
+  int dev = 0;
+  BM_CK(cudaGetDevice(&dev));
+  BM_CK(cudaDeviceGetAttribute(sms, cudaDevAttrMultiProcessorCount, dev));
+  return BITSMOE_OK;
+}
+
+
 int forward_impl(const void* x, const float* logits, int T, int top_k, const bitsmoe_layer* L, float* y,
-                 void* ws, size_t ws_bytes, cudaStream_t st, cudaEvent_t* ev = nullptr) {
+                 void* ws, size_t ws_bytes, cudaStream_t st, cudaEvent_t* ev = nullptr, bool accum = false) {
   const ImageHeader& hd = L->hd();
   const bool pdl = ev == nullptr;   // profiling runs the phases back to back without overlap
   const WsLayout w = ws_layout(hd, T, top_k);
@@ -1810,7 +2055,9 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
   p.x = static_cast<const uint16_t*>(x);
   p.logits = logits;
   p.y = y;
+  p.accum = accum ? 1 : 0;
   p.status = reinterpret_cast<int*>(wb + w.status);
+  p.route_flag = p.status + 1;
   p.pair_expert = reinterpret_cast<int*>(wb + w.pair_expert);
   p.pair_weight = reinterpret_cast<float*>(wb + w.pair_weight);
   p.expert_count = reinterpret_cast<int*>(wb + w.expert_count);
@@ -1829,9 +2076,12 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
   const int G = std::max(1, kRows / hd.group);
   if (p.decode) {
     const int A_max = std::min(hd.E, p.P);
+    const size_t rsm = (size_t)route_words(p.T, hd.E, p.P) * 4 + 16;
     if ((rc = mark(0))) return rc;
+    if ((rc = set_smem(k_route_publish, rsm))) return rc;
+    if ((rc = launch(k_route_publish, dim3(1), dim3(kThreads), rsm, st, false, p))) return rc;
     if ((rc = mark(1))) return rc;
-    if ((rc = launch_gemv_bulk(true, p, sms, st, false))) return rc;
+    if ((rc = launch_gemv_bulk(true, p, sms, st, pdl))) return rc;
     if ((rc = mark(2))) return rc;
     std::function<int()> between = ev ? std::function<int()>([&]() { return mark(3); }) : std::function<int()>();
     if (T == 1) {
@@ -2096,6 +2346,44 @@ int bitsmoe_profile_forward(const void* x, const float* logits, int T, int top_k
   for (int i = 0; i < 6; ++i)
     if (ev[i]) cudaEventDestroy(ev[i]);
   return rc;
+}
+
+int bitsmoe_rmsnorm_router(const float* h, const void* w_router, float eps, int T, int D, int E, void* x_out,
+                           float* logits_out, void* stream) {
+  if (T < 0 || D < 8 || D % 8 || E < 1 || E > 1024 || !(eps >= 0.f)) return BITSMOE_ERR_INVALID_ARG;
+  if ((int64_t)T * D > (1ll << 31) || D > (1 << 16)) return BITSMOE_ERR_SHAPE;
+  if (T == 0) return BITSMOE_OK;
+  if (!h || !w_router || !x_out || !logits_out) return BITSMOE_ERR_INVALID_ARG;
+  if (!aligned(h, 16) || !aligned(w_router, 16) || !aligned(x_out, 16) || !aligned(logits_out, 16))
+    return BITSMOE_ERR_ALIGNMENT;
+  int sms = 0, rc = num_sms_current(&sms);
+  if (rc) return rc;
+  NormArgs a{h, static_cast<const uint16_t*>(w_router), eps, T, D, E, (D + 7) / 8 * 8,
+             static_cast<uint16_t*>(x_out), logits_out};
+  return launch_norm_router(a, sms, static_cast<cudaStream_t>(stream));
+}
+
+int bitsmoe_moe_block_forward(float* h, const void* w_router, float eps, int T, int top_k, const bitsmoe_layer* L,
+                              void* ws, size_t ws_bytes, void* stream) {
+  if (!L || T < 0 || !(eps >= 0.f)) return BITSMOE_ERR_INVALID_ARG;
+  const ImageHeader& hd = L->hd();
+  if (top_k < 1 || top_k > std::min(hd.E, 32)) return BITSMOE_ERR_INVALID_ARG;
+  if ((int64_t)T * top_k > 24576 || (int64_t)T * hd.D > (1ll << 31) || hd.D % 8 || hd.D > (1 << 16))
+    return BITSMOE_ERR_SHAPE;
+  if (T == 0) return BITSMOE_OK;
+  if (!h || !w_router || !ws) return BITSMOE_ERR_INVALID_ARG;
+  if (!aligned(h, 16) || !aligned(w_router, 16) || !aligned(ws, 256)) return BITSMOE_ERR_ALIGNMENT;
+  const WsLayout w = ws_layout(hd, T, top_k);
+  if (ws_bytes < w.total) return BITSMOE_ERR_WORKSPACE_TOO_SMALL;
+  int rc = check_device(L);
+  if (rc) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  uint8_t* wb = static_cast<uint8_t*>(ws);
+  NormArgs a{h, static_cast<const uint16_t*>(w_router), eps, T, hd.D, hd.E, hd.D_pad,
+             reinterpret_cast<uint16_t*>(wb + w.x_stage), reinterpret_cast<float*>(wb + w.logits_stage)};
+  if ((rc = launch_norm_router(a, L->num_sms, st))) return rc;
+  return forward_impl(wb + w.x_stage, reinterpret_cast<const float*>(wb + w.logits_stage), T, top_k, L, h, ws,
+                      ws_bytes, st, nullptr, true);
 }
 
 int bitsmoe_last_device_status(void* ws, void* stream) {

@@ -11,10 +11,15 @@ Mixtral-8x7B, plus a tiny layer); no model weights or datasets are used.
 Recipe (one ``numpy.random.Generator`` per layer, draws in this order):
 
 1. three shared bases Phi_h (h = gate, up, down), each the Q factor of a QR
-   decomposition of an N(0, 1/D) D x n matrix, rounded to bf16;
+   decomposition of an N(0, 1/D) D x n matrix, rounded to bf16 (layers of the
+   48-layer stack instead use a random signed permutation times four random
+   Householder reflections: also exactly orthonormal, and cheap enough to
+   draw 48 layers);
 2. per-unit bit-widths b[h, e, j] i.i.d. from the config's distribution;
-3. integer codes uniform on [0, 2^b) for every element of every unit
-   (b = 16 units instead hold fp16 values drawn N(0, 1/I));
+3. integer codes uniform on [0, 2^b) for every element of every unit: the low
+   b bits of 16-bit words cut from SplitMix64 outputs (Steele, Lea, Flood 2014)
+   of the counter key(seed, layer) + i, computed block by block in threads
+   (b = 16 units instead hold fp16 values drawn N(0, 1/I) from the layer generator);
 4. per (unit, group) fp16 scale 2*sqrt(3/I)/(2^b - 1) * U(0.75, 1.25) and fp16
    zero (2^b - 1)/2 + U(-0.5, 0.5) (so dequantised units have about unit norm,
    like the paper's normalised spectral vectors, while every group differs);
@@ -28,6 +33,8 @@ from __future__ import annotations
 
 import dataclasses
 import math
+import os
+from concurrent.futures import ThreadPoolExecutor
 from typing import Dict, Optional, Sequence, Tuple
 
 import numpy as np
@@ -100,15 +107,41 @@ def f32_to_f16_bits(a: np.ndarray) -> np.ndarray:
     return np.ascontiguousarray(a, dtype=np.float16).view(np.uint16)
 
 
-def _draw_basis(rng: np.random.Generator, D: int, n: int) -> np.ndarray:
-    g = rng.standard_normal((D, n)) / math.sqrt(D)
-    q, _ = np.linalg.qr(g)          # D x n, orthonormal columns
+def _draw_basis(rng: np.random.Generator, D: int, n: int, method: str = "qr") -> np.ndarray:
+    if method == "qr":
+        g = rng.standard_normal((D, n)) / math.sqrt(D)
+        q, _ = np.linalg.qr(g)          # D x n, orthonormal columns
+    else:                               # signed permutation x 4 Householder reflections
+        q = np.zeros((D, n))
+        q[rng.permutation(D)[:n], np.arange(n)] = rng.choice([-1.0, 1.0], size=n)
+        for _ in range(4):
+            v = rng.standard_normal(D)
+            v /= np.linalg.norm(v)
+            q -= 2.0 * np.outer(v, v @ q)
     return f32_to_bf16_bits(q.astype(np.float32))
+
+
+_SM_GOLDEN = np.uint64(0x9E3779B97F4A7C15)
+_SM_C1 = np.uint64(0xBF58476D1CE4E5B9)
+_SM_C2 = np.uint64(0x94D049BB133111EB)
+
+
+def splitmix64(counter: np.ndarray) -> np.ndarray:
+    """SplitMix64 output for each 64-bit counter value (wrapping arithmetic)."""
+    with np.errstate(over="ignore"):
+        z = counter * _SM_GOLDEN
+        z ^= z >> np.uint64(30)
+        z *= _SM_C1
+        z ^= z >> np.uint64(27)
+        z *= _SM_C2
+        z ^= z >> np.uint64(31)
+    return z
 
 
 def make_layer(spec: LayerSpec, seed: int = 0, layer_index: int = 0,
                alpha_scale: float = 1.0,
-               bits_dist: Optional[Dict[int, float]] = None) -> Dict[str, np.ndarray]:
+               bits_dist: Optional[Dict[int, float]] = None,
+               basis_method: Optional[str] = None) -> Dict[str, np.ndarray]:
     """Draw one packed-format layer as host arrays.
 
     Returns a dict with
@@ -125,7 +158,8 @@ def make_layer(spec: LayerSpec, seed: int = 0, layer_index: int = 0,
         raise ValueError("I must be a multiple of group")
     ng = I // group
     rng = np.random.default_rng([seed, layer_index, 17])
-    basis = np.stack([_draw_basis(rng, D, n) for _ in range(3)])
+    method = basis_method or ("householder" if spec.layers > 1 else "qr")
+    basis = np.stack([_draw_basis(rng, D, n, method) for _ in range(3)])
 
     dist = _dist(bits_dist) if bits_dist is not None else spec.bits_dist
     vals = np.array([b for b, _ in dist], dtype=np.uint8)
@@ -133,9 +167,21 @@ def make_layer(spec: LayerSpec, seed: int = 0, layer_index: int = 0,
     probs = probs / probs.sum()
     bits = vals[rng.choice(len(vals), size=(3, E, n), p=probs)]
 
-    codes = rng.integers(0, 1 << 16, size=(3, E, n, I), dtype=np.uint16)
+    # codes: SplitMix64 words of a per-layer counter, cut into 16-bit pieces and
+    # masked to b bits; blocks of one (projection, expert) drawn in threads
+    codes = np.empty((3, E, n, I), dtype=np.uint16)
     mask = np.where(bits >= 16, 0xFFFF, (1 << bits.astype(np.uint32)) - 1).astype(np.uint16)
-    codes &= mask[..., None]
+    words = (n * I + 3) // 4
+    key = int(np.random.SeedSequence([seed, layer_index, 19]).generate_state(1, np.uint64)[0])
+
+    def _draw(q):
+        h, e = divmod(q, E)
+        ctr = np.arange(words, dtype=np.uint64) + np.uint64((key + q * words) % (1 << 64))
+        blk = splitmix64(ctr).view(np.uint16)[: n * I].reshape(n, I)
+        codes[h, e] = blk & mask[h, e][:, None]
+
+    with ThreadPoolExecutor(max_workers=min(16, os.cpu_count() or 1)) as ex:
+        list(ex.map(_draw, range(3 * E)))
     sixteen = bits == 16
     if sixteen.any():
         cnt = int(sixteen.sum())
