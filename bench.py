@@ -47,7 +47,7 @@ METRIC = "MoE-layer decode tokens/s at 2.0 avg bits; achieved HBM GB/s vs ~8 TB/
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
 PHASES = ["route", "basis_proj_gate_up", "gate_up_factors", "down_factor_sum", "out_basis"]
-KERNELS_PER_FORWARD = 5
+KERNELS_PER_FORWARD = 5   # router, projection, gate/up, down, output basis
 
 
 def measured_peaks():
@@ -198,10 +198,139 @@ def config_of(spec, T, args):
             "l2": f"rotating {args.copies} packed layer copies (>> 129 MB L2)", "seed": 0}
 
 
+def run_stack(args, spec, T, torch, bm, dev, rank, world, local):
+    """48-layer pre-norm MoE FFN stack: a step feeds one batch of hidden states
+    through every block (RMSNorm + router + quantized MoE + residual)."""
+    eps = 1e-6
+    layers, routers, moved = [None] * spec.layers, [], []
+    pend = []
+
+    def pack(l, host):
+        layers[l] = bm.bitsmoe_pack(host, device=local)
+
+    for l in range(spec.layers):
+        host = synth.make_layer(spec, seed=0, layer_index=l)
+        th = threading.Thread(target=pack, args=(l, host))
+        th.start()
+        pend.append(th)
+        routers.append(torch.from_numpy(synth.make_router_weight(spec, seed=0, layer_index=l).view(np.int16)).to(dev))
+        if len(pend) > 1:
+            pend.pop(0).join()
+    for th in pend:
+        th.join()
+    for L in layers:
+        moved.append(np.array([L.expert_moved_bytes(e) for e in range(spec.E)], dtype=np.float64))
+    k = spec.top_k
+    NI = 8
+    h0 = [torch.from_numpy(synth.make_hidden(spec, T, seed=0, step=i)).to(dev) for i in range(NI)]
+    h = torch.empty((T, spec.D), dtype=torch.float32, device=dev)
+    ws = bm.Workspace(layers[0], T, k, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def step(i, st):
+        h.copy_(h0[i % NI])
+        for l in range(spec.layers):
+            bm.bitsmoe_moe_block_forward(h.data_ptr(), routers[l].data_ptr(), eps, T, k, layers[l], ws.ptr,
+                                         ws.nbytes, st.cuda_stream)
+
+    # realised routing of step 0, layer by layer (outside the timed region): byte accounting
+    x = torch.empty((T, spec.D), dtype=torch.int16, device=dev)
+    lg = torch.empty((T, spec.E), dtype=torch.float32, device=dev)
+    step_bytes = 0.0
+    with torch.cuda.stream(stream):
+        h.copy_(h0[0])
+        for l in range(spec.layers):
+            bm.bitsmoe_rmsnorm_router(h.data_ptr(), routers[l].data_ptr(), eps, T, spec.D, spec.E, x.data_ptr(),
+                                      lg.data_ptr(), stream.cuda_stream)
+            stream.synchronize()
+            used = np.unique(host_route(lg.cpu().numpy(), k))
+            # bases, routed experts' factors, router matrix, hidden state in and out
+            step_bytes += (3.0 * spec.D * spec.n * 2 + moved[l][used].sum() + spec.E * spec.D * 2 +
+                           2.0 * T * spec.D * 4)
+            bm.bitsmoe_moe_block_forward(h.data_ptr(), routers[l].data_ptr(), eps, T, k, layers[l], ws.ptr,
+                                         ws.nbytes, stream.cuda_stream)
+    stream.synchronize()
+    with torch.cuda.stream(stream):
+        for i in range(min(args.warmup, 3)):
+            step(i, stream)
+    stream.synchronize()
+    G = max(1, min(args.graph // spec.layers or 1, args.steps))
+    graphs = {}
+
+    def capture(n, off):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for i in range(n):
+                step(off + i, stream)
+        return g
+
+    nfull, rem = divmod(args.steps, G)
+    g_main = capture(G, 0)
+    g_rem = capture(rem, 0) if rem else None
+    with torch.cuda.stream(stream):
+        for _ in range(max(1, args.warmup // G)):
+            g_main.replay()
+    stream.synchronize()
+    clk = ClockSampler(local)
+    clk.start()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clk.mark("t0")
+    e0.record(stream)
+    with torch.cuda.stream(stream):
+        for _ in range(nfull):
+            g_main.replay()
+        if g_rem is not None:
+            g_rem.replay()
+    e1.record(stream)
+    e1.synchronize()
+    clk.mark("t1")
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    clocks = clk.stop()
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+    value = world * args.steps * T / (ms / 1e3)
+    gbs = step_bytes * args.steps / (ms / 1e3) / 1e9
+    peaks, peak_src = measured_peaks()
+    peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    # e2e: host hidden state in, host hidden state out, every step
+    hh = torch.from_numpy(synth.make_hidden(spec, T, seed=0, step=0)).pin_memory()
+    ho = torch.empty((T, spec.D), dtype=torch.float32).pin_memory()
+    ne = max(3, min(args.steps, 50))
+    t0 = time.perf_counter()
+    for i in range(ne):
+        with torch.cuda.stream(stream):
+            h.copy_(hh, non_blocking=True)
+            for l in range(spec.layers):
+                bm.bitsmoe_moe_block_forward(h.data_ptr(), routers[l].data_ptr(), eps, T, k, layers[l], ws.ptr,
+                                             ws.nbytes, stream.cuda_stream)
+            ho.copy_(h, non_blocking=True)
+        stream.synchronize()
+    e2e_s = time.perf_counter() - t0
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": dict(config_of(spec, T, args), layers=spec.layers, l2="48 distinct layers per step (>> L2)"),
+        "hbm_gbs": gbs, "hbm_frac_of_8tbs": gbs / NOMINAL_HBM_GBS, "hbm_frac_of_measured": gbs / peak,
+        "bytes_per_step": step_bytes,
+        "e2e": {"value": world * ne * T / e2e_s, "unit": "tokens/s", "steps": ne,
+                "h2d_bytes_per_step": T * spec.D * 4, "d2h_bytes_per_step": T * spec.D * 4},
+        "clocks": clocks, "gpu_launches": args.steps * spec.layers * (KERNELS_PER_FORWARD + 1),
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20000)
+    ap.add_argument("--steps", type=int, default=None, help="default 20000 (one layer), 400 (layer stack)")
     ap.add_argument("--warmup", type=int, default=200)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="qw3")
@@ -213,6 +342,8 @@ def main():
     args = ap.parse_args()
     spec = synth.WORKLOADS[args.workload]
     T = args.tokens or spec.tokens[0]
+    if args.steps is None:
+        args.steps = 20000 if spec.layers == 1 else 400
     if args.impl == "reference":
         run_reference(args, spec, T)
         return
@@ -227,6 +358,13 @@ def main():
         dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
+
+    if spec.layers > 1:
+        run_stack(args, spec, T, torch, bm, dev, rank, world, local)
+        if world > 1:
+            torch.distributed.barrier()
+            torch.distributed.destroy_process_group()
+        return
 
     # ---- workload: one generated layer, packed once, uploaded as rotating copies
     layer = synth.make_layer(spec, seed=0)

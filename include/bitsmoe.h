@@ -162,6 +162,27 @@ int bitsmoe_moe_forward_host(const void* x_host, const float* logits_host, int T
                              const bitsmoe_layer* layer, float* y_host,
                              void* ws, size_t ws_bytes, void* stream);
 
+/* Pre-norm of one MoE block of a decoder stack (the 48-layer MoE FFN stack
+ * workload; attention is outside this library):
+ *   r = h / sqrt(mean_d h^2 + eps)  (RMSNorm with unit weight), x = bf16(r),
+ *   logits = W_r x  (fp32 accumulation of bf16 products).
+ *   h          device, T x D fp32 (row-major), 16-byte aligned
+ *   w_router   device, E x D bf16 bit patterns, row e = router row of expert e
+ *   x_out      device, T x D bf16 bit patterns (written)
+ *   logits_out device, T x E fp32 (written)
+ * D must be a multiple of 8 (<= 65536), E <= 1024.  Asynchronous on `stream`.
+ * The routing rule of the paper's MoE layers is the host model's; this is the
+ * common pre-norm + linear router of the evaluated models. */
+int bitsmoe_rmsnorm_router(const float* h, const void* w_router, float eps, int T, int D, int E,
+                           void* x_out, float* logits_out, void* stream);
+
+/* One pre-norm MoE block in place: h += MoE(x, logits) with x, logits from
+ * bitsmoe_rmsnorm_router(h, w_router, eps) and MoE the quantised MoE-layer
+ * forward of `layer`.  Workspace and errors as bitsmoe_moe_forward (the
+ * normalised activations and logits live in the workspace).  Asynchronous. */
+int bitsmoe_moe_block_forward(float* h, const void* w_router, float eps, int T, int top_k,
+                              const bitsmoe_layer* layer, void* ws, size_t ws_bytes, void* stream);
+
 /* Profiling variant of bitsmoe_moe_forward (same arguments and results): the
  * five phases run without overlap, each bracketed by CUDA events on `stream`,
  * and the call synchronises.  phase_ms[0..4] receive the durations of

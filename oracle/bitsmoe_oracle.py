@@ -210,6 +210,11 @@ def rms_norm(h: np.ndarray, eps: float = 1e-6) -> np.ndarray:
     return h / np.sqrt(np.mean(h * h, axis=-1, keepdims=True) + eps)
 
 
+def router_logits(w_router_bits: np.ndarray, x_bits: np.ndarray) -> np.ndarray:
+    """Router logits W_r x of a stacked MoE block (W_r: E x D bf16 bits, x: T x D bf16 bits)."""
+    return bf16_bits_to_f64(x_bits) @ bf16_bits_to_f64(w_router_bits).T
+
+
 # ----------------------------------------------------------------------------
 # Offline pieces used by the pins (not on the hot path)
 # ----------------------------------------------------------------------------

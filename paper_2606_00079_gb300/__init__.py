@@ -57,6 +57,8 @@ SIGNATURES = {
     "bitsmoe_moe_forward": (_I, [_P, _P, _I, _I, _P, _P, _P, _SZ, _P]),
     "bitsmoe_moe_forward_host": (_I, [_P, _P, _I, _I, _P, _P, _P, _SZ, _P]),
     "bitsmoe_moe_forward_noalloc": (_I, [_P, _P, _I, _I, _P, _P, _P]),
+    "bitsmoe_rmsnorm_router": (_I, [_P, _P, ctypes.c_float, _I, _I, _I, _P, _P, _P]),
+    "bitsmoe_moe_block_forward": (_I, [_P, _P, ctypes.c_float, _I, _I, _P, _P, _SZ, _P]),
     "bitsmoe_last_device_status": (_I, [_P, _P]),
     "bitsmoe_free": (None, [_P]),
     "bitsmoe_strerror": (ctypes.c_char_p, [_I]),
@@ -251,6 +253,18 @@ def bitsmoe_moe_forward_noalloc(x_ptr: int, logits_ptr: int, T: int, top_k: int,
     calls on that device, so overlapping calls race)."""
     _check(_lib().bitsmoe_moe_forward_noalloc(x_ptr, logits_ptr, T, top_k, layer.handle, y_ptr, stream),
            "bitsmoe_moe_forward_noalloc")
+
+
+def bitsmoe_rmsnorm_router(h_ptr: int, w_router_ptr: int, eps: float, T: int, D: int, E: int,
+                           x_out_ptr: int, logits_out_ptr: int, stream: int = 0) -> None:
+    _check(_lib().bitsmoe_rmsnorm_router(h_ptr, w_router_ptr, eps, T, D, E, x_out_ptr, logits_out_ptr, stream),
+           "bitsmoe_rmsnorm_router")
+
+
+def bitsmoe_moe_block_forward(h_ptr: int, w_router_ptr: int, eps: float, T: int, top_k: int, layer: Layer,
+                              ws_ptr: int, ws_bytes: int, stream: int = 0) -> None:
+    _check(_lib().bitsmoe_moe_block_forward(h_ptr, w_router_ptr, eps, T, top_k, layer.handle, ws_ptr, ws_bytes,
+                                            stream), "bitsmoe_moe_block_forward")
 
 
 def bitsmoe_profile_forward(x_ptr: int, logits_ptr: int, T: int, top_k: int, layer: Layer, y_ptr: int,

@@ -12,13 +12,14 @@ Recipe (one ``numpy.random.Generator`` per layer, draws in this order):
 
 1. three shared bases Phi_h (h = gate, up, down), each the Q factor of a QR
    decomposition of an N(0, 1/D) D x n matrix, rounded to bf16 (layers of the
-   48-layer stack instead use a random signed permutation times four random
-   Householder reflections: also exactly orthonormal, and cheap enough to
-   draw 48 layers);
+   48-layer stack instead use a random signed permutation times two random
+   Householder reflections: also orthonormal, dense, and cheap enough to draw
+   48 layers);
 2. per-unit bit-widths b[h, e, j] i.i.d. from the config's distribution;
 3. integer codes uniform on [0, 2^b) for every element of every unit: the low
-   b bits of 16-bit words cut from SplitMix64 outputs (Steele, Lea, Flood 2014)
-   of the counter key(seed, layer) + i, computed block by block in threads
+   b bits of 4-bit (blocks whose units have at most 4 bits) or 16-bit fields
+   cut from SplitMix64 outputs (Steele, Lea, Flood 2014) of the counter
+   key(seed, layer) + i, computed block by block in threads
    (b = 16 units instead hold fp16 values drawn N(0, 1/I) from the layer generator);
 4. per (unit, group) fp16 scale 2*sqrt(3/I)/(2^b - 1) * U(0.75, 1.25) and fp16
    zero (2^b - 1)/2 + U(-0.5, 0.5) (so dequantised units have about unit norm,
@@ -111,13 +112,13 @@ def _draw_basis(rng: np.random.Generator, D: int, n: int, method: str = "qr") ->
     if method == "qr":
         g = rng.standard_normal((D, n)) / math.sqrt(D)
         q, _ = np.linalg.qr(g)          # D x n, orthonormal columns
-    else:                               # signed permutation x 4 Householder reflections
-        q = np.zeros((D, n))
+    else:                               # signed permutation x 2 Householder reflections
+        q = np.zeros((D, n), dtype=np.float32)
         q[rng.permutation(D)[:n], np.arange(n)] = rng.choice([-1.0, 1.0], size=n)
-        for _ in range(4):
+        for _ in range(2):
             v = rng.standard_normal(D)
-            v /= np.linalg.norm(v)
-            q -= 2.0 * np.outer(v, v @ q)
+            v = (v / np.linalg.norm(v)).astype(np.float32)
+            q -= np.outer(2.0 * v, v @ q)
     return f32_to_bf16_bits(q.astype(np.float32))
 
 
@@ -177,7 +178,15 @@ def make_layer(spec: LayerSpec, seed: int = 0, layer_index: int = 0,
     def _draw(q):
         h, e = divmod(q, E)
         ctr = np.arange(words, dtype=np.uint64) + np.uint64((key + q * words) % (1 << 64))
-        blk = splitmix64(ctr).view(np.uint16)[: n * I].reshape(n, I)
+        if int(bits[h, e].max()) <= 4:   # 4-bit fields: 16 codes per word
+            ctr = ctr[: (n * I + 15) // 16]
+            by = splitmix64(ctr).view(np.uint8)
+            nib = np.empty(2 * by.size, dtype=np.uint8)
+            nib[0::2] = by & 15
+            nib[1::2] = by >> 4
+            blk = nib[: n * I].reshape(n, I).astype(np.uint16)
+        else:                            # 16-bit fields: 4 codes per word
+            blk = splitmix64(ctr).view(np.uint16)[: n * I].reshape(n, I)
         codes[h, e] = blk & mask[h, e][:, None]
 
     with ThreadPoolExecutor(max_workers=min(16, os.cpu_count() or 1)) as ex:

@@ -1,0 +1,94 @@
+"""48-layer Qwen3-30B-A3B-shaped MoE FFN stack (pre-norm blocks, RMSNorm with unit
+weight between layers, linear router), decode batch 1 and 32.
+
+Parity is layer-local: for sampled layers the oracle takes the GPU's own input
+hidden state h_in, and checks (1) x = bf16(RMSNorm(h_in)) to within one bf16
+ulp, (2) the router logits W_r x, (3) the block's update h_out - h_in against
+the oracle MoE forward on the GPU's x and logits (bar 2e-3 of its max).
+"""
+import threading
+
+import numpy as np
+import pytest
+
+import oracle
+import synth
+
+pytestmark = pytest.mark.gpu
+EPS = 1e-6
+SAMPLED = (0, 1, 23, 47)
+
+
+@pytest.fixture(scope="module")
+def stack():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2606_00079_gb300 as bm
+    torch.cuda.set_device(0)
+    spec = synth.WORKLOADS["qw3_stack"]
+    layers, kept, routers = [None] * spec.layers, {}, []
+    lock = threading.Lock()
+    pending = []
+
+    def pack(l, host):
+        L = bm.bitsmoe_pack(host, device=0)
+        with lock:
+            layers[l] = L
+
+    for l in range(spec.layers):   # draw layer l while layer l-1 is packed
+        host = synth.make_layer(spec, seed=0, layer_index=l)
+        if l in SAMPLED:
+            kept[l] = host
+        th = threading.Thread(target=pack, args=(l, host))
+        th.start()
+        pending.append(th)
+        routers.append(torch.from_numpy(synth.make_router_weight(spec, seed=0, layer_index=l).view(np.int16)).cuda())
+        if len(pending) > 1:
+            pending.pop(0).join()
+    for th in pending:
+        th.join()
+    return torch, bm, spec, layers, kept, routers
+
+
+@pytest.mark.parametrize("T", [1, 32])
+def test_stack_layer_local_parity(stack, T):
+    torch, bm, spec, layers, kept, routers = stack
+    k = spec.top_k
+    h = torch.from_numpy(synth.make_hidden(spec, T, seed=0, step=0)).cuda()
+    ws = bm.Workspace(layers[0], T, k)
+    x = torch.empty((T, spec.D), dtype=torch.int16, device="cuda")
+    lg = torch.empty((T, spec.E), dtype=torch.float32, device="cuda")
+    st = torch.cuda.current_stream().cuda_stream
+    saved = {}
+    for l in range(spec.layers):
+        if l in SAMPLED:
+            h_in = h.clone()
+            bm.bitsmoe_rmsnorm_router(h_in.data_ptr(), routers[l].data_ptr(), EPS, T, spec.D, spec.E,
+                                      x.data_ptr(), lg.data_ptr(), st)
+        bm.bitsmoe_moe_block_forward(h.data_ptr(), routers[l].data_ptr(), EPS, T, k, layers[l], ws.ptr,
+                                     ws.nbytes, st)
+        if l in SAMPLED:
+            torch.cuda.synchronize()
+            saved[l] = (h_in.cpu().numpy().astype(np.float64), x.cpu().numpy().view(np.uint16).copy(),
+                        lg.cpu().numpy().copy(), h.cpu().numpy().astype(np.float64))
+    torch.cuda.synchronize()
+    assert np.isfinite(h.cpu().numpy()).all()
+    for l, (h_in, xg, lgg, h_out) in saved.items():
+        # (1) RMSNorm, rounded to bf16: at most one bf16 ulp from the fp64 value rounded
+        r = oracle.rms_norm(h_in, EPS)
+        xr = oracle.bf16_bits_to_f64(synth.f32_to_bf16_bits(r.astype(np.float32)))
+        xv = oracle.bf16_bits_to_f64(xg)
+        ulp = np.abs(xr) * 2.0 ** -7 + 1e-30
+        assert np.all(np.abs(xv - xr) <= ulp * 1.01), l
+        assert np.mean(xv != xr) < 0.01, l
+        # (2) router logits on the GPU's x
+        lr = oracle.router_logits(synth.make_router_weight(spec, seed=0, layer_index=l), xg)
+        assert np.max(np.abs(lgg - lr)) <= 1e-4 * np.max(np.abs(lr)), l
+        # (3) the block's update against the oracle MoE forward of that layer
+        y_ref = oracle.moe_forward_factored(kept[l], xg, lgg, k)
+        y_gpu = h_out - h_in
+        err = np.max(np.abs(y_gpu - y_ref)) / np.max(np.abs(y_ref))
+        assert err <= 2e-3, (l, err)

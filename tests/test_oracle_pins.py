@@ -358,3 +358,16 @@ def test_factor_matrix_matches_per_unit_definition():
                 col = oracle.dequantize_unit(int(layer["bits"][h, e, k]), layer["codes"][h, e, k],
                                              layer["scale"][h, e, k], layer["zero"][h, e, k], spec.group)
                 np.testing.assert_array_equal(P[:, k], col)
+
+
+def test_rms_norm_closed_forms():
+    # constant rows: r = c / sqrt(c^2 + eps) exactly
+    for c in (3.0, -0.5, 1e-3):
+        h = np.full((1, 64), c)
+        np.testing.assert_allclose(oracle.rms_norm(h, 1e-6), c / math.sqrt(c * c + 1e-6), rtol=1e-14)
+    # any row: mean(r^2) = m / (m + eps) with m = mean(h^2); scale invariance for eps = 0
+    h = np.random.default_rng(3).standard_normal((5, 100))
+    m = np.mean(h * h, axis=1)
+    r = oracle.rms_norm(h, 1e-2)
+    np.testing.assert_allclose(np.mean(r * r, axis=1), m / (m + 1e-2), rtol=1e-12)
+    np.testing.assert_allclose(oracle.rms_norm(7.0 * h, 0.0), oracle.rms_norm(h, 0.0), rtol=1e-12)
