@@ -255,7 +255,6 @@ def run_stack(args, spec, T, torch, bm, dev, rank, world, local):
             step(i, stream)
     stream.synchronize()
     G = max(1, min(args.graph // spec.layers or 1, args.steps))
-    graphs = {}
 
     def capture(n, off):
         g = torch.cuda.CUDAGraph()
