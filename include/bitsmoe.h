@@ -138,6 +138,15 @@ int bitsmoe_expert_moved_bytes(const bitsmoe_layer* layer, int e, uint64_t out[3
  * top_k; 0 if the arguments are invalid. */
 size_t bitsmoe_workspace_bytes(const bitsmoe_layer* layer, int T, int top_k);
 
+/* Kernels one bitsmoe_moe_forward call launches for (T, top_k) on this layer
+ * (no counterpart in the paper: for callers that capture the forward into a
+ * CUDA graph or count launches).  A single token runs as a one-block prep
+ * kernel plus one fused persistent kernel (2) when the layer's per-block
+ * shares of the bases and factors fit in shared memory; otherwise the forward
+ * is a chain of 5 kernels.  Returns a negative error code for invalid
+ * arguments. */
+int bitsmoe_forward_launches(const bitsmoe_layer* layer, int T, int top_k);
+
 /* The quantised MoE-layer forward, asynchronous on `stream`:
  *   x       device, T x D bf16 bit patterns (row-major), 16-byte aligned
  *   logits  device, T x E fp32 router logits (row-major), 16-byte aligned
@@ -187,7 +196,9 @@ int bitsmoe_moe_block_forward(float* h, const void* w_router, float eps, int T, 
  * five phases run without overlap, each bracketed by CUDA events on `stream`,
  * and the call synchronises.  phase_ms[0..4] receive the durations of
  * routing, shared-basis projection (gate, up), gate/up factors + SwiGLU
- * inputs, down factor + weighted expert sum, output basis. */
+ * inputs, down factor + weighted expert sum, output basis.  When the forward
+ * runs as one fused kernel (see bitsmoe_forward_launches), its phases cannot
+ * be separated: phase_ms[0] receives the whole forward and the others 0. */
 int bitsmoe_profile_forward(const void* x, const float* logits, int T, int top_k,
                             const bitsmoe_layer* layer, float* y,
                             void* ws, size_t ws_bytes, void* stream, float phase_ms[5]);

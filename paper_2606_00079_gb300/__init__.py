@@ -54,6 +54,7 @@ SIGNATURES = {
     "bitsmoe_expert_moved_bytes": (_I, [_P, _I, ctypes.POINTER(ctypes.c_uint64)]),
     "bitsmoe_profile_forward": (_I, [_P, _P, _I, _I, _P, _P, _P, _SZ, _P, ctypes.POINTER(ctypes.c_float)]),
     "bitsmoe_workspace_bytes": (_SZ, [_P, _I, _I]),
+    "bitsmoe_forward_launches": (_I, [_P, _I, _I]),
     "bitsmoe_moe_forward": (_I, [_P, _P, _I, _I, _P, _P, _P, _SZ, _P]),
     "bitsmoe_moe_forward_host": (_I, [_P, _P, _I, _I, _P, _P, _P, _SZ, _P]),
     "bitsmoe_moe_forward_noalloc": (_I, [_P, _P, _I, _I, _P, _P, _P]),
@@ -224,6 +225,14 @@ def bitsmoe_unpack(layer: Layer) -> Dict:
 
 def bitsmoe_workspace_bytes(layer: Layer, T: int, top_k: int) -> int:
     return int(_lib().bitsmoe_workspace_bytes(layer.handle, T, top_k))
+
+
+def bitsmoe_forward_launches(layer: Layer, T: int, top_k: int) -> int:
+    """Kernels one forward call launches (2: prep + fused single-token kernel; 5: the chain)."""
+    n = int(_lib().bitsmoe_forward_launches(layer.handle, T, top_k))
+    if n < 0:
+        raise BitsMoEError(n, "bitsmoe_forward_launches")
+    return n
 
 
 def bitsmoe_moe_forward(x_ptr: int, logits_ptr: int, T: int, top_k: int, layer: Layer, y_ptr: int,

@@ -1,7 +1,8 @@
 """Build libbitsmoe.so in-tree with nvcc for sm_103a (GB300).
 
-Two translation units, compiled in parallel: the host packer (pack.cpp, plain
-C++) and the CUDA kernels + C ABI (forward.cu).  The CUDA runtime is linked
+Three translation units, compiled in parallel: the host packer (pack.cpp,
+plain C++), the CUDA kernel chain + C ABI (forward.cu) and the fused
+single-token decode kernel (fused.cu).  The CUDA runtime is linked
 statically, so the library loads on a machine without a GPU (the host-only
 entry points then work; the device ones return BITSMOE_ERR_CUDA).
 """
@@ -36,7 +37,7 @@ def _run(cmd):
 
 
 def sources():
-    return [os.path.join(CSRC, f) for f in ("pack.cpp", "forward.cu")]
+    return [os.path.join(CSRC, f) for f in ("pack.cpp", "forward.cu", "fused.cu")]
 
 
 def up_to_date() -> bool:

@@ -7,6 +7,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <vector>
+
 #include "internal.h"
 
 namespace bmoe {
@@ -41,6 +43,56 @@ struct Fwd {
   float* gu;        // [P][2][I_pad]
   float* s;         // [T][n_pad]
 };
+
+// Staging records of the fused single-token kernel, derived from the image
+// when a layer is uploaded (flat image offsets, so that a block finds every
+// copy of a work item with one vector load).
+struct CStage {            // one per gate/up item (h < 2, e, segment)
+  uint64_t code0;          // image offset of the item's code bytes in row block 0
+  uint64_t unit0, alpha0;  // image offsets of its slots' unit indices and alphas
+  uint64_t sz0;            // image offset of its first slot's scale/zero in group row 0
+  uint32_t rb_stride;      // bytes between row blocks of the code stream
+  uint32_t sz_row;         // bytes between group rows of the scale/zero matrix
+  uint32_t bytes;          // code bytes per row block (0: empty item)
+  uint32_t mb;             // bytes of the slot arrays (4 per slot)
+  uint16_t nls;            // quantised slots (the 16-bit ones come last)
+  uint8_t nr;              // buckets the item touches
+  uint8_t bits[kNumBk];    // their bit-widths
+  uint16_t ntl[kNumBk];    // tiles per touched bucket
+  uint8_t pad_[8];
+};
+static_assert(sizeof(CStage) == 80, "CStage layout");
+
+struct DStage {            // one per down tile (e, tile < ul_max_tiles)
+  uint64_t code;           // image offset of the tile's codes over all row blocks
+  uint64_t unit, alpha;    // image offsets of its 32 unit indices and alphas
+  uint64_t sz;             // image offset of its first slot's scale/zero in group row 0
+  uint32_t sz_row;         // bytes between group rows
+  uint32_t bits;           // 0: the expert has no tile of this index
+  uint32_t pad_[2];
+};
+static_assert(sizeof(DStage) == 48, "DStage layout");
+
+// Fused single-token decode kernel (fused.cu): workspace pointers and the
+// shared-memory plan chosen on the host.
+struct FusedArgs {
+  uint32_t* cnt;     // [4] grid-barrier counters
+  const CStage* cst; // [2][E][nseg]
+  const DStage* dst; // [E][ul_max_tiles]
+  int b_per, b_stage, b_nst, e_per;     // basis rows per block, rows per stage, stages; output rows per block
+  int nslot_c, slot_c, nslot_d, slot_d; // gate/up and down staging slots (count, bytes)
+  int off_route, off_xs, off_r1, off_d, off_rc, off_cq, off_rec, smem;
+  int smax, s16, seg_al, ul_max_tiles, d_code_bytes, d_h_bytes;
+};
+
+// Shared-memory plan of the fused kernel for this layer, or false when the
+// layer does not fit it (then the kernel chain runs).
+bool fused_plan(const ImageHeader& hd, int T, int top_k, int seg_bytes, int ul_max_chunks, int s16, int sms,
+                FusedArgs* f);
+// Prep kernel + fused kernel on `st` (grid = sms blocks).
+cudaError_t launch_fused(const Fwd& p, const FusedArgs& f, int sms, cudaStream_t st, bool pdl);
+// Staging records of a packed image (host side, at upload).
+void build_stage_tables(const uint8_t* img, std::vector<CStage>& cst, std::vector<DStage>& dst);
 
 }  // namespace bmoe
 
@@ -134,6 +186,9 @@ __device__ __forceinline__ void stage_bytes(void* dst, const uint8_t* src, uint3
     bulk_g2s(static_cast<uint8_t*>(dst) + o, src + o, c, bar);
     o += c;
   }
+}
+__device__ __forceinline__ void fence_proxy_async() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 __device__ __forceinline__ int ld_acquire(const int* ptr) {
   int v;

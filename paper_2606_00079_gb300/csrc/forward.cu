@@ -1418,7 +1418,9 @@ __global__ void __launch_bounds__(kK3DecWarps * 32) k_down_dec(Fwd p) {
 // ---------------------------------------------------------------------------
 struct WsLayout {
   size_t status, pair_expert, pair_weight, expert_count, expert_start, pair_list, active, z, gu, s;
-  size_t x_stage, logits_stage, y_stage, total;
+  size_t x_stage, logits_stage, y_stage;
+  size_t sync, hq, hsc, hsum;   // fused decode kernel
+  size_t total;
 };
 
 WsLayout ws_layout(const ImageHeader& hd, int T, int k) {
@@ -1443,6 +1445,11 @@ WsLayout ws_layout(const ImageHeader& hd, int T, int k) {
   w.x_stage = take((size_t)T * hd.D * 2);
   w.logits_stage = take((size_t)T * hd.E * 4);
   w.y_stage = take((size_t)T * hd.D * 4);
+  const size_t G = std::max(1, kRows / hd.group);
+  w.sync = take((4 + (size_t)hd.E * hd.NRB) * 4);
+  w.hq = take(P * hd.I_pad * 2);
+  w.hsc = take(P * hd.NRB * 4);
+  w.hsum = take(P * hd.NRB * G * 4);
   w.total = off;
   return w;
 }
@@ -1687,6 +1694,21 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
     return BITSMOE_OK;
   };
   const int G = std::max(1, kRows / hd.group);
+  FusedArgs fa;
+  if (p.decode && fused_plan(hd, T, top_k, L->seg_bytes, L->ul_max_chunks, p.s16, sms, &fa)) {
+    // one token: the whole layer in one persistent kernel (after a one-block prep kernel)
+    fa.cnt = reinterpret_cast<uint32_t*>(wb + w.sync);
+    fa.ctr = fa.cnt + 4;
+    fa.hq = reinterpret_cast<int16_t*>(wb + w.hq);
+    fa.hsc = reinterpret_cast<float*>(wb + w.hsc);
+    fa.hsum = reinterpret_cast<int*>(wb + w.hsum);
+    if ((rc = mark(0))) return rc;
+    const cudaError_t e = launch_fused(p, fa, hd.E * hd.NRB, sms, st, pdl);
+    if (e != cudaSuccess) return cuda_fail(e);
+    for (int i = 1; i <= 5; ++i)
+      if ((rc = mark(i))) return rc;
+    return BITSMOE_OK;
+  }
   if (p.decode) {
     const int A_max = std::min(hd.E, p.P);
     const size_t rsm = (size_t)route_words(p.T, hd.E, p.P) * 4 + 16;
@@ -1885,6 +1907,18 @@ int bitsmoe_expert_moved_bytes(const bitsmoe_layer* L, int e, uint64_t out[3]) {
   const ExpertDesc* d = L->desc();
   for (int h = 0; h < 3; ++h) out[h] = d[h * hd.E + e].moved;
   return BITSMOE_OK;
+}
+
+int bitsmoe_forward_launches(const bitsmoe_layer* L, int T, int top_k) {
+  if (!L || T < 0) return BITSMOE_ERR_INVALID_ARG;
+  const ImageHeader& hd = L->hd();
+  if (top_k < 1 || top_k > std::min(hd.E, 32)) return BITSMOE_ERR_INVALID_ARG;
+  if (T == 0) return 0;
+  const bool decode = T <= 8 && T * hd.E <= 4096;
+  FusedArgs fa;
+  const int s16 = (int)align_up(std::max(hd.seg_max_slots, 8), 64) + 8;
+  if (decode && fused_plan(hd, T, top_k, L->seg_bytes, L->ul_max_chunks, s16, L->num_sms, &fa)) return 2;
+  return 5;
 }
 
 size_t bitsmoe_workspace_bytes(const bitsmoe_layer* L, int T, int top_k) {

@@ -1,0 +1,157 @@
+"""GPU parity of the fused single-token decode kernel (prep kernel + one
+persistent kernel with grid barriers) against the fp64 oracle.
+
+The fused path runs whenever T == 1 and the layer's per-block shares fit in
+shared memory; these cases check that it was taken and cover every bit-width,
+group size, evicted units and experts, extreme top-k, consecutive calls and
+different layers on one workspace, a workspace full of garbage (the prep
+kernel must reset what the kernel's barriers count on), and replay from a CUDA
+graph.  Bar: max|y_gpu - y_ref| / ||y_ref||_inf <= 2e-3.
+"""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+
+pytestmark = pytest.mark.gpu
+TOL = 2e-3
+ALL_BITS = {0: 0.1, 1: 0.15, 2: 0.2, 3: 0.15, 4: 0.1, 6: 0.1, 8: 0.1, 16: 0.1}
+
+
+@pytest.fixture(scope="module")
+def env():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2606_00079_gb300 as bm
+    torch.cuda.set_device(0)
+    return torch, bm
+
+
+def rel_err(y, ref):
+    return float(np.max(np.abs(y - ref)) / max(np.max(np.abs(ref)), 1e-30))
+
+
+def small(**kw):
+    base = dict(D=96, E=4, I=256, n=72, group=64, top_k=2)
+    base.update(kw)
+    return synth.scaled_spec(synth.WORKLOADS["tiny"], **base)
+
+
+def run(env, L, x, logits, k, ws=None):
+    torch, bm = env
+    assert bm.bitsmoe_forward_launches(L, x.shape[0], k) == 2, "fused path not taken"
+    xd = torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).cuda()
+    ld = torch.from_numpy(np.ascontiguousarray(logits)).cuda()
+    if ws is None:
+        ws = bm.Workspace(L, x.shape[0], k)
+    y = bm.moe_forward(L, xd, ld, k, ws=ws)
+    torch.cuda.synchronize()
+    assert bm.bitsmoe_last_device_status(ws.ptr) == 0
+    return y.cpu().numpy().astype(np.float64)
+
+
+def check(env, layer, x, logits, k, L=None, ws=None):
+    torch, bm = env
+    L = L or bm.bitsmoe_pack(layer, device=0)
+    y = run(env, L, x, logits, k, ws)
+    ref = oracle.moe_forward_factored(layer, x, logits, k)
+    err = rel_err(y, ref)
+    assert err <= TOL, err
+    return y, ref
+
+
+@pytest.mark.parametrize("b", [1, 2, 3, 4, 6, 8, 16])
+def test_fused_uniform_bit_width(env, b):
+    spec = small(n=70)
+    layer = synth.make_layer(spec, seed=b, bits_dist={b: 1.0}, alpha_scale=3.0)
+    x, logits = synth.make_inputs(spec, 1, seed=b)
+    check(env, layer, x, logits, spec.top_k)
+
+
+@pytest.mark.parametrize("group,I", [(32, 96), (64, 256), (128, 384), (256, 512)])
+def test_fused_all_bit_widths_and_groups(env, group, I):
+    spec = small(group=group, I=I, n=75, D=100, E=8, top_k=3)
+    layer = synth.make_layer(spec, seed=group, bits_dist=ALL_BITS, alpha_scale=4.0)
+    x, logits = synth.make_inputs(spec, 1, seed=group)
+    check(env, layer, x, logits, spec.top_k)
+
+
+def test_fused_evicted_units_and_experts(env):
+    spec = small()
+    layer = synth.make_layer(spec, seed=5, bits_dist=ALL_BITS, alpha_scale=3.0)
+    layer["bits"][:, 1, :] = 0            # expert 1 fully evicted
+    layer["bits"][0, 2, :] = 0            # gate of expert 2 evicted: h = 0
+    x, logits = synth.make_inputs(spec, 1, seed=5)
+    for route in ((1, 2), (1, 3), (2, 0)):
+        lg = logits.copy()
+        lg[0, list(route)] += 10.0
+        check(env, layer, x, lg, spec.top_k)
+
+
+def test_fused_top1_and_all_experts(env):
+    spec = small(E=6)
+    layer = synth.make_layer(spec, seed=9, bits_dist=ALL_BITS, alpha_scale=3.0)
+    x, _ = synth.make_inputs(spec, 1, seed=9)
+    logits = np.array([[1.0, 2.0, 2.0, -1.0, 2.0, 0.0]], np.float32)   # ties
+    torch, bm = env
+    L = bm.bitsmoe_pack(layer, device=0)
+    for k in (1, 2, spec.E):
+        check(env, layer, x, logits, k, L=L)
+
+
+def test_fused_consecutive_calls_layers_and_garbage_workspace(env):
+    torch, bm = env
+    spec = synth.scaled_spec(synth.WORKLOADS["qw3"], D=512, E=32, I=384, n=512, top_k=4)
+    layers = [synth.make_layer(spec, seed=s) for s in (21, 22)]
+    Ls = [bm.bitsmoe_pack(l, device=0) for l in layers]
+    ws = bm.Workspace(Ls[0], 1, spec.top_k)
+    ws.buf.fill_(0xA5)                    # garbage: counters and status must be reset per call
+    for step in range(6):
+        i = step % 2
+        x, logits = synth.make_inputs(spec, 1, seed=3, step=step)
+        check(env, layers[i], x, logits, spec.top_k, L=Ls[i], ws=ws)
+
+
+def test_fused_graph_replay(env):
+    torch, bm = env
+    spec = synth.scaled_spec(synth.WORKLOADS["qw3"], D=512, E=32, I=384, n=512, top_k=4)
+    layer = synth.make_layer(spec, seed=31)
+    L = bm.bitsmoe_pack(layer, device=0)
+    ws = bm.Workspace(L, 1, spec.top_k)
+    xd = torch.zeros((1, spec.D), dtype=torch.int16, device="cuda")
+    ld = torch.zeros((1, spec.E), dtype=torch.float32, device="cuda")
+    ys = [torch.zeros((1, spec.D), dtype=torch.float32, device="cuda") for _ in range(3)]
+    stream = torch.cuda.Stream()
+    with torch.cuda.stream(stream):        # warm-up outside the capture
+        bm.moe_forward(L, xd, ld, spec.top_k, ws=ws, y=ys[0], stream=stream)
+    stream.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for y in ys:                       # three forwards back to back in one graph
+            bm.moe_forward(L, xd, ld, spec.top_k, ws=ws, y=y, stream=stream)
+    for step in range(3):
+        x, logits = synth.make_inputs(spec, 1, seed=4, step=step)
+        xd.copy_(torch.from_numpy(x.view(np.int16)))
+        ld.copy_(torch.from_numpy(logits))
+        g.replay()
+        torch.cuda.synchronize()
+        ref = oracle.moe_forward_factored(layer, x, logits, spec.top_k)
+        for y in ys:
+            assert rel_err(y.cpu().numpy().astype(np.float64), ref) <= TOL
+    assert bm.bitsmoe_last_device_status(ws.ptr) == 0
+
+
+def test_fused_plan_taken_for_qw3_dims_not_for_d4096(env):
+    torch, bm = env
+    qw3 = synth.scaled_spec(synth.WORKLOADS["qw3"], E=8, top_k=8)   # full qw3 dims, fewer experts
+    L = bm.bitsmoe_pack(synth.make_layer(qw3, seed=1), device=0)
+    assert bm.bitsmoe_forward_launches(L, 1, 8) == 2
+    assert bm.bitsmoe_forward_launches(L, 2, 8) == 5
+    # D = n = 4096: a block's share of the input bases (54 rows of 8 KB) exceeds shared memory
+    big = synth.scaled_spec(synth.WORKLOADS["mixtral"], E=2, I=128, top_k=1)
+    Lb = bm.bitsmoe_pack(synth.make_layer(big, seed=1), device=0)
+    assert bm.bitsmoe_forward_launches(Lb, 1, 1) == 5
