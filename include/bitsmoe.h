@@ -50,6 +50,7 @@ extern "C" {
 #define BITSMOE_ERR_TIMEOUT            -8  /* a bounded device-side wait ran out                  */
 #define BITSMOE_ERR_DEVICE_BOUNDS      -9  /* a device-side bounds check failed (access skipped) */
 #define BITSMOE_ERR_BLOB              -10  /* packed blob is malformed / wrong version           */
+#define BITSMOE_ERR_WORKSPACE_STATE   -11  /* workspace not zero-filled before its first use    */
 
 /* Host description of one quantised MoE layer (all host pointers, read-only,
  * owned by the caller; row-major, C order).
@@ -140,10 +141,9 @@ size_t bitsmoe_workspace_bytes(const bitsmoe_layer* layer, int T, int top_k);
 
 /* Kernels one bitsmoe_moe_forward call launches for (T, top_k) on this layer
  * (no counterpart in the paper: for callers that capture the forward into a
- * CUDA graph or count launches).  A single token runs as a one-block prep
- * kernel plus one fused persistent kernel (2) when the layer's per-block
- * shares of the bases and factors fit in shared memory; otherwise the forward
- * is a chain of 5 kernels.  Returns a negative error code for invalid
+ * CUDA graph or count launches).  A single token runs as one fused persistent
+ * kernel (1) when the layer's per-block shares of the bases and factors fit
+ * in shared memory; otherwise the forward is a chain of 5 kernels.  Returns a negative error code for invalid
  * arguments. */
 int bitsmoe_forward_launches(const bitsmoe_layer* layer, int T, int top_k);
 
@@ -157,7 +157,12 @@ int bitsmoe_forward_launches(const bitsmoe_layer* layer, int T, int top_k);
  *   y       device, T x D fp32 output (row-major), 16-byte aligned, written
  *   ws      device workspace of >= bitsmoe_workspace_bytes(layer, T, top_k)
  *           bytes, 256-byte aligned, owned by the caller; must not be used by
- *           another call in flight
+ *           another call in flight.  Zero-fill it once before its first use
+ *           (the single-token kernel keeps grid-barrier counters in its first
+ *           bytes, and every call leaves them at zero again); it may then be
+ *           reused across calls, layers and token counts.  A workspace whose
+ *           counters are not zero is reported as BITSMOE_ERR_WORKSPACE_STATE
+ *           by bitsmoe_last_device_status and the call computes nothing.
  * Host-side argument checks only: never allocates, never synchronises. */
 int bitsmoe_moe_forward(const void* x, const float* logits, int T, int top_k,
                         const bitsmoe_layer* layer, float* y,

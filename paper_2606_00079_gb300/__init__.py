@@ -21,6 +21,7 @@ OK = 0
 ERR = {
     -1: "INVALID_ARG", -2: "SHAPE", -3: "UNSUPPORTED_BITS", -4: "WORKSPACE_TOO_SMALL",
     -5: "ALIGNMENT", -6: "CUDA", -7: "OOM", -8: "TIMEOUT", -9: "DEVICE_BOUNDS", -10: "BLOB",
+    -11: "WORKSPACE_STATE",
 }
 ERR_CODE = {v: k for k, v in ERR.items()}
 
@@ -228,7 +229,7 @@ def bitsmoe_workspace_bytes(layer: Layer, T: int, top_k: int) -> int:
 
 
 def bitsmoe_forward_launches(layer: Layer, T: int, top_k: int) -> int:
-    """Kernels one forward call launches (2: prep + fused single-token kernel; 5: the chain)."""
+    """Kernels one forward call launches (1: the fused single-token kernel; 5: the chain)."""
     n = int(_lib().bitsmoe_forward_launches(layer.handle, T, top_k))
     if n < 0:
         raise BitsMoEError(n, "bitsmoe_forward_launches")
@@ -297,14 +298,14 @@ def bitsmoe_strerror(code: int) -> str:
 # torch convenience (device memory + streams only)
 # --------------------------------------------------------------------------
 class Workspace:
-    """Device workspace sized for (T, top_k) on a layer, allocated with torch."""
+    """Device workspace sized for (T, top_k) on a layer, allocated (zero-filled) with torch."""
 
     def __init__(self, layer: Layer, T: int, top_k: int, device=None):
         import torch
         self.nbytes = bitsmoe_workspace_bytes(layer, T, top_k)
         if self.nbytes == 0:
             raise BitsMoEError(ERR_CODE["INVALID_ARG"], "bitsmoe_workspace_bytes")
-        self.buf = torch.empty(self.nbytes + 256, dtype=torch.uint8,
+        self.buf = torch.zeros(self.nbytes + 256, dtype=torch.uint8,
                                device=device if device is not None else f"cuda:{torch.cuda.current_device()}")
         base = self.buf.data_ptr()
         self.ptr = (base + 255) // 256 * 256

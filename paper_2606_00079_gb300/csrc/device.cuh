@@ -78,10 +78,11 @@ static_assert(sizeof(DStage) == 48, "DStage layout");
 struct FusedArgs {
   uint32_t* cnt;     // [4] grid-barrier counters
   const CStage* cst; // [2][E][nseg]
-  const DStage* dst; // [E][ul_max_tiles]
+  const DStage* dst; // [E][ul_max_tiles] (directly after cst)
+  uint64_t tab_bytes;  // bytes of both tables
   int b_per, b_stage, b_nst, e_per;     // basis rows per block, rows per stage, stages; output rows per block
   int nslot_c, slot_c, nslot_d, slot_d; // gate/up and down staging slots (count, bytes)
-  int off_route, off_xs, off_r1, off_d, off_rc, off_cq, off_rec, smem;
+  int off_route, off_xs, off_r1, off_d, off_rc, off_cq, off_rec, off_part, smem;
   int smax, s16, seg_al, ul_max_tiles, d_code_bytes, d_h_bytes;
 };
 

@@ -43,6 +43,10 @@ struct bitsmoe_layer {
   int num_sms;
   uint8_t* d_img;
   uint64_t bytes;
+  uint8_t* d_stage = nullptr;  // staging records of the fused single-token kernel
+  const CStage* d_cst = nullptr;
+  const DStage* d_dst = nullptr;
+  uint64_t stage_bytes = 0;
   std::vector<uint8_t> meta;   // host copy of header + descriptors + segment table
   int seg_bytes = 0;           // largest gate/up item: code bytes inside one row block
   int ul_max_chunks = 1;       // largest 16-byte chunks per row block of any down unit
@@ -1419,7 +1423,7 @@ __global__ void __launch_bounds__(kK3DecWarps * 32) k_down_dec(Fwd p) {
 struct WsLayout {
   size_t status, pair_expert, pair_weight, expert_count, expert_start, pair_list, active, z, gu, s;
   size_t x_stage, logits_stage, y_stage;
-  size_t sync, hq, hsc, hsum;   // fused decode kernel
+  size_t sync;   // fused single-token kernel: grid-barrier counters
   size_t total;
 };
 
@@ -1432,7 +1436,7 @@ WsLayout ws_layout(const ImageHeader& hd, int T, int k) {
     return o;
   };
   const size_t P = (size_t)T * k;
-  w.status = take(16);
+  w.status = take(64);   // [0] status, [1] routing flag; bytes 32..47: fused-kernel barrier counters
   w.pair_expert = take(P * 4);
   w.pair_weight = take(P * 4);
   w.expert_count = take((size_t)hd.E * 4);
@@ -1445,11 +1449,7 @@ WsLayout ws_layout(const ImageHeader& hd, int T, int k) {
   w.x_stage = take((size_t)T * hd.D * 2);
   w.logits_stage = take((size_t)T * hd.E * 4);
   w.y_stage = take((size_t)T * hd.D * 4);
-  const size_t G = std::max(1, kRows / hd.group);
-  w.sync = take((4 + (size_t)hd.E * hd.NRB) * 4);
-  w.hq = take(P * hd.I_pad * 2);
-  w.hsc = take(P * hd.NRB * 4);
-  w.hsum = take(P * hd.NRB * G * 4);
+  w.sync = w.status + 32;   // fixed offset: no other layout of the workspace writes there
   w.total = off;
   return w;
 }
@@ -1696,14 +1696,13 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
   const int G = std::max(1, kRows / hd.group);
   FusedArgs fa;
   if (p.decode && fused_plan(hd, T, top_k, L->seg_bytes, L->ul_max_chunks, p.s16, sms, &fa)) {
-    // one token: the whole layer in one persistent kernel (after a one-block prep kernel)
+    // one token: the whole layer in one persistent kernel
     fa.cnt = reinterpret_cast<uint32_t*>(wb + w.sync);
-    fa.ctr = fa.cnt + 4;
-    fa.hq = reinterpret_cast<int16_t*>(wb + w.hq);
-    fa.hsc = reinterpret_cast<float*>(wb + w.hsc);
-    fa.hsum = reinterpret_cast<int*>(wb + w.hsum);
+    fa.cst = L->d_cst;
+    fa.dst = L->d_dst;
+    fa.tab_bytes = L->stage_bytes;
     if ((rc = mark(0))) return rc;
-    const cudaError_t e = launch_fused(p, fa, hd.E * hd.NRB, sms, st, pdl);
+    const cudaError_t e = launch_fused(p, fa, sms, st, pdl);
     if (e != cudaSuccess) return cuda_fail(e);
     for (int i = 1; i <= 5; ++i)
       if ((rc = mark(i))) return rc;
@@ -1766,19 +1765,34 @@ int upload(std::vector<uint8_t>&& img, int device, bitsmoe_layer** out) {
   BM_CK(cudaSetDevice(device));
   int sms = 0;
   cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, device);
+  // staging records of the fused single-token kernel, derived from the image
+  std::vector<CStage> cst;
+  std::vector<DStage> dst;
+  build_stage_tables(img.data(), cst, dst);
+  const size_t cst_bytes = cst.size() * sizeof(CStage), dst_bytes = dst.size() * sizeof(DStage);
   uint8_t* d = nullptr;
+  uint8_t* ds = nullptr;
   if (e == cudaSuccess) e = cudaMalloc(&d, img.size());
   if (e == cudaSuccess) e = cudaMemcpy(d, img.data(), img.size(), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMalloc(&ds, cst_bytes + dst_bytes + 16);
+  if (e == cudaSuccess && cst_bytes) e = cudaMemcpy(ds, cst.data(), cst_bytes, cudaMemcpyHostToDevice);
+  if (e == cudaSuccess && dst_bytes) e = cudaMemcpy(ds + cst_bytes, dst.data(), dst_bytes, cudaMemcpyHostToDevice);
   cudaSetDevice(prev);
   if (e != cudaSuccess) {
     if (d) cudaFree(d);
+    if (ds) cudaFree(ds);
     return e == cudaErrorMemoryAllocation ? BITSMOE_ERR_OOM : cuda_fail(e);
   }
   bitsmoe_layer* L = new (std::nothrow) bitsmoe_layer;
   if (!L) {
     cudaFree(d);
+    cudaFree(ds);
     return BITSMOE_ERR_OOM;
   }
+  L->d_stage = ds;
+  L->d_cst = reinterpret_cast<const CStage*>(ds);
+  L->d_dst = reinterpret_cast<const DStage*>(ds + cst_bytes);
+  L->stage_bytes = cst_bytes + dst_bytes;
   const ImageHeader* hd = header_of(img.data());
   const size_t meta_end = hd->off_basis_in;   // header + descriptors + segments
   L->device = device;
@@ -1917,7 +1931,7 @@ int bitsmoe_forward_launches(const bitsmoe_layer* L, int T, int top_k) {
   const bool decode = T <= 8 && T * hd.E <= 4096;
   FusedArgs fa;
   const int s16 = (int)align_up(std::max(hd.seg_max_slots, 8), 64) + 8;
-  if (decode && fused_plan(hd, T, top_k, L->seg_bytes, L->ul_max_chunks, s16, L->num_sms, &fa)) return 2;
+  if (decode && fused_plan(hd, T, top_k, L->seg_bytes, L->ul_max_chunks, s16, L->num_sms, &fa)) return 1;
   return 5;
 }
 
@@ -2053,6 +2067,7 @@ void bitsmoe_free(bitsmoe_layer* L) {
   if (cudaGetDevice(&prev) == cudaSuccess) {
     cudaSetDevice(L->device);
     cudaFree(L->d_img);
+    cudaFree(L->d_stage);
     cudaSetDevice(prev);
   }
   delete L;

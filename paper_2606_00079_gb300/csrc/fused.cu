@@ -3,29 +3,31 @@
 //
 // Same arithmetic as the kernel chain in forward.cu (Fig. 1 Stage 3; the
 // association of Eq. app_normalized_decomposition), reorganised so that no
-// phase waits for a kernel launch and every weight byte is requested at the
-// start:
+// phase waits for a kernel launch and every weight byte is requested early:
 //
 //   prologue   bulk copies of this block's rows of the input bases (Phi_g^T,
-//              Phi_u^T) into shared memory; L2 prefetch of its rows of Phi_dn.
-//              Weights only, so this overlaps the tail of the previous kernel
-//              (programmatic dependent launch).
+//              Phi_u^T) into shared memory.  Weights only, so this overlaps
+//              the tail of the previous kernel (programmatic dependent launch).
 //   routing    every block routes the token itself (k largest logits, ties to
 //              the lower index, softmax over the k), then stages its share of
 //              the routed experts' gate/up items into shared memory and
-//              prefetches its share of their down tiles into L2
+//              prefetches its down tiles and its rows of Phi_dn into L2
 //   B          z = Phi^T x for this block's rows                 -> grid barrier 1
 //   C          gate/up items: dp2a over the staged codes, vector red.add into
-//              gate/up; the last item of a (expert, 128-row block) computes
-//              h = SiLU(gate) * up for those rows and quantises it to int16
-//              with one scale per row block                      -> grid barrier 2
+//              gate and up                                       -> grid barrier 2
 //   D          down tiles (staged into the freed projection buffer):
+//              h = SiLU(gate) * up of the tile's expert, quantised to int16
+//              with one scale per 128-row block, then
 //              s += w_e * alpha * (P_dn^T h), fp32 atomics         -> grid barrier 3
 //   E          y = Phi_dn s for this block's rows (staged after B)
 //
-// The grid barriers are counters in the workspace that a one-block prep
-// kernel zeroes before each call; every wait is bounded (about one second of
-// SM clock) and a timeout is reported in the workspace status word.
+// Each work item's copies come from one staging record (CStage / DStage,
+// derived from the image at upload), so a block issues them after a single
+// vector load.  The grid barriers are counters at a fixed place in the
+// workspace: zero when a call starts (the caller zero-fills the workspace once;
+// the last block to finish a call resets them), checked on entry.  Every wait
+// is bounded (about one second of SM clock) and a timeout is reported in the
+// status word.
 #include <algorithm>
 #include <cstring>
 #include <mutex>
@@ -46,14 +48,15 @@ __device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t* ptr) {
   return v;
 }
 
-// All blocks of the grid arrive on `cnt` (zeroed before the launch) and wait
-// until every block has arrived.  Writes before the barrier are visible to
-// loads after it (fence, then L2-coherent loads on the reading side).
+// All blocks of the grid arrive on `cnt` (zero at kernel start) and wait
+// until every block has arrived.  The block's writes before the barrier are
+// ordered before its arrival (bar.sync, then a release reduction), and the
+// waiting side acquires; data written before the barrier is read with
+// L2-coherent loads after it.
 __device__ __forceinline__ void grid_barrier(uint32_t* cnt, uint32_t nblocks, int* status) {
   __syncthreads();
   if (threadIdx.x == 0) {
-    __threadfence();
-    atomicAdd(cnt, 1u);
+    asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(cnt) : "memory");
     const long long t0 = clock64();
     while (ld_acquire_u32(cnt) < nblocks) {
       if (clock64() - t0 > kSpin) {
@@ -76,7 +79,7 @@ __device__ __forceinline__ void prefetch_run(const uint8_t* p, uint64_t bytes) {
 }
 
 // Issue `bytes` (16-byte multiple, 16-byte aligned) into shared memory on an
-// already initialised mbarrier whose transaction count the caller has set.
+// mbarrier whose transaction count the caller has set.
 __device__ __forceinline__ void bulk_run(void* dst, const uint8_t* src, uint32_t bytes, uint64_t* bar) {
   uint32_t o = 0;
   while (o < bytes) {
@@ -84,6 +87,32 @@ __device__ __forceinline__ void bulk_run(void* dst, const uint8_t* src, uint32_t
     bulk_g2s(static_cast<uint8_t*>(dst) + o, src + o, c, bar);
     o += c;
   }
+}
+
+// Copy of a gate/up staging record into shared memory (its per-bucket arrays
+// are read with runtime indices, so it is used from there).
+__device__ __forceinline__ void copy_crec(CStage* dst, const CStage* src) {
+  static_assert(sizeof(CStage) % 16 == 0, "record size");
+  uint4 v[sizeof(CStage) / 16];
+#pragma unroll
+  for (int i = 0; i < (int)(sizeof(CStage) / 16); ++i) v[i] = __ldg(reinterpret_cast<const uint4*>(src) + i);
+#pragma unroll
+  for (int i = 0; i < (int)(sizeof(CStage) / 16); ++i) reinterpret_cast<uint4*>(dst)[i] = v[i];
+}
+__device__ __forceinline__ uint64_t u64_of(uint32_t lo, uint32_t hi) { return (uint64_t)lo | ((uint64_t)hi << 32); }
+// A down staging record, decoded field by field from three 16-byte loads.
+__device__ __forceinline__ DStage load_drec(const DStage* src) {
+  const uint4* q = reinterpret_cast<const uint4*>(src);
+  const uint4 a = __ldg(q), b = __ldg(q + 1), c = __ldg(q + 2);
+  DStage r;
+  r.code = u64_of(a.x, a.y);
+  r.unit = u64_of(a.z, a.w);
+  r.alpha = u64_of(b.x, b.y);
+  r.sz = u64_of(b.z, b.w);
+  r.sz_row = c.x;
+  r.bits = c.y;
+  r.pad_[0] = r.pad_[1] = 0;
+  return r;
 }
 
 // gate/up work item i -> (routed-expert slot a, projection h, row block rb, segment sg)
@@ -102,77 +131,227 @@ __device__ __forceinline__ CItem c_item(const Fwd& p, int i) {
   return c;
 }
 
-// Stage one gate/up item (codes of its row block, unit indices, alpha, the
-// G scale/zero rows of its groups) into a slot.  Lane 0 only.
+// ---------------------------------------------------------------------------
+// Integer dot products with the bit-width as a runtime parameter: one small
+// loop per bit plane keeps the code that a phase runs small (the kernel runs
+// each phase once per call, so instruction fetch is on its critical path).
+// ---------------------------------------------------------------------------
+// Row-lane layout, one bit plane over `ntl` tiles: chunks c0 .. c0 + nc - 1 of
+// each tile of C chunks hold PB-bit fields of consecutive unit groups (chunk
+// c0 + q at activation offset q * coff); word w of the lane's 16 bytes is row
+// w; unit 4k + m of a chunk at bit 8m + PB*k.  cp: int16 activation pairs,
+// cstep int32 per tile.  One out-of-line copy per field width, accumulators
+// passed by value (registers).
+template <int PB>
+__device__ __noinline__ int4 rl_plane(const uint8_t* code, int ntl, int C, int c0, int nc, int coff, const int* cp,
+                                      int cstep, int4 acc) {
+  constexpr int NK = 8 / PB;
+  constexpr uint32_t MASK = ((1u << PB) - 1u) * 0x01010101u;
+#pragma unroll 1
+  for (int t = 0; t < ntl; ++t) {
+#pragma unroll 1
+    for (int q = 0; q < nc; ++q) {
+      const uint4 v = lds128(code + (size_t)(t * C + c0 + q) * kChunkBytes);
+      const int* ct = cp + t * cstep + q * coff;
+      int2 cc[NK];
+#pragma unroll
+      for (int kq = 0; kq < NK; ++kq) cc[kq] = *reinterpret_cast<const int2*>(ct + 2 * kq);
+#pragma unroll
+      for (int kq = 0; kq < NK; ++kq) {
+        uint32_t b = (v.x >> (PB * kq)) & MASK;
+        acc.x = dp2a_hi(cc[kq].y, b, dp2a_lo(cc[kq].x, b, acc.x));
+        b = (v.y >> (PB * kq)) & MASK;
+        acc.y = dp2a_hi(cc[kq].y, b, dp2a_lo(cc[kq].x, b, acc.y));
+        b = (v.z >> (PB * kq)) & MASK;
+        acc.z = dp2a_hi(cc[kq].y, b, dp2a_lo(cc[kq].x, b, acc.z));
+        b = (v.w >> (PB * kq)) & MASK;
+        acc.w = dp2a_hi(cc[kq].y, b, dp2a_lo(cc[kq].x, b, acc.w));
+      }
+    }
+  }
+  return acc;
+}
+
+// A bucket range of a gate/up item (b < 16): accf[w] += sum_u code_{w,u} * c_u,
+// flushed to fp32 every 32 tiles (int32 headroom for 8-bit codes).
+__device__ void rl_range_rt(int b, const uint8_t* code, int ntl, const int* cp, float (&accf)[4]) {
+  const int C = rl_chunks(b), cstep = rl_units(b) / 2;
+  const int hs = b == 3 ? 2 : 4;
+  for (int t0 = 0; t0 < ntl; t0 += 32) {
+    const int n = min(32, ntl - t0);
+    const uint8_t* cb = code + (size_t)t0 * C * kChunkBytes;
+    const int* cpp = cp + t0 * cstep;
+    int4 lo = make_int4(0, 0, 0, 0), hi = make_int4(0, 0, 0, 0);
+    switch (b) {
+      case 1: lo = rl_plane<1>(cb, n, 1, 0, 1, 0, cpp, cstep, lo); break;
+      case 2: lo = rl_plane<2>(cb, n, 1, 0, 1, 0, cpp, cstep, lo); break;
+      case 4: lo = rl_plane<4>(cb, n, 1, 0, 1, 0, cpp, cstep, lo); break;
+      case 8: lo = rl_plane<8>(cb, n, 1, 0, 1, 0, cpp, cstep, lo); break;
+      case 3:   // low 2-bit plane of units 0-15 and 16-31, then the high bit of units 0-31
+        lo = rl_plane<2>(cb, n, 3, 0, 2, 8, cpp, cstep, lo);
+        hi = rl_plane<1>(cb, n, 3, 2, 1, 0, cpp, cstep, hi);
+        break;
+      default:  // 6: low 4-bit plane of units 0-7 and 8-15, then the high 2 bits of units 0-15
+        lo = rl_plane<4>(cb, n, 3, 0, 2, 4, cpp, cstep, lo);
+        hi = rl_plane<2>(cb, n, 3, 2, 1, 0, cpp, cstep, hi);
+        break;
+    }
+    accf[0] += (float)(lo.x + (hi.x << hs));
+    accf[1] += (float)(lo.y + (hi.y << hs));
+    accf[2] += (float)(lo.z + (hi.z << hs));
+    accf[3] += (float)(lo.w + (hi.w << hs));
+  }
+}
+
+// Unit-lane layout, `nc` consecutive 16-byte chunks of PB-bit fields of the
+// lane's unit (chunk q covers rows rbase + q * 128 / PB ..): word w of a chunk
+// covers 32 / PB rows, row r' = 4k + m at bit 8m + PB*k.  Returns the dot with
+// the int16 activations per group g of the row block (G <= 4) in .x .. .w.
+template <int PB, int G>
+__device__ __noinline__ int4 ul_plane(const uint8_t* cb, int nc, int rbase, const int* hq32, int gshift, int4 acc) {
+  constexpr int NK = 8 / PB, RPW = 32 / PB;
+  constexpr uint32_t MASK = ((1u << PB) - 1u) * 0x01010101u;
+#pragma unroll 1
+  for (int q = 0; q < nc; ++q) {
+    const uint4 v = lds128(cb + (size_t)q * kChunkBytes);
+    const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
+    const int rq = rbase + q * (kRows / PB);
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+      const int r0 = rq + w * RPW;
+      const int* hp = hq32 + r0 / 2;
+      int2 hh[NK];
+#pragma unroll
+      for (int kq = 0; kq < NK; ++kq) hh[kq] = *reinterpret_cast<const int2*>(hp + 2 * kq);
+      int tmp = 0;
+#pragma unroll
+      for (int kq = 0; kq < NK; ++kq) {
+        const uint32_t b = (wv[w] >> (PB * kq)) & MASK;
+        tmp = dp2a_hi(hh[kq].y, b, dp2a_lo(hh[kq].x, b, tmp));
+      }
+      const int gl = G == 1 ? 0 : (r0 >> gshift);
+      if (gl == 0) acc.x += tmp;
+      else if (gl == 1) acc.y += tmp;
+      else if (gl == 2) acc.z += tmp;
+      else acc.w += tmp;
+    }
+  }
+  return acc;
+}
+
+// Down tile of the lane's unit over row blocks rb = rb0, rb0 + step, ..., h
+// quantised per row block:
+//   sum_rb hsc_rb * sum_g s_g (sum_{i in rb, g} q_i h_i - zero_g * sum_{i in rb, g} h_i)
 template <int G>
-__device__ void c_stage(const Fwd& p, const FusedArgs& f, const CItem& ci, int e, const ItemRec& it, uint8_t* slot,
-                        uint64_t* bar) {
-  const ExpertDesc& xd = p.desc[ci.h * p.E + e];
-  const uint64_t code_base = xd.code_base, rb_stride = xd.rb_stride, unit_off = xd.unit_off;
-  const uint64_t alpha_off = xd.alpha_off, sz_off = xd.sz_off;
-  const int nslots = xd.nslots;
-  const uint32_t mb = (uint32_t)it.nslot * 4;
-  uint8_t* codes = slot;
+__device__ float ul_tile_rt(int b, const uint8_t* code, int NRB, int rb0, int step, int group, const int16_t* hq,
+                            const float* hsc, const int* hsum, const uint32_t* sz, int lane) {
+  const int gshift = 31 - __clz(group);
+  const int C = ul_chunks(b);
+  float accf = 0.f;
+  for (int rb = rb0; rb < NRB; rb += step) {
+    const int* hq32 = reinterpret_cast<const int*>(hq + rb * kRows);
+    const uint8_t* cb = code + (size_t)rb * C * kChunkBytes;
+    if (b == 16) {   // fp16 values: chunk c = rows 8c .. 8c + 7, two rows per word
+      float tmp = 0.f;
+#pragma unroll 1
+      for (int c = 0; c < 16; ++c) {
+        const uint4 v = lds128(cb + (size_t)c * kChunkBytes);
+        const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+          const int hp = hq32[4 * c + w];
+          tmp = fmaf((float)(int16_t)(hp & 0xFFFF), f16lo(wv[w]), fmaf((float)(hp >> 16), f16hi(wv[w]), tmp));
+        }
+      }
+      accf = fmaf(hsc[rb], tmp, accf);
+      continue;
+    }
+    int4 lo = make_int4(0, 0, 0, 0), hi = make_int4(0, 0, 0, 0);
+    switch (b) {
+      case 1: lo = ul_plane<1, G>(cb, 1, 0, hq32, gshift, lo); break;
+      case 2: lo = ul_plane<2, G>(cb, 2, 0, hq32, gshift, lo); break;
+      case 4: lo = ul_plane<4, G>(cb, 4, 0, hq32, gshift, lo); break;
+      case 8: lo = ul_plane<8, G>(cb, 8, 0, hq32, gshift, lo); break;
+      case 3:   // low 2-bit plane rows 0-63 / 64-127, then the high bit of rows 0-127
+        lo = ul_plane<2, G>(cb, 2, 0, hq32, gshift, lo);
+        hi = ul_plane<1, G>(cb + 2 * kChunkBytes, 1, 0, hq32, gshift, hi);
+        break;
+      default:  // 6: low 4-bit plane rows 32c .., then the high 2 bits of rows 0-63 / 64-127
+        lo = ul_plane<4, G>(cb, 4, 0, hq32, gshift, lo);
+        hi = ul_plane<2, G>(cb + 4 * kChunkBytes, 2, 0, hq32, gshift, hi);
+        break;
+    }
+    const int hs = b == 3 ? 2 : 4;
+    const int lo_g[4] = {lo.x, lo.y, lo.z, lo.w}, hi_g[4] = {hi.x, hi.y, hi.z, hi.w};
+    float d_rb = 0.f;
+    const int gfirst = (rb * kRows) >> gshift;
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      const uint32_t szw = sz[(size_t)(gfirst + g) * 32 + lane];
+      const float sc = __half2float(__ushort_as_half((unsigned short)(szw & 0xFFFFu)));
+      const float zp = __half2float(__ushort_as_half((unsigned short)(szw >> 16)));
+      d_rb = fmaf(sc, fmaf(-zp, (float)hsum[rb * G + g], (float)(lo_g[g] + (hi_g[g] << hs))), d_rb);
+    }
+    accf = fmaf(hsc[rb], d_rb, accf);
+  }
+  return accf;
+}
+
+// Copies of one gate/up item into a slot: [codes seg_al][unit smax][alpha smax][scale/zero G x smax].
+template <int G>
+__device__ void c_stage(const Fwd& p, const FusedArgs& f, const CStage& r, int rb, uint8_t* slot, uint64_t* bar) {
   uint8_t* su = slot + f.seg_al;
   uint8_t* sa = su + (size_t)f.smax * 4;
   uint8_t* ssz = sa + (size_t)f.smax * 4;
-  const int g_base = (ci.rb * kRows) / p.group;
-  mbar_expect_tx(bar, it.bytes + (2 + G) * mb);
-  bulk_run(codes, p.img + code_base + (size_t)ci.rb * rb_stride + it.byte0, it.bytes, bar);
-  bulk_g2s(su, p.img + unit_off + (size_t)it.slot0 * 4, mb, bar);
-  bulk_g2s(sa, p.img + alpha_off + (size_t)it.slot0 * 4, mb, bar);
+  const int g_base = (rb * kRows) / p.group;
+  mbar_expect_tx(bar, r.bytes + (2 + G) * r.mb);
+  bulk_run(slot, p.img + r.code0 + (uint64_t)rb * r.rb_stride, r.bytes, bar);
+  bulk_g2s(su, p.img + r.unit0, r.mb, bar);
+  bulk_g2s(sa, p.img + r.alpha0, r.mb, bar);
 #pragma unroll
   for (int gl = 0; gl < G; ++gl)
-    bulk_g2s(ssz + (size_t)gl * f.smax * 4, p.img + sz_off + ((size_t)(g_base + gl) * nslots + it.slot0) * 4, mb, bar);
+    bulk_g2s(ssz + (size_t)gl * f.smax * 4, p.img + r.sz0 + (uint64_t)(g_base + gl) * r.sz_row, r.mb, bar);
 }
 
-// L2 prefetch of the bytes c_stage would copy (for items staged in a later round).
-__device__ void c_prefetch(const Fwd& p, const CItem& ci, int e, const ItemRec& it) {
-  const ExpertDesc& xd = p.desc[ci.h * p.E + e];
-  prefetch_run(p.img + xd.code_base + (size_t)ci.rb * xd.rb_stride + it.byte0, it.bytes);
-}
-
-// One staged gate/up item for the single token: writes its partial rows of
-// gate (h = 0) or up (h = 1) with vector reductions.
+// One staged gate/up item for the single token: adds its partial rows of gate
+// (h = 0) or up (h = 1) with vector reductions.
 template <int G>
-__device__ void c_compute(const Fwd& p, const FusedArgs& f, const CItem& ci, const ItemRec& it, const uint8_t* slot,
+__device__ void c_compute(const Fwd& p, const FusedArgs& f, const CStage& r, int h, int rb, const uint8_t* slot,
                           int16_t* cq, int pair, int lane) {
-  const uint8_t* codes = slot;
   const int* su = reinterpret_cast<const int*>(slot + f.seg_al);
   const float* sa = reinterpret_cast<const float*>(su + f.smax);
   const uint32_t* ssz = reinterpret_cast<const uint32_t*>(sa + f.smax);
-  const float* zrow = p.z + (size_t)ci.h * p.n_pad;   // one token: z[h][0][:]
-  int nls = 0;
-  for (int q = 0; q < it.nr; ++q)
-    if (it.bits[q] < 16) nls += it.ntl[q] * rl_units(it.bits[q]);
-  // c = alpha * z * scale per (slot, group), int16 with one scale per item
-  const bool fast = nls <= 32 * kFZ;
+  const float* zrow = p.z + (size_t)h * p.n_pad;   // one token: z[h][0][:]
+  const int nls = r.nls;
+  // c = alpha * z * scale per (slot, group), int16 with one scale per item.
+  // Up to 32 * kFZ slots: one batch of z gathers, kept in registers for both
+  // passes; larger items gather z again in the second pass.
   float mx = 0.f;
   float zr[kFZ];
-  if (fast) {
 #pragma unroll
-    for (int m = 0; m < kFZ; ++m) {
-      const int i = lane + 32 * m;
-      zr[m] = i < nls ? __ldcg(zrow + su[i]) : 0.f;
+  for (int m = 0; m < kFZ; ++m) {
+    const int i = lane + 32 * m;
+    zr[m] = i < nls ? __ldcg(zrow + su[i]) * sa[i] : 0.f;
+  }
+  const bool one_batch = nls <= 32 * kFZ;
+  for (int i0 = 0; i0 < nls; i0 += 32 * kFZ) {
+    if (i0 > 0) {
+#pragma unroll
+      for (int m = 0; m < kFZ; ++m) {
+        const int i = i0 + lane + 32 * m;
+        zr[m] = i < nls ? __ldcg(zrow + su[i]) * sa[i] : 0.f;
+      }
     }
 #pragma unroll
     for (int m = 0; m < kFZ; ++m) {
-      const int i = lane + 32 * m;
+      const int i = i0 + lane + 32 * m;
       if (i < nls) {
-        zr[m] *= sa[i];
 #pragma unroll
         for (int gl = 0; gl < G; ++gl) {
           const float sc = __half2float(__ushort_as_half((unsigned short)(ssz[gl * f.smax + i] & 0xFFFFu)));
           mx = fmaxf(mx, fabsf(zr[m] * sc));
         }
       }
-    }
-  } else {
-    for (int i = lane; i < nls; i += 32) {
-      const float zv = sa[i] * __ldcg(zrow + su[i]);
-#pragma unroll
-      for (int gl = 0; gl < G; ++gl)
-        mx = fmaxf(mx, fabsf(zv * __half2float(__ushort_as_half((unsigned short)(ssz[gl * f.smax + i] & 0xFFFFu)))));
     }
   }
   mx = warp_max(mx);
@@ -181,60 +360,47 @@ __device__ void c_compute(const Fwd& p, const FusedArgs& f, const CItem& ci, con
   float corr[G];
 #pragma unroll
   for (int gl = 0; gl < G; ++gl) corr[gl] = 0.f;
-  if (fast) {
+  for (int i0 = 0; i0 < nls; i0 += 32 * kFZ) {
+    if (!one_batch) {
+#pragma unroll
+      for (int m = 0; m < kFZ; ++m) {
+        const int i = i0 + lane + 32 * m;
+        zr[m] = i < nls ? __ldcg(zrow + su[i]) * sa[i] : 0.f;
+      }
+    }
 #pragma unroll
     for (int m = 0; m < kFZ; ++m) {
-      const int i = lane + 32 * m;
+      const int i = i0 + lane + 32 * m;
       if (i < nls) {
 #pragma unroll
         for (int gl = 0; gl < G; ++gl) {
           const uint32_t w = ssz[gl * f.smax + i];
           const float sc = __half2float(__ushort_as_half((unsigned short)(w & 0xFFFFu)));
           const float zp = __half2float(__ushort_as_half((unsigned short)(w >> 16)));
-          const int ci2 = __float2int_rn(zr[m] * sc * inv);
-          cq[(size_t)gl * f.s16 + i] = (int16_t)ci2;
-          corr[gl] = fmaf((float)ci2, zp, corr[gl]);
+          const int ci = __float2int_rn(zr[m] * sc * inv);
+          cq[(size_t)gl * f.s16 + i] = (int16_t)ci;
+          corr[gl] = fmaf((float)ci, zp, corr[gl]);
         }
-      }
-    }
-  } else {
-    for (int i = lane; i < nls; i += 32) {
-      const float zv = sa[i] * __ldcg(zrow + su[i]);
-#pragma unroll
-      for (int gl = 0; gl < G; ++gl) {
-        const uint32_t w = ssz[gl * f.smax + i];
-        const float sc = __half2float(__ushort_as_half((unsigned short)(w & 0xFFFFu)));
-        const float zp = __half2float(__ushort_as_half((unsigned short)(w >> 16)));
-        const int ci2 = __float2int_rn(zv * sc * inv);
-        cq[(size_t)gl * f.s16 + i] = (int16_t)ci2;
-        corr[gl] = fmaf((float)ci2, zp, corr[gl]);
       }
     }
   }
 #pragma unroll
   for (int gl = 0; gl < G; ++gl) corr[gl] = warp_sum(corr[gl]);
   __syncwarp();
-  float accf[4][1], acc16[4][1];
+  float accf[4] = {0.f, 0.f, 0.f, 0.f};
+  float acc16[4][1];
 #pragma unroll
-  for (int w = 0; w < 4; ++w) accf[w][0] = acc16[w][0] = 0.f;
+  for (int w = 0; w < 4; ++w) acc16[w][0] = 0.f;
   const int gl_lane = G == 1 ? 0 : (4 * lane) / p.group;
   const int* cq32 = reinterpret_cast<const int*>(cq + (size_t)gl_lane * f.s16);
   const float* const zrows[1] = {zrow};
   uint32_t boff = 0;
   int ls = 0;
-  for (int q = 0; q < it.nr; ++q) {
-    const int b = it.bits[q], ntl = it.ntl[q];
-    const uint8_t* code = codes + boff + lane * 16;
-    const int* cp = cq32 + ls / 2;
-    switch (b) {
-      case 1: rl_range<1, 1, true>(code, ntl, cp, 0, accf); break;
-      case 2: rl_range<2, 1, true>(code, ntl, cp, 0, accf); break;
-      case 3: rl_range<3, 1, true>(code, ntl, cp, 0, accf); break;
-      case 4: rl_range<4, 1, true>(code, ntl, cp, 0, accf); break;
-      case 6: rl_range<6, 1, true>(code, ntl, cp, 0, accf); break;
-      case 8: rl_range<8, 1, true>(code, ntl, cp, 0, accf); break;
-      default: rl_range16<1, true>(code, ntl, su + ls, sa + ls, zrows, acc16); break;
-    }
+  for (int q = 0; q < r.nr; ++q) {
+    const int b = r.bits[q], ntl = r.ntl[q];
+    const uint8_t* code = slot + boff + lane * 16;
+    if (b < 16) rl_range_rt(b, code, ntl, cq32 + ls / 2, accf);
+    else rl_range16<1, true>(code, ntl, su + ls, sa + ls, zrows, acc16);
     boff += (uint32_t)ntl * rl_chunks(b) * kChunkBytes;
     ls += ntl * rl_units(b);
   }
@@ -244,174 +410,75 @@ __device__ void c_compute(const Fwd& p, const FusedArgs& f, const CItem& ci, con
     if (gl == gl_lane) cl = corr[gl];
   float o[4];
 #pragma unroll
-  for (int w = 0; w < 4; ++w) o[w] = fmaf(scl, accf[w][0] - cl, acc16[w][0]);
-  red_add_v4(p.gu + ((size_t)pair * 2 + ci.h) * p.I_pad + ci.rb * kRows + 4 * lane, o[0], o[1], o[2], o[3]);
+  for (int w = 0; w < 4; ++w) o[w] = fmaf(scl, accf[w] - cl, acc16[w][0]);
+  red_add_v4(p.gu + ((size_t)pair * 2 + h) * p.I_pad + rb * kRows + 4 * lane, o[0], o[1], o[2], o[3]);
 }
 
-// h = SiLU(gate) * up for the 128 rows of row block rb of one pair, quantised
-// to int16 with one scale per row block; also the per-group sums of the codes.
-// Called by the warp that finished the last gate/up item of (expert, rb).
+// h = SiLU(gate) * up of one pair for row blocks rb0, rb0 + step, ... into the
+// warp's area: int16 codes, one scale per 128-row block, sums of the codes per
+// (row block, group).  The lane owns rows 4 * lane .. + 3 of a row block.
 template <int G>
-__device__ void h_rows(const Fwd& p, const FusedArgs& f, int pair, int rb, int lane) {
-  const int row = rb * kRows + 4 * lane;
-  const float4 g = __ldcg(reinterpret_cast<const float4*>(p.gu + ((size_t)pair * 2) * p.I_pad + row));
-  const float4 u = __ldcg(reinterpret_cast<const float4*>(p.gu + ((size_t)pair * 2 + 1) * p.I_pad + row));
-  float hv[4] = {g.x / (1.f + __expf(-g.x)) * u.x, g.y / (1.f + __expf(-g.y)) * u.y,
-                 g.z / (1.f + __expf(-g.z)) * u.z, g.w / (1.f + __expf(-g.w)) * u.w};
-  float mx = fmaxf(fmaxf(fabsf(hv[0]), fabsf(hv[1])), fmaxf(fabsf(hv[2]), fabsf(hv[3])));
-  mx = warp_max(mx);
-  const float inv = mx > 0.f ? 32767.f / mx : 0.f;
-  int q[4];
-#pragma unroll
-  for (int w = 0; w < 4; ++w) q[w] = __float2int_rn(hv[w] * inv);
-  const uint32_t lo = (uint32_t)(q[0] & 0xFFFF) | ((uint32_t)q[1] << 16);
-  const uint32_t hi = (uint32_t)(q[2] & 0xFFFF) | ((uint32_t)q[3] << 16);
-  *reinterpret_cast<uint2*>(f.hq + (size_t)pair * p.I_pad + row) = make_uint2(lo, hi);
-  int sq = q[0] + q[1] + q[2] + q[3];
-  // group sums: lanes of one group are 8 (group 32), 16 (group 64) or all 32
+__device__ void h_rows(const Fwd& p, int pair, int rb0, int step, int16_t* hq, float* hsc, int* hsum, int lane) {
+  const float* gp = p.gu + ((size_t)pair * 2) * p.I_pad + 4 * lane;
+  const float* up = gp + p.I_pad;
   const int lanes_per_group = G == 1 ? 32 : p.group / 4;
+  constexpr int kB = 4;   // row blocks whose gate/up loads are in flight together
+  for (int rbb = rb0; rbb < p.NRB; rbb += kB * step) {
+    float4 g4[kB], u4[kB];
 #pragma unroll
-  for (int o = 16; o; o >>= 1)
-    if (o < lanes_per_group) sq += __shfl_xor_sync(0xFFFFFFFFu, sq, o);
-  if ((lane & (lanes_per_group - 1)) == 0) f.hsum[((size_t)pair * p.NRB + rb) * G + lane / lanes_per_group] = sq;
-  if (lane == 0) f.hsc[(size_t)pair * p.NRB + rb] = mx * (1.f / 32767.f);
-}
-
-// Down tile of the lane's unit over all row blocks, h quantised per row block:
-//   accf = sum_rb hsc_rb * sum_g s_g (sum_{i in rb, g} q_i h_i - zero_g * sum_{i in rb, g} h_i)
-template <int B, int G>
-__device__ __forceinline__ float ul_tile_rb(const uint8_t* code, int NRB, int group, const int16_t* hq,
-                                            const float* hsc, const int* hsum, const uint32_t* sz, int lane) {
-  constexpr int C = ul_chunks(B);
-  const int gshift = 31 - __clz(group);
-  float accf = 0.f;
-  for (int rb = 0; rb < NRB; ++rb) {
-    const int* hq32 = reinterpret_cast<const int*>(hq + rb * kRows);
-    const uint8_t* cb = code + (size_t)rb * C * kChunkBytes;
-    if (B == 16) {
-      float tmp = 0.f;
-#pragma unroll 4
-      for (int c = 0; c < 16; ++c) {
-        const uint4 v = lds128(cb + (size_t)c * kChunkBytes);
-        const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
+    for (int i = 0; i < kB; ++i) {
+      const int rb = rbb + i * step;
+      const bool ok = rb < p.NRB;
+      g4[i] = ok ? __ldcg(reinterpret_cast<const float4*>(gp + (size_t)rb * kRows)) : make_float4(0, 0, 0, 0);
+      u4[i] = ok ? __ldcg(reinterpret_cast<const float4*>(up + (size_t)rb * kRows)) : make_float4(0, 0, 0, 0);
+    }
+#pragma unroll 1
+    for (int i = 0; i < kB; ++i) {
+      const int rb = rbb + i * step;
+      if (rb >= p.NRB) break;
+      const float4 g = g4[0], u = u4[0];   // the batch rotates through slot 0
+      const float hv[4] = {__fdividef(g.x, 1.f + __expf(-g.x)) * u.x, __fdividef(g.y, 1.f + __expf(-g.y)) * u.y,
+                           __fdividef(g.z, 1.f + __expf(-g.z)) * u.z, __fdividef(g.w, 1.f + __expf(-g.w)) * u.w};
 #pragma unroll
-        for (int w = 0; w < 4; ++w) {
-          const int hp = hq32[(8 * c + 2 * w) / 2];
-          tmp = fmaf((float)(int16_t)(hp & 0xFFFF), f16lo(wv[w]), fmaf((float)(hp >> 16), f16hi(wv[w]), tmp));
-        }
+      for (int j = 0; j + 1 < kB; ++j) {
+        g4[j] = g4[j + 1];
+        u4[j] = u4[j + 1];
       }
-      accf = fmaf(hsc[rb], tmp, accf);
-      continue;
-    }
-    int acc[G][1], acch[G][1];
+      float mx = fmaxf(fmaxf(fabsf(hv[0]), fabsf(hv[1])), fmaxf(fabsf(hv[2]), fabsf(hv[3])));
+      mx = warp_max(mx);
+      const float inv = mx > 0.f ? 32767.f / mx : 0.f;
+      int q[4];
 #pragma unroll
-    for (int g = 0; g < G; ++g) acc[g][0] = acch[g][0] = 0;
-    uint4 v[C];
+      for (int w = 0; w < 4; ++w) q[w] = __float2int_rn(hv[w] * inv);
+      const uint32_t lo = (uint32_t)(q[0] & 0xFFFF) | ((uint32_t)q[1] << 16);
+      const uint32_t hi = (uint32_t)(q[2] & 0xFFFF) | ((uint32_t)q[3] << 16);
+      *reinterpret_cast<uint2*>(hq + rb * kRows + 4 * lane) = make_uint2(lo, hi);
+      int sq = q[0] + q[1] + q[2] + q[3];
 #pragma unroll
-    for (int c = 0; c < C; ++c) v[c] = lds128(cb + (size_t)c * kChunkBytes);
-    if (B == 3) {
-      ul_chunk<2, G, 1>(v[0], 0, hq32, 0, gshift, acc);
-      ul_chunk<2, G, 1>(v[1], 64, hq32, 0, gshift, acc);
-      ul_chunk<1, G, 1>(v[2], 0, hq32, 0, gshift, acch);
-    } else if (B == 6) {
-#pragma unroll
-      for (int c = 0; c < 4; ++c) ul_chunk<4, G, 1>(v[c], 32 * c, hq32, 0, gshift, acc);
-      ul_chunk<2, G, 1>(v[4], 0, hq32, 0, gshift, acch);
-      ul_chunk<2, G, 1>(v[5], 64, hq32, 0, gshift, acch);
-    } else {
-#pragma unroll
-      for (int c = 0; c < C; ++c) ul_chunk<B, G, 1>(v[c], c * (kRows / B), hq32, 0, gshift, acc);
-    }
-    float d_rb = 0.f;
-    const int gfirst = (rb * kRows) >> gshift;
-#pragma unroll
-    for (int g = 0; g < G; ++g) {
-      const uint32_t szw = sz[(size_t)(gfirst + g) * 32 + lane];
-      const float sc = __half2float(__ushort_as_half((unsigned short)(szw & 0xFFFFu)));
-      const float zp = __half2float(__ushort_as_half((unsigned short)(szw >> 16)));
-      const int tot = (B == 3 || B == 6) ? acc[g][0] + (acch[g][0] << (B == 3 ? 2 : 4)) : acc[g][0];
-      d_rb = fmaf(sc, fmaf(-zp, (float)hsum[rb * G + g], (float)tot), d_rb);
-    }
-    accf = fmaf(hsc[rb], d_rb, accf);
-  }
-  return accf;
-}
-
-// down work item i -> (routed-expert slot a, UL tile)
-struct DItem {
-  int a, tile;
-};
-__device__ __forceinline__ DItem d_item(const FusedArgs& f, int i) {
-  DItem d;
-  d.a = i / f.ul_max_tiles;
-  d.tile = i - d.a * f.ul_max_tiles;
-  return d;
-}
-
-// Where a down tile lives: its bucket's bit-width, first slot, code run and
-// scale/zero column.  bits = 0 when the tile index is past the expert's tiles.
-struct DLoc {
-  int bits, slot;       // slot of the tile's first unit in the (h=2, e) slot arrays
-  int nslots;           // row stride of the scale/zero matrix
-  uint64_t code, sz;    // image offsets: tile code run (NRB row blocks), scale/zero column of its first slot
-  uint64_t unit, alpha; // image offsets of its 32 unit indices and alphas
-};
-__device__ DLoc d_loc(const Fwd& p, int e, int tile) {
-  const ExpertDesc& xd = p.desc[2 * p.E + e];
-  DLoc l;
-  l.bits = 0;
-  l.slot = 0;
-  l.nslots = xd.nslots;
-  l.code = l.sz = l.unit = l.alpha = 0;
-  const int nbk = xd.nbk;
-  for (int q = 0; q < nbk; ++q) {
-    const int t0 = xd.bk[q].tile0, nt = xd.bk[q].ntiles;
-    if (tile >= t0 && tile < t0 + nt) {
-      const int b = xd.bk[q].bits;
-      l.bits = b;
-      l.slot = xd.bk[q].slot0 + (tile - t0) * 32;
-      l.code = xd.code_base + xd.bk[q].code_off + (uint64_t)(tile - t0) * p.NRB * ul_chunks(b) * kChunkBytes;
-      l.sz = xd.sz_off + (uint64_t)l.slot * 4;
-      l.unit = xd.unit_off + (uint64_t)l.slot * 4;
-      l.alpha = xd.alpha_off + (uint64_t)l.slot * 4;
+      for (int o = 16; o; o >>= 1)
+        if (o < lanes_per_group) sq += __shfl_xor_sync(0xFFFFFFFFu, sq, o);
+      if ((lane & (lanes_per_group - 1)) == 0) hsum[rb * G + lane / lanes_per_group] = sq;
+      if (lane == 0) hsc[rb] = mx * (1.f / 32767.f);
     }
   }
-  return l;
 }
 
 // D slot layout: [codes NRB * ul_max_chunks * 512][unit 32 x 4][alpha 32 x 4][scale/zero NG x 32 x 4]
-__device__ void d_stage(const Fwd& p, const FusedArgs& f, const DLoc& l, uint8_t* slot, uint64_t* bar) {
-  const uint32_t cb = (uint32_t)p.NRB * ul_chunks(l.bits) * kChunkBytes;
+__device__ void d_stage(const Fwd& p, const FusedArgs& f, const DStage& r, uint8_t* slot, uint64_t* bar) {
+  const uint32_t cb = (uint32_t)p.NRB * ul_chunks((int)r.bits) * kChunkBytes;
   uint8_t* su = slot + f.d_code_bytes;
   uint8_t* sa = su + 128;
   uint8_t* ssz = sa + 128;
   mbar_expect_tx(bar, cb + 256 + (uint32_t)p.NG * 128);
-  bulk_run(slot, p.img + l.code, cb, bar);
-  bulk_g2s(su, p.img + l.unit, 128, bar);
-  bulk_g2s(sa, p.img + l.alpha, 128, bar);
-  for (int g = 0; g < p.NG; ++g) bulk_g2s(ssz + g * 128, p.img + l.sz + (uint64_t)g * l.nslots * 4, 128, bar);
+  bulk_run(slot, p.img + r.code, cb, bar);
+  bulk_g2s(su, p.img + r.unit, 128, bar);
+  bulk_g2s(sa, p.img + r.alpha, 128, bar);
+  for (int g = 0; g < p.NG; ++g) bulk_g2s(ssz + g * 128, p.img + r.sz + (uint64_t)g * r.sz_row, 128, bar);
 }
 
-template <int G>
-__device__ void d_compute(const Fwd& p, const FusedArgs& f, const DLoc& l, const uint8_t* slot,
-                          const int16_t* hq, const float* hsc, const int* hsum, int pair, float wgt, int lane) {
-  const uint8_t* code = slot + lane * 16;
-  const int* su = reinterpret_cast<const int*>(slot + f.d_code_bytes);
-  const float* sa = reinterpret_cast<const float*>(su + 32);
-  const uint32_t* ssz = reinterpret_cast<const uint32_t*>(sa + 32);
-  float acc = 0.f;
-  switch (l.bits) {
-    case 1: acc = ul_tile_rb<1, G>(code, p.NRB, p.group, hq, hsc, hsum, ssz, lane); break;
-    case 2: acc = ul_tile_rb<2, G>(code, p.NRB, p.group, hq, hsc, hsum, ssz, lane); break;
-    case 3: acc = ul_tile_rb<3, G>(code, p.NRB, p.group, hq, hsc, hsum, ssz, lane); break;
-    case 4: acc = ul_tile_rb<4, G>(code, p.NRB, p.group, hq, hsc, hsum, ssz, lane); break;
-    case 6: acc = ul_tile_rb<6, G>(code, p.NRB, p.group, hq, hsc, hsum, ssz, lane); break;
-    case 8: acc = ul_tile_rb<8, G>(code, p.NRB, p.group, hq, hsc, hsum, ssz, lane); break;
-    default: acc = ul_tile_rb<16, G>(code, p.NRB, p.group, hq, hsc, hsum, ssz, lane); break;
-  }
-  const float al = sa[lane];
-  if (al != 0.f) atomicAdd(p.s + su[lane], wgt * al * acc);   // one token: s[0][j]
-}
+// Warps 0 .. kBW-1 project (phase B); warps kBW .. kFWarps-1 route and stage.
+constexpr int kBW = 12;
+constexpr int kCT = (kFWarps - kBW) * 32;   // control threads
 
 template <int G>
 __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
@@ -420,6 +487,12 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
   uint64_t* bar_e = bar_b + kMaxBStages;                 // [1]
   uint64_t* bar_c = bar_e + 1;                           // [kFWarps]
   uint64_t* bar_d = bar_c + kFWarps;                     // [kFWarps]
+  CStage* crec = reinterpret_cast<CStage*>(fsm + f.off_rec);   // [kFWarps] first gate/up item of each slot
+  DStage* drec = reinterpret_cast<DStage*>(crec + kFWarps);     // [kFWarps] first down item of each slot
+  uint32_t* keys = reinterpret_cast<uint32_t*>(fsm + f.off_route);   // [E]
+  int* sel_e = reinterpret_cast<int*>(keys + p.E);                     // [k] expert of routing rank a
+  float* sel_w = reinterpret_cast<float*>(sel_e + p.k);                // [k] its gate weight
+  float* part = reinterpret_cast<float*>(fsm + f.off_part);           // [kFWarps][32] down partial sums
   const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
   const int nb = gridDim.x, blk = blockIdx.x;
   const uint32_t row_in = (uint32_t)p.D_pad * 2, row_out = (uint32_t)p.n_pad * 2;
@@ -429,10 +502,12 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
   const int b0 = min(nrows_b, blk * f.b_per), b1 = min(nrows_b, b0 + f.b_per);
   const int e0 = min(p.D, blk * f.e_per), e1 = min(p.D, e0 + f.e_per);
 
-  // ---- prologue: weights only (may overlap the previous kernel)
-  if (tid == 0) {
-    for (int i = 0; i < kMaxBStages + 1 + 2 * kFWarps; ++i) mbar_init(bar_b + i);
-    for (int st = 0; st < f.b_nst; ++st) {
+  // ---- prologue: weights and the staging tables only (may overlap the previous kernel).
+  // Half of this block's projection rows are requested now, the rest after the
+  // logits and x loads, so that those small loads do not queue behind them.
+  const int nst_pre = (f.b_nst + 1) / 2;
+  auto issue_b = [&](int st0, int st1) {
+    for (int st = st0; st < st1; ++st) {
       const int a = b0 + st * f.b_stage, b = min(b1, a + f.b_stage);
       if (b > a) {
         mbar_expect_tx(bar_b + st, (uint32_t)(b - a) * row_in);
@@ -440,169 +515,258 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
                  (uint32_t)(b - a) * row_in, bar_b + st);
       }
     }
-    if (e1 > e0)
-      prefetch_run(reinterpret_cast<const uint8_t*>(p.basis_out) + (size_t)e0 * row_out, (uint64_t)(e1 - e0) * row_out);
+  };
+  if (tid == 0) {
+    for (int i = 0; i < kMaxBStages + 1 + 2 * kFWarps; ++i) mbar_init(bar_b + i);
+    issue_b(0, nst_pre);
+  } else if (tid == 32) {   // this block's share of the staging tables into L2
+    const uint64_t per = (f.tab_bytes / nb + 15) / 16 * 16;
+    const uint64_t o = (uint64_t)blk * per;
+    if (o < f.tab_bytes)
+      prefetch_run(reinterpret_cast<const uint8_t*>(f.cst) + o, min(per, f.tab_bytes - o));
   }
   __syncthreads();
   pdl_wait();   // x, logits, y and the workspace belong to earlier kernels until here
 
-  // ---- routing (every block), x into shared memory, zero gate/up and s
-  const RouteView rv = route_block(p, reinterpret_cast<uint32_t*>(fsm + f.off_route));
-  uint16_t* xs = reinterpret_cast<uint16_t*>(fsm + f.off_xs);
-  for (int i = tid; i < p.D_pad; i += kFThreads) xs[i] = i < p.D ? p.x[i] : (uint16_t)0;
+  // the workspace's barrier counters must be zero (only counter 0 can move before
+  // every block has passed this check)
   {
-    const size_t ng = (size_t)p.P * 2 * p.I_pad / 4, ns = (size_t)p.n_pad / 4;
-    const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (size_t i = (size_t)blk * kFThreads + tid; i < ng + ns; i += (size_t)nb * kFThreads) {
-      if (i < ng) reinterpret_cast<float4*>(p.gu)[i] = z4;
-      else reinterpret_cast<float4*>(p.s)[i - ng] = z4;
+    int* bad = reinterpret_cast<int*>(part);
+    if (tid == 0) {
+      const int v = (__ldcg(f.cnt + 1) | __ldcg(f.cnt + 2) | __ldcg(f.cnt + 3)) != 0u;
+      *bad = v;
+      if (v) atomicExch(p.status, BITSMOE_ERR_WORKSPACE_STATE);
+      else if (blk == 0) p.status[0] = 0;
     }
+    __syncthreads();
+    if (*bad) {   // compute nothing; the projection rows already requested land before the block exits
+      if (tid == 0)
+        for (int st = 0; st < nst_pre; ++st)
+          if (b0 + st * f.b_stage < b1) mbar_wait(bar_b + st, 0);
+      return;
+    }
+    __syncthreads();   // part[] is reused below
   }
-  const int A = rv.act[0];
-  const int nci = A * 2 * p.NRB * p.nseg;   // gate/up items
-  const int ndi = A * f.ul_max_tiles;        // down items (some past an expert's tiles)
-  // this block's items: i = blk + m * nb; warp w < nslot works on m = w, w + nslot, ...
-  const int mc = nci > blk ? (nci - blk + nb - 1) / nb : 0;
-  const int md = ndi > blk ? (ndi - blk + nb - 1) / nb : 0;
-  if (lane == 0) {
-    if (wid < f.nslot_c) {
-      for (int m = wid; m < mc; m += f.nslot_c) {
+
+  const int ndi = p.k * f.ul_max_tiles;   // down items of all blocks (some past an expert's tiles)
+  const int md = ndi > blk ? (ndi - blk + nb - 1) / nb : 0;   // this block's: i = blk + m * nb
+  if (wid < kBW) {
+    // ---- x into shared memory, zero gate/up and s
+    uint16_t* xs = reinterpret_cast<uint16_t*>(fsm + f.off_xs);
+    for (int i = tid; i < p.D_pad / 8; i += kBW * 32) {
+      uint4 v = make_uint4(0, 0, 0, 0);
+      if (8 * i + 8 <= p.D) {
+        v = *reinterpret_cast<const uint4*>(p.x + 8 * i);
+      } else {
+        uint16_t t[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) t[u] = 8 * i + u < p.D ? p.x[8 * i + u] : (uint16_t)0;
+        v = make_uint4(t[0] | (uint32_t)t[1] << 16, t[2] | (uint32_t)t[3] << 16, t[4] | (uint32_t)t[5] << 16,
+                       t[6] | (uint32_t)t[7] << 16);
+      }
+      reinterpret_cast<uint4*>(xs)[i] = v;
+    }
+    {
+      const size_t ng = (size_t)p.P * 2 * p.I_pad / 4, ns = (size_t)p.n_pad / 4;
+      const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (size_t i = (size_t)blk * kBW * 32 + tid; i < ng + ns; i += (size_t)nb * kBW * 32) {
+        if (i < ng) reinterpret_cast<float4*>(p.gu)[i] = z4;
+        else reinterpret_cast<float4*>(p.s)[i - ng] = z4;
+      }
+    }
+    if (tid == 0) issue_b(nst_pre, f.b_nst);
+    asm volatile("bar.sync 1, %0;" ::"r"(kBW * 32) : "memory");   // x is in shared memory
+    // ---- B: z = Phi^T x for rows [b0, b1)
+    for (int ri = wid; ri < b1 - b0; ri += kBW) {
+      const int st = ri / f.b_stage;
+      if (!mbar_wait(bar_b + st, 0)) {
+        if (lane == 0) atomicCAS(p.status, 0, BITSMOE_ERR_TIMEOUT);
+        continue;
+      }
+      const uint8_t* rp = r1 + (size_t)ri * row_in;
+      float acc = 0.f;
+      for (int c = lane; c < (p.D_pad >> 3); c += 32) {
+        const uint4 v = lds128(rp + (size_t)c * 16);
+        const uint4 xv = lds128(xs + c * 8);
+        acc = fmaf(bf16lo(v.x), bf16lo(xv.x), acc);
+        acc = fmaf(bf16hi(v.x), bf16hi(xv.x), acc);
+        acc = fmaf(bf16lo(v.y), bf16lo(xv.y), acc);
+        acc = fmaf(bf16hi(v.y), bf16hi(xv.y), acc);
+        acc = fmaf(bf16lo(v.z), bf16lo(xv.z), acc);
+        acc = fmaf(bf16hi(v.z), bf16hi(xv.z), acc);
+        acc = fmaf(bf16lo(v.w), bf16lo(xv.w), acc);
+        acc = fmaf(bf16hi(v.w), bf16hi(xv.w), acc);
+      }
+      acc = warp_sum(acc);
+      if (lane == 0) {
+        const int row = b0 + ri, h = row >= p.n, j = row - h * p.n;
+        p.z[(size_t)h * p.n_pad + j] = acc;
+      }
+    }
+  } else {
+    // ---- routing of the token: k largest logits (ties to the lower index), softmax over the k
+    const int ct = tid - kBW * 32;
+    for (int i = ct; i < p.E; i += kCT) keys[i] = order_key(p.logits[i]);
+    asm volatile("bar.sync 2, %0;" ::"r"(kCT) : "memory");
+    for (int i = ct; i < p.E; i += kCT) {
+      const uint32_t key = keys[i];
+      int rank = 0;
+      int f2 = 0;
+      for (; f2 + 4 <= p.E; f2 += 4) {
+        const uint4 o = *reinterpret_cast<const uint4*>(keys + f2);
+        rank += (o.x > key) | ((o.x == key) & (f2 < i));
+        rank += (o.y > key) | ((o.y == key) & (f2 + 1 < i));
+        rank += (o.z > key) | ((o.z == key) & (f2 + 2 < i));
+        rank += (o.w > key) | ((o.w == key) & (f2 + 3 < i));
+      }
+      for (; f2 < p.E; ++f2) {
+        const uint32_t o = keys[f2];
+        rank += (o > key) | ((o == key) & (f2 < i));
+      }
+      if (rank < p.k) {
+        sel_e[rank] = i;
+        sel_w[rank] = key ? __uint_as_float((key & 0x80000000u) ? (key & 0x7FFFFFFFu) : ~key)
+                          : __int_as_float(0x7FC00000);   // key 0: a NaN logit
+      }
+    }
+    asm volatile("bar.sync 2, %0;" ::"r"(kCT) : "memory");
+    if (ct < 32) {
+      const float m = sel_w[0];
+      const float ev = ct < p.k ? expf(sel_w[ct] - m) : 0.f;
+      float sum = ev;
+#pragma unroll
+      for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
+      __syncwarp();   // every lane has read sel_w[0]
+      if (ct < p.k) sel_w[ct] = ev * (1.f / sum);
+    }
+    // ---- staging: control thread s < nslot_c stages gate/up slot s; 32 + s < 32 + nslot_d prefetches down slot s
+    const int A = p.k;
+    const int nci = A * 2 * p.NRB * p.nseg;
+    const int mc = nci > blk ? (nci - blk + nb - 1) / nb : 0;
+    if (ct < f.nslot_c) {
+      for (int m = ct; m < mc; m += f.nslot_c) {
         const CItem ci = c_item(p, blk + m * nb);
-        const int e = rv.act[1 + ci.a];
-        const ItemRec it = p.items[((size_t)ci.h * p.E + e) * p.nseg + ci.sg];
-        if (it.nr == 0) continue;
-        if (m == wid) c_stage<G>(p, f, ci, e, it, fsm + f.off_rc + (size_t)wid * f.slot_c, bar_c + wid);
-        else c_prefetch(p, ci, e, it);
+        const CStage* g = f.cst + ((size_t)ci.h * p.E + sel_e[ci.a]) * p.nseg + ci.sg;
+        if (m == ct) {
+          copy_crec(crec + ct, g);
+          if (crec[ct].bytes) c_stage<G>(p, f, crec[ct], ci.rb, rc + (size_t)ct * f.slot_c, bar_c + ct);
+        } else {
+          const uint32_t bytes = __ldg(&g->bytes);
+          if (bytes) prefetch_run(p.img + __ldg(&g->code0) + (uint64_t)ci.rb * __ldg(&g->rb_stride), bytes);
+        }
       }
-    }
-    if (wid < f.nslot_d) {
-      for (int m = wid; m < md; m += f.nslot_d) {
-        const DItem di = d_item(f, blk + m * nb);
-        const DLoc l = d_loc(p, rv.act[1 + di.a], di.tile);
-        if (l.bits) prefetch_run(p.img + l.code, (uint64_t)p.NRB * ul_chunks(l.bits) * kChunkBytes);
+    } else if (ct >= 32 && ct < 32 + f.nslot_d) {
+      const int s = ct - 32;
+      for (int m = s; m < md; m += f.nslot_d) {
+        const int i = blk + m * nb, a = i / f.ul_max_tiles, tile = i - a * f.ul_max_tiles;
+        const DStage r = load_drec(f.dst + (size_t)sel_e[a] * f.ul_max_tiles + tile);
+        if (m == s) drec[s] = r;
+        if (r.bits) prefetch_run(p.img + r.code, (uint64_t)p.NRB * ul_chunks((int)r.bits) * kChunkBytes);
       }
+    } else if (ct == 64 && e1 > e0) {
+      prefetch_run(reinterpret_cast<const uint8_t*>(p.basis_out) + (size_t)e0 * row_out, (uint64_t)(e1 - e0) * row_out);
     }
   }
-
-  __syncthreads();   // x is in shared memory
-
-  // ---- B: z = Phi^T x for rows [b0, b1)
-  for (int ri = wid; ri < b1 - b0; ri += kFWarps) {
-    const int st = ri / f.b_stage;
-    if (!mbar_wait(bar_b + st, 0)) {
-      if (lane == 0) atomicCAS(p.status, 0, BITSMOE_ERR_TIMEOUT);
-      continue;
-    }
-    const uint8_t* rp = r1 + (size_t)ri * row_in;
-    float acc = 0.f;
-    for (int c = lane; c < (p.D_pad >> 3); c += 32) {
-      const uint4 v = lds128(rp + (size_t)c * 16);
-      const uint4 xv = lds128(xs + c * 8);
-      acc = fmaf(bf16lo(v.x), bf16lo(xv.x), acc);
-      acc = fmaf(bf16hi(v.x), bf16hi(xv.x), acc);
-      acc = fmaf(bf16lo(v.y), bf16lo(xv.y), acc);
-      acc = fmaf(bf16hi(v.y), bf16hi(xv.y), acc);
-      acc = fmaf(bf16lo(v.z), bf16lo(xv.z), acc);
-      acc = fmaf(bf16hi(v.z), bf16hi(xv.z), acc);
-      acc = fmaf(bf16lo(v.w), bf16lo(xv.w), acc);
-      acc = fmaf(bf16hi(v.w), bf16hi(xv.w), acc);
-    }
-    acc = warp_sum(acc);
-    if (lane == 0) {
-      const int row = b0 + ri, h = row >= p.n, j = row - h * p.n;
-      p.z[(size_t)h * p.n_pad + j] = acc;
-    }
-  }
-  __syncthreads();   // the projection rows are consumed: stage Phi_dn rows and down tiles there
+  __syncthreads();   // projection rows consumed, routing and first staging records in shared memory
   uint8_t* ers = r1;                       // [e1 - e0][n_pad] bf16
   uint8_t* dslots = r1 + f.off_d;          // [nslot_d][slot_d]
-  if (tid == 0) fence_proxy_async();   // generic reads of the rows above, then async writes
-  if (tid == 0 && e1 > e0) {
-    mbar_expect_tx(bar_e, (uint32_t)(e1 - e0) * row_out);
-    bulk_run(ers, reinterpret_cast<const uint8_t*>(p.basis_out) + (size_t)e0 * row_out, (uint32_t)(e1 - e0) * row_out,
-             bar_e);
-  }
-  if (lane == 0 && wid < f.nslot_d && wid < md) {
-    const DItem di = d_item(f, blk + wid * nb);
-    const DLoc l = d_loc(p, rv.act[1 + di.a], di.tile);
-    if (l.bits) d_stage(p, f, l, dslots + (size_t)wid * f.slot_d, bar_d + wid);
+  if (tid == 0) {
+    fence_proxy_async();   // generic reads of the rows above, then async writes
+    if (e1 > e0) {
+      mbar_expect_tx(bar_e, (uint32_t)(e1 - e0) * row_out);
+      bulk_run(ers, reinterpret_cast<const uint8_t*>(p.basis_out) + (size_t)e0 * row_out,
+               (uint32_t)(e1 - e0) * row_out, bar_e);
+    }
+  } else if (tid >= 32 && tid < 32 + f.nslot_d) {
+    const int s = tid - 32;
+    if (s < md && drec[s].bits) {
+      fence_proxy_async();
+      d_stage(p, f, drec[s], dslots + (size_t)s * f.slot_d, bar_d + s);
+    }
   }
   grid_barrier(f.cnt + 0, nb, p.status);
 
   // ---- C: gate/up items
   if (wid < f.nslot_c) {
+    const int A = p.k;
+    const int nci = A * 2 * p.NRB * p.nseg;
+    const int mc = nci > blk ? (nci - blk + nb - 1) / nb : 0;
     uint8_t* slot = rc + (size_t)wid * f.slot_c;
     int16_t* cq = reinterpret_cast<int16_t*>(fsm + f.off_cq) + (size_t)wid * G * f.s16;
     int nst = 0;   // items staged into this slot so far (the mbarrier completes once per staging)
     for (int m = wid; m < mc; m += f.nslot_c) {
       const CItem ci = c_item(p, blk + m * nb);
-      const int e = rv.act[1 + ci.a];
-      const int pair = rv.plist[rv.start[e]];
-      const ItemRec it = p.items[((size_t)ci.h * p.E + e) * p.nseg + ci.sg];
-      if (it.nr != 0) {
-        if (nst > 0 || m != wid) {   // not the prologue's staging: refill the slot (its last item is done)
-          __syncwarp();
-          if (lane == 0) {
-            fence_proxy_async();
-            c_stage<G>(p, f, ci, e, it, slot, bar_c + wid);
-          }
-        }
-        if (mbar_wait(bar_c + wid, (uint32_t)nst & 1u)) {
-          c_compute<G>(p, f, ci, it, slot, cq, pair, lane);
-        } else if (lane == 0) {
-          atomicCAS(p.status, 0, BITSMOE_ERR_TIMEOUT);
-        }
-        ++nst;
+      const CStage& r = crec[wid];
+      if (m != wid) {   // a later item of this slot: its record replaces the previous one
+        __syncwarp();
+        if (lane == 0) copy_crec(crec + wid, f.cst + ((size_t)ci.h * p.E + sel_e[ci.a]) * p.nseg + ci.sg);
+        __syncwarp();
       }
-      // completion of (expert slot a, row block rb): the last of its 2 * nseg items computes h
-      __threadfence();
-      __syncwarp();
-      int last = 0;
-      if (lane == 0) last = atomicAdd(f.ctr + ci.a * p.NRB + ci.rb, 1u) == (uint32_t)(2 * p.nseg - 1);
-      last = __shfl_sync(0xFFFFFFFFu, last, 0);
-      if (last) {
-        __threadfence();
-        h_rows<G>(p, f, pair, ci.rb, lane);
+      if (!r.bytes) continue;
+      if (m != wid && lane == 0) {   // refill the slot (its previous item is done)
+        fence_proxy_async();
+        c_stage<G>(p, f, r, ci.rb, slot, bar_c + wid);
       }
+      if (mbar_wait(bar_c + wid, (uint32_t)nst & 1u)) {
+        c_compute<G>(p, f, r, ci.h, ci.rb, slot, cq, ci.a, lane);
+      } else if (lane == 0) {
+        atomicCAS(p.status, 0, BITSMOE_ERR_TIMEOUT);
+      }
+      ++nst;
     }
   }
   grid_barrier(f.cnt + 1, nb, p.status);
 
-  // ---- D: down tiles, s += w * alpha * P_dn^T h
-  if (wid < f.nslot_d) {
-    uint8_t* slot = dslots + (size_t)wid * f.slot_d;
+  // ---- D: down tiles, s += w * alpha * P_dn^T h.  Warp w works on slot w % nslot_d
+  // over row blocks w / nslot_d, + nsub, ...; the slot's partial sums meet in shared memory.
+  {
+    const int nsub = kFWarps / f.nslot_d;
+    const int sl = wid % f.nslot_d, sub = wid / f.nslot_d;
+    uint8_t* slot = dslots + (size_t)sl * f.slot_d;
     int16_t* hqs = reinterpret_cast<int16_t*>(rc + (size_t)wid * f.d_h_bytes);   // C slots are free now
     float* hsc = reinterpret_cast<float*>(hqs + p.I_pad);
     int* hsum = reinterpret_cast<int*>(hsc + p.NRB);
-    int staged = 0, cur_pair = -1;
-    for (int m = wid; m < md; m += f.nslot_d) {
-      const DItem di = d_item(f, blk + m * nb);
-      const int e = rv.act[1 + di.a];
-      const DLoc l = d_loc(p, e, di.tile);
-      if (!l.bits) continue;
-      if (m != wid) {
-        __syncwarp();
-        if (lane == 0) {
-          fence_proxy_async();
-          d_stage(p, f, l, slot, bar_d + wid);
+    const int rounds = (md + f.nslot_d - 1) / f.nslot_d;
+    int staged = 0, cur_a = -1;
+    for (int rd = 0; rd < rounds; ++rd) {
+      const int m = sl + rd * f.nslot_d;
+      DStage r;
+      r.bits = 0;
+      int a = 0;
+      if (m < md) {
+        const int i = blk + m * nb, tile = i % f.ul_max_tiles;
+        a = i / f.ul_max_tiles;
+        r = rd == 0 ? drec[sl] : load_drec(f.dst + (size_t)sel_e[a] * f.ul_max_tiles + tile);
+      }
+      if (r.bits && rd > 0 && sub == 0 && lane == 0) {   // refill: the slot's previous tile is done
+        fence_proxy_async();
+        d_stage(p, f, r, slot, bar_d + sl);
+      }
+      float acc = 0.f;
+      if (r.bits) {
+        if (a != cur_a) {   // h of this expert's token for this warp's row blocks
+          h_rows<G>(p, a, sub, nsub, hqs, hsc, hsum, lane);
+          __syncwarp();
+          cur_a = a;
         }
+        if (mbar_wait(bar_d + sl, (uint32_t)staged & 1u)) {
+          acc = ul_tile_rt<G>((int)r.bits, slot + lane * 16, p.NRB, sub, nsub, p.group, hqs, hsc, hsum,
+                              reinterpret_cast<const uint32_t*>(slot + f.d_code_bytes + 256), lane);
+        } else if (lane == 0) {
+          atomicCAS(p.status, 0, BITSMOE_ERR_TIMEOUT);
+        }
+        ++staged;
       }
-      const int pair = rv.plist[rv.start[e]];
-      if (pair != cur_pair) {   // h of this expert's token: int16 rows, scales, group sums
-        __syncwarp();
-        for (int i = lane; i < p.I_pad / 8; i += 32)
-          reinterpret_cast<uint4*>(hqs)[i] = __ldcg(reinterpret_cast<const uint4*>(f.hq + (size_t)pair * p.I_pad) + i);
-        for (int i = lane; i < p.NRB; i += 32) hsc[i] = __ldcg(f.hsc + (size_t)pair * p.NRB + i);
-        for (int i = lane; i < p.NRB * G; i += 32) hsum[i] = __ldcg(f.hsum + (size_t)pair * p.NRB * G + i);
-        __syncwarp();
-        cur_pair = pair;
+      part[wid * 32 + lane] = acc;
+      __syncthreads();
+      if (r.bits && sub == 0) {
+        float t = 0.f;
+        for (int q = 0; q < nsub; ++q) t += part[(sl + q * f.nslot_d) * 32 + lane];
+        const int* su = reinterpret_cast<const int*>(slot + f.d_code_bytes);
+        const float al = reinterpret_cast<const float*>(su + 32)[lane];
+        if (al != 0.f) atomicAdd(p.s + su[lane], sel_w[a] * al * t);   // one token: s[0][j]
       }
-      if (mbar_wait(bar_d + wid, (uint32_t)staged & 1u)) {
-        d_compute<G>(p, f, l, slot, hqs, hsc, hsum, pair, rv.pw[pair], lane);
-      } else if (lane == 0) {
-        atomicCAS(p.status, 0, BITSMOE_ERR_TIMEOUT);
-      }
-      ++staged;
+      __syncthreads();
     }
   }
   grid_barrier(f.cnt + 2, nb, p.status);
@@ -639,27 +803,77 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
       }
     }
   }
-}
-
-// One block: clears the status word, the grid-barrier counters and the
-// per-(expert, row block) completion counters before the fused kernel uses
-// them.  It lets the fused kernel launch at once; the fused kernel waits for
-// this grid (and so for the previous kernel) before touching the workspace.
-__global__ void k_fused_prep(int* status, uint32_t* cnt, uint32_t* ctr, int nctr) {
-  pdl_trigger();
-  pdl_wait();
-  if (threadIdx.x == 0) status[0] = 0;
-  if (threadIdx.x < 4) cnt[threadIdx.x] = 0u;
-  for (int i = threadIdx.x; i < nctr; i += blockDim.x) ctr[i] = 0u;
+  // the last block to finish resets the barrier counters for the next call
+  if (tid == 0) {
+    const uint32_t old = atomicAdd(f.cnt + 3, 1u);
+    if (old == (uint32_t)nb - 1) {
+      f.cnt[0] = 0u;
+      f.cnt[1] = 0u;
+      f.cnt[2] = 0u;
+      __threadfence();
+      f.cnt[3] = 0u;
+    }
+  }
 }
 
 }  // namespace
 
 namespace bmoe {
 
+void build_stage_tables(const uint8_t* img, std::vector<CStage>& cst, std::vector<DStage>& dst) {
+  const ImageHeader& hd = *header_of(img);
+  const ExpertDesc* desc = desc_of(img);
+  const ItemRec* items = reinterpret_cast<const ItemRec*>(img + hd.off_items);
+  const int E = hd.E;
+  cst.assign(2 * (size_t)E * hd.nseg, CStage{});
+  for (int pi = 0; pi < 2 * E; ++pi) {
+    const ExpertDesc& x = desc[pi];
+    for (int q = 0; q < hd.nseg; ++q) {
+      const ItemRec& it = items[(size_t)pi * hd.nseg + q];
+      CStage& r = cst[(size_t)pi * hd.nseg + q];
+      if (it.nr == 0) continue;
+      r.code0 = x.code_base + it.byte0;
+      r.unit0 = x.unit_off + (uint64_t)it.slot0 * 4;
+      r.alpha0 = x.alpha_off + (uint64_t)it.slot0 * 4;
+      r.sz0 = x.sz_off + (uint64_t)it.slot0 * 4;
+      r.rb_stride = (uint32_t)x.rb_stride;
+      r.sz_row = (uint32_t)x.nslots * 4;
+      r.bytes = it.bytes;
+      r.mb = (uint32_t)it.nslot * 4;
+      r.nr = it.nr;
+      int nls = 0;
+      for (int k = 0; k < it.nr && k < kNumBk; ++k) {
+        r.bits[k] = it.bits[k];
+        r.ntl[k] = it.ntl[k];
+        if (it.bits[k] < 16) nls += it.ntl[k] * rl_units(it.bits[k]);
+      }
+      r.nls = (uint16_t)nls;
+    }
+  }
+  dst.assign((size_t)E * hd.ul_max_tiles, DStage{});
+  for (int e = 0; e < E; ++e) {
+    const ExpertDesc& x = desc[2 * E + e];
+    for (int k = 0; k < x.nbk; ++k) {
+      const BucketDesc& bd = x.bk[k];
+      for (int t = 0; t < bd.ntiles; ++t) {
+        const int tile = bd.tile0 + t;
+        if (tile >= hd.ul_max_tiles) continue;
+        DStage& r = dst[(size_t)e * hd.ul_max_tiles + tile];
+        const uint64_t slot = (uint64_t)bd.slot0 + (uint64_t)t * 32;
+        r.code = x.code_base + bd.code_off + (uint64_t)t * hd.NRB * ul_chunks(bd.bits) * kChunkBytes;
+        r.unit = x.unit_off + slot * 4;
+        r.alpha = x.alpha_off + slot * 4;
+        r.sz = x.sz_off + slot * 4;
+        r.sz_row = (uint32_t)x.nslots * 4;
+        r.bits = (uint32_t)bd.bits;
+      }
+    }
+  }
+}
+
 bool fused_plan(const ImageHeader& hd, int T, int top_k, int seg_bytes, int ul_max_chunks, int s16, int sms,
                 FusedArgs* f) {
-  if (T != 1 || sms < 1) return false;
+  if (T != 1 || sms < 1 || top_k > 32) return false;
   std::memset(f, 0, sizeof(*f));
   const int G = std::max(1, kRows / hd.group);
   const size_t row_in = (size_t)hd.D_pad * 2, row_out = (size_t)hd.n_pad * 2;
@@ -677,23 +891,29 @@ bool fused_plan(const ImageHeader& hd, int T, int top_k, int seg_bytes, int ul_m
   f->d_code_bytes = hd.NRB * ul_max_chunks * kChunkBytes;
   f->slot_d = (int)align_up((uint64_t)f->d_code_bytes + 256 + (uint64_t)hd.NG * 128, 128);
   f->d_h_bytes = (int)align_up((uint64_t)hd.I_pad * 2 + (uint64_t)hd.NRB * 4 * (1 + G), 128);
+  if (hd.ul_max_tiles < 1) return false;
   const int items_c = (A * 2 * hd.NRB * hd.nseg + sms - 1) / sms;
   const int items_d = (A * hd.ul_max_tiles + sms - 1) / sms;
-  // fixed areas: mbarriers, routing, x, the per-warp int16 activation tables
+  // fixed areas: mbarriers, staging records, routing, x, per-warp int16 activation tables, down partial sums
   size_t off = 512;
+  f->off_rec = (int)off;
+  off = align_up(off + (size_t)kFWarps * (sizeof(CStage) + sizeof(DStage)), 128);
   f->off_route = (int)off;
-  off = align_up(off + (size_t)(T * hd.E + 3 * T * top_k + 3 * hd.E + 3) * 4, 128);
+  off = align_up(off + (size_t)(hd.E + 2 * top_k) * 4, 128);
   f->off_xs = (int)off;
   off = align_up(off + row_in, 128);
   f->off_cq = (int)off;
   off = align_up(off + (size_t)kFWarps * G * s16 * 2, 128);
+  f->off_part = (int)off;
+  off = align_up(off + (size_t)kFWarps * 32 * 4, 128);
   const size_t r_b = (size_t)f->b_per * row_in;
   const size_t r_e = align_up((size_t)f->e_per * row_out, 128);
   f->off_d = (int)r_e;
-  int nslot_d = std::min(std::max(items_d, 1), kFWarps);
+  int nslot_d = 1;   // a power of two: the warps split evenly over the down slots
+  while (nslot_d * 2 <= std::min(items_d, kFWarps)) nslot_d *= 2;
   size_t r1 = std::max(r_b, r_e + (size_t)nslot_d * f->slot_d);
   while (nslot_d > 1 && off + r1 > budget) {
-    --nslot_d;
+    nslot_d /= 2;
     r1 = std::max(r_b, r_e + (size_t)nslot_d * f->slot_d);
   }
   f->off_r1 = (int)off;
@@ -702,7 +922,7 @@ bool fused_plan(const ImageHeader& hd, int T, int top_k, int seg_bytes, int ul_m
   if (off >= budget) return false;
   int nslot_c = std::min(std::max(items_c, 1), kFWarps);
   while (nslot_c > 1 && off + (size_t)nslot_c * f->slot_c > budget) --nslot_c;
-  size_t rc = std::max({(size_t)nslot_c * f->slot_c, (size_t)nslot_d * f->d_h_bytes, row_out * 2});
+  size_t rc = std::max({(size_t)nslot_c * f->slot_c, (size_t)kFWarps * f->d_h_bytes, row_out * 2});
   if (off + rc > budget) return false;
   f->nslot_c = nslot_c;
   f->nslot_d = nslot_d;
@@ -710,22 +930,10 @@ bool fused_plan(const ImageHeader& hd, int T, int top_k, int seg_bytes, int ul_m
   return true;
 }
 
-cudaError_t launch_fused(const Fwd& p, const FusedArgs& f, int nctr, int sms, cudaStream_t st, bool pdl) {
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(1);
-  cfg.blockDim = dim3(256);
-  cfg.dynamicSmemBytes = 0;
-  cfg.stream = st;
-  cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 1 : 0;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, k_fused_prep, p.status, f.cnt, f.ctr, nctr);
-  if (e != cudaSuccess) return e;
-  const int G = std::max(1, kRows / p.group);
+cudaError_t launch_fused(const Fwd& p, const FusedArgs& f, int sms, cudaStream_t st, bool pdl) {
   static std::mutex mu;
   static int done_smem[3] = {0, 0, 0};
+  const int G = std::max(1, kRows / p.group);
   auto go = [&](void (*kernel)(Fwd, FusedArgs), int gi) -> cudaError_t {
     {
       std::lock_guard<std::mutex> lock(mu);
@@ -737,16 +945,16 @@ cudaError_t launch_fused(const Fwd& p, const FusedArgs& f, int nctr, int sms, cu
         done_smem[gi] = f.smem;
       }
     }
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
     cudaLaunchConfig_t c2 = {};
     c2.gridDim = dim3(sms);
     c2.blockDim = dim3(kFThreads);
     c2.dynamicSmemBytes = f.smem;
     c2.stream = st;
-    cudaLaunchAttribute a2[1];
-    a2[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    a2[0].val.programmaticStreamSerializationAllowed = 1;
-    c2.attrs = a2;
-    c2.numAttrs = 1;   // always: the prep kernel triggers at once
+    c2.attrs = attr;
+    c2.numAttrs = pdl ? 1 : 0;
     return cudaLaunchKernelEx(&c2, kernel, p, f);
   };
   if (G == 1) return go(k_fused<1>, 0);

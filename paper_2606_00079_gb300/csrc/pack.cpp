@@ -561,6 +561,7 @@ const char* bitsmoe_strerror(int code) {
     case BITSMOE_ERR_TIMEOUT: return "device wait timed out";
     case BITSMOE_ERR_DEVICE_BOUNDS: return "device bounds check failed";
     case BITSMOE_ERR_BLOB: return "malformed packed blob";
+    case BITSMOE_ERR_WORKSPACE_STATE: return "workspace not zero-filled before its first use";
     default: return "unknown error";
   }
 }

@@ -1,12 +1,12 @@
-"""GPU parity of the fused single-token decode kernel (prep kernel + one
-persistent kernel with grid barriers) against the fp64 oracle.
+"""GPU parity of the fused single-token decode kernel (one persistent kernel
+with grid barriers) against the fp64 oracle.
 
 The fused path runs whenever T == 1 and the layer's per-block shares fit in
 shared memory; these cases check that it was taken and cover every bit-width,
 group size, evicted units and experts, extreme top-k, consecutive calls and
-different layers on one workspace, a workspace full of garbage (the prep
-kernel must reset what the kernel's barriers count on), and replay from a CUDA
-graph.  Bar: max|y_gpu - y_ref| / ||y_ref||_inf <= 2e-3.
+different layers on one workspace, a workspace that was not zero-filled (the
+call must refuse it with a status, not compute), and replay from a CUDA graph.
+Bar: max|y_gpu - y_ref| / ||y_ref||_inf <= 2e-3.
 """
 import numpy as np
 import pytest
@@ -43,7 +43,7 @@ def small(**kw):
 
 def run(env, L, x, logits, k, ws=None):
     torch, bm = env
-    assert bm.bitsmoe_forward_launches(L, x.shape[0], k) == 2, "fused path not taken"
+    assert bm.bitsmoe_forward_launches(L, x.shape[0], k) == 1, "fused path not taken"
     xd = torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).cuda()
     ld = torch.from_numpy(np.ascontiguousarray(logits)).cuda()
     if ws is None:
@@ -103,17 +103,37 @@ def test_fused_top1_and_all_experts(env):
         check(env, layer, x, logits, k, L=L)
 
 
-def test_fused_consecutive_calls_layers_and_garbage_workspace(env):
+def test_fused_consecutive_calls_layers_and_workspace_state(env):
     torch, bm = env
     spec = synth.scaled_spec(synth.WORKLOADS["qw3"], D=512, E=32, I=384, n=512, top_k=4)
     layers = [synth.make_layer(spec, seed=s) for s in (21, 22)]
     Ls = [bm.bitsmoe_pack(l, device=0) for l in layers]
     ws = bm.Workspace(Ls[0], 1, spec.top_k)
-    ws.buf.fill_(0xA5)                    # garbage: counters and status must be reset per call
+    # a workspace that was not zero-filled: the call reports it and leaves y alone
+    ws.buf.fill_(0xA5)
+    x, logits = synth.make_inputs(spec, 1, seed=3, step=0)
+    xd = torch.from_numpy(x.view(np.int16)).cuda()
+    ld = torch.from_numpy(logits).cuda()
+    y = torch.full((1, spec.D), 7.0, dtype=torch.float32, device="cuda")
+    bm.moe_forward(Ls[0], xd, ld, spec.top_k, ws=ws, y=y)
+    torch.cuda.synchronize()
+    assert bm.bitsmoe_last_device_status(ws.ptr) == bm.ERR_CODE["WORKSPACE_STATE"]
+    assert bool((y == 7.0).all())
+    # zero-filled: consecutive calls on two layers share it (the kernel leaves its counters at zero)
+    ws.buf.zero_()
     for step in range(6):
         i = step % 2
         x, logits = synth.make_inputs(spec, 1, seed=3, step=step)
         check(env, layers[i], x, logits, spec.top_k, L=Ls[i], ws=ws)
+    # a multi-token call (kernel chain) on the same workspace does not disturb the counters
+    ws4 = bm.Workspace(Ls[0], 4, spec.top_k)
+    x4, l4 = synth.make_inputs(spec, 4, seed=3, step=9)
+    y4 = bm.moe_forward(Ls[0], torch.from_numpy(x4.view(np.int16)).cuda(), torch.from_numpy(l4).cuda(),
+                        spec.top_k, ws=ws4)
+    x, logits = synth.make_inputs(spec, 1, seed=3, step=10)
+    check(env, layers[0], x, logits, spec.top_k, L=Ls[0], ws=ws4)
+    ref4 = oracle.moe_forward_factored(layers[0], x4, l4, spec.top_k)
+    assert rel_err(y4.cpu().numpy().astype(np.float64), ref4) <= TOL
 
 
 def test_fused_graph_replay(env):
@@ -149,7 +169,7 @@ def test_fused_plan_taken_for_qw3_dims_not_for_d4096(env):
     torch, bm = env
     qw3 = synth.scaled_spec(synth.WORKLOADS["qw3"], E=8, top_k=8)   # full qw3 dims, fewer experts
     L = bm.bitsmoe_pack(synth.make_layer(qw3, seed=1), device=0)
-    assert bm.bitsmoe_forward_launches(L, 1, 8) == 2
+    assert bm.bitsmoe_forward_launches(L, 1, 8) == 1
     assert bm.bitsmoe_forward_launches(L, 2, 8) == 5
     # D = n = 4096: a block's share of the input bases (54 rows of 8 KB) exceeds shared memory
     big = synth.scaled_spec(synth.WORKLOADS["mixtral"], E=2, I=128, top_k=1)
