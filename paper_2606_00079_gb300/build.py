@@ -1,8 +1,9 @@
 """Build libbitsmoe.so in-tree with nvcc for sm_103a (GB300).
 
-Three translation units, compiled in parallel: the host packer (pack.cpp,
-plain C++), the CUDA kernel chain + C ABI (forward.cu) and the fused
-single-token decode kernel (fused.cu).  The CUDA runtime is linked
+Four translation units, compiled in parallel: the host packer (pack.cpp,
+plain C++), the CUDA kernel chain + C ABI (forward.cu), the fused
+single-token decode kernel (fused.cu) and the tensor-core projections
+(gemm.cu).  The CUDA runtime is linked
 statically, so the library loads on a machine without a GPU (the host-only
 entry points then work; the device ones return BITSMOE_ERR_CUDA).
 """
@@ -37,7 +38,7 @@ def _run(cmd):
 
 
 def sources():
-    return [os.path.join(CSRC, f) for f in ("pack.cpp", "forward.cu", "fused.cu")]
+    return [os.path.join(CSRC, f) for f in ("pack.cpp", "forward.cu", "fused.cu", "gemm.cu")]
 
 
 def up_to_date() -> bool:

@@ -92,6 +92,12 @@ bool fused_plan(const ImageHeader& hd, int T, int top_k, int seg_bytes, int ul_m
                 FusedArgs* f);
 // Prep kernel + fused kernel on `st` (grid = sms blocks).
 cudaError_t launch_fused(const Fwd& p, const FusedArgs& f, int sms, cudaStream_t st, bool pdl);
+// Tensor-core projections (gemm.cu): a TMA map of a bf16 basis [rows][cols_pad]
+// (128 bytes, written to map_out), and the launch of z += Phi^T x (mode 0) or
+// y += Phi_dn s (mode 1) for all T tokens of p (z, resp. y, zeroed before
+// unless y carries a residual).
+bool make_basis_map(void* map_out, const void* base, int rows, int cols_pad);
+cudaError_t launch_gemm_tc(int mode, const void* map, const Fwd& p, int sms, cudaStream_t st, bool pdl);
 // Staging records of a packed image (host side, at upload).
 void build_stage_tables(const uint8_t* img, std::vector<CStage>& cst, std::vector<DStage>& dst);
 

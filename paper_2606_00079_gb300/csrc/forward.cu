@@ -47,6 +47,9 @@ struct bitsmoe_layer {
   const CStage* d_cst = nullptr;
   const DStage* d_dst = nullptr;
   uint64_t stage_bytes = 0;
+  alignas(64) uint8_t map_in[128];    // TMA maps of the two input bases and of the output basis
+  alignas(64) uint8_t map_out[128];
+  bool maps = false;
   std::vector<uint8_t> meta;   // host copy of header + descriptors + segment table
   int seg_bytes = 0;           // largest gate/up item: code bytes inside one row block
   int ul_max_chunks = 1;       // largest 16-byte chunks per row block of any down unit
@@ -231,22 +234,26 @@ __global__ void __launch_bounds__(kThreads) k_route_publish(Fwd p) {
 // ---------------------------------------------------------------------------
 // K0: routing.  k largest logits per token (ties to the lower expert index),
 // gate weights = softmax over the selected k, then a stable grouping of the
-// (token, slot) pairs p = t * k + slot by expert.
+// (token, slot) pairs p = t * k + slot by expert.  Blocks select for tpb
+// tokens each; the last block to finish (a counter in the workspace, which it
+// resets) groups all pairs and publishes the routing with a release flag.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(1024) k_router(Fwd p) {
+  if (blockIdx.x == 0 && threadIdx.x == 0) {   // before the trigger: no later kernel may see the previous flag
+    p.status[0] = 0;
+    p.route_flag[0] = 0;
+    __threadfence();
+  }
+  __syncthreads();
   pdl_trigger();
-  // shared: keys [tpb][E] | pair expert [P] | pair logit/weight [P] | count [E] | start [E+1]
+  // shared: keys [tpb][E] | pair expert [P] | count [E] | start [E+1]
   extern __shared__ uint32_t keys[];
+  __shared__ int last;
   const int E = p.E, k = p.k, T = p.T, P = p.P;
   const int tid = threadIdx.x;
   const int tpb = max(1, (int)blockDim.x / E);
-  int* s_pe = reinterpret_cast<int*>(keys + tpb * E);
-  float* s_pw = reinterpret_cast<float*>(s_pe + P);
-  int* s_cnt = reinterpret_cast<int*>(s_pw + P);
-  int* s_start = s_cnt + E;
-  if (tid == 0) *p.status = 0;
-  for (int t0 = 0; t0 < T; t0 += tpb) {
-    const int tt = tid / E, e = tid - tt * E, t = t0 + tt;
+  {   // this block's tokens
+    const int tt = tid / E, e = tid - tt * E, t = blockIdx.x * tpb + tt;
     const bool valid = tt < tpb && t < T;
     float lg = 0.f;
     if (valid) {
@@ -263,24 +270,36 @@ __global__ void __launch_bounds__(1024) k_router(Fwd p) {
         rank += (o > key) | ((o == key) & (f < e));
       }
       if (rank < k) {
-        s_pe[t * k + rank] = e;
-        s_pw[t * k + rank] = lg;
+        p.pair_expert[t * k + rank] = e;
+        reinterpret_cast<float*>(keys)[tpb * E + tt * k + rank] = lg;   // logits of the selected, in rank order
       }
     }
     __syncthreads();
-  }
-  for (int t = tid; t < T; t += blockDim.x) {
-    float* w = s_pw + (size_t)t * k;
-    const float m = w[0];
-    float sum = 0.f;
-    for (int r = 0; r < k; ++r) sum += expf(w[r] - m);
-    const float inv = 1.f / sum;
-    for (int r = 0; r < k; ++r) {
-      const float v = expf(w[r] - m) * inv;
-      p.pair_weight[t * k + r] = v;
-      p.pair_expert[t * k + r] = s_pe[t * k + r];
+    for (int q = tid; q < tpb * k; q += blockDim.x) {   // softmax over the k selected of each token
+      const int t2 = blockIdx.x * tpb + q / k, r = q - (q / k) * k;
+      if (t2 >= T) continue;
+      const float* w = reinterpret_cast<const float*>(keys) + tpb * E + (q / k) * k;
+      const float m = w[0];
+      float sum = 0.f;
+      for (int r2 = 0; r2 < k; ++r2) sum += expf(w[r2] - m);
+      p.pair_weight[t2 * k + r] = expf(w[r] - m) * (1.f / sum);
     }
   }
+  __syncthreads();
+  if (tid == 0) {
+    __threadfence();
+    const int old = atomicAdd(p.status + 2, 1);
+    last = old == (int)gridDim.x - 1;
+    if (last) p.status[2] = 0;   // reset for the next call
+  }
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  int* s_pe = reinterpret_cast<int*>(keys);   // reuse: all pairs' experts
+  int* s_cnt = s_pe + P;
+  int* s_start = s_cnt + E;
+  for (int q = tid; q < P; q += blockDim.x) s_pe[q] = __ldcg(p.pair_expert + q);
+  __syncthreads();
   const int warp = tid >> 5, lane = tid & 31, nw = blockDim.x >> 5;
   for (int e = warp; e < E; e += nw) {
     int c = 0;
@@ -327,6 +346,11 @@ __global__ void __launch_bounds__(1024) k_router(Fwd p) {
       if (m) p.pair_list[base + __popc(b & ((1u << lane) - 1u))] = q;
       base += __popc(b);
     }
+  }
+  __syncthreads();
+  if (tid == 0) {   // the routing is published: kernels that stage by it may go on
+    __threadfence();
+    st_release(p.route_flag, 1);
   }
 }
 
@@ -1079,6 +1103,7 @@ __global__ void __launch_bounds__(kK2DecWarps * 32) k_gateup_dec(Fwd p) {
 #pragma unroll
       for (int u = 1; u < kDecMaxT; ++u)
         if (u == q) pv = plist[u];
+      if (q >= kDecMaxT) pv = p.pair_list[pst + q];   // more tokens than the prologue held
       pair[tt] = pv;
       zrow[tt] = p.z + ((size_t)h * p.T + pair[tt] / p.k) * p.n_pad;
     }
@@ -1333,6 +1358,7 @@ __global__ void __launch_bounds__(kK3DecWarps * 32) k_down_dec(Fwd p) {
 #pragma unroll
           for (int u = 1; u < kDecMaxT; ++u)
             if (u == tb0 + tt) pr = plist[u];
+          if (tb0 + tt >= kDecMaxT) pr = p.pair_list[pst + tb0 + tt];
           const float g = p.gu[((size_t)pr * 2) * p.I_pad + row0 + i];
           const float u = p.gu[((size_t)pr * 2 + 1) * p.I_pad + row0 + i];
           v = g / (1.f + __expf(-g)) * u;
@@ -1409,6 +1435,10 @@ __global__ void __launch_bounds__(kK3DecWarps * 32) k_down_dec(Fwd p) {
               pr = plist[u];
               wv = pwt[u];
             }
+          if (tb0 + tt >= kDecMaxT) {
+            pr = p.pair_list[pst + tb0 + tt];
+            wv = p.pair_weight[pr];
+          }
           const float scale = shs[tt] * (1.f / 32767.f);
           atomicAdd(p.s + (size_t)(pr / p.k) * p.n_pad + j, wv * al * scale * accf[tt]);
         }
@@ -1665,7 +1695,7 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
   p.seg_bytes = L->seg_bytes;
   // decode mode: every kernel can afford the routing of all tokens
   p.decode = T <= 8 && T * hd.E <= 4096;
-  if (p.decode) {   // down staging: keep a warp's tile within ~48 KB of shared memory
+  {   // down staging: keep a warp's tile within ~48 KB of shared memory
     const int need = std::max(1, hd.group / kRows);
     int rbc = std::min(p.rbc, std::max(1, (48 * 1024) / (L->ul_max_chunks * kChunkBytes)));
     rbc = std::max(need, rbc / need * need);
@@ -1733,20 +1763,36 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
     return mark(5);
   }
   const int tpb = std::max(1, 1024 / hd.E);
-  const size_t router_smem = ((size_t)tpb * hd.E + 2 * (size_t)p.P + 2 * (size_t)hd.E + 1) * 4;
+  const size_t router_smem =
+      std::max((size_t)tpb * (hd.E + top_k), (size_t)p.P + 2 * (size_t)hd.E + 1) * 4;   // selection | grouping
   if (router_smem > 200 * 1024) return BITSMOE_ERR_SHAPE;
   if ((rc = mark(0))) return rc;
   if ((rc = set_smem(k_router, router_smem))) return rc;
-  if ((rc = launch(k_router, dim3(1), dim3(1024), router_smem, st, false, p))) return rc;
+  if ((rc = launch(k_router, dim3((T + tpb - 1) / tpb), dim3(1024), router_smem, st, false, p))) return rc;
   if ((rc = mark(1))) return rc;
-  if ((rc = launch_gemv_any(true, p, sms, st, pdl))) return rc;
+  const bool tc = L->maps;   // tensor-core projections for multi-token calls
+  if (tc) {
+    // the projection, the gate/up and the down kernels add into z, gu and s (adjacent in
+    // the workspace); the output basis adds into y (which keeps the residual when accumulating)
+    BM_CK(cudaMemsetAsync(p.z, 0, (size_t)(reinterpret_cast<uint8_t*>(p.s) - reinterpret_cast<uint8_t*>(p.z)) +
+                                      (size_t)T * hd.n_pad * 4, st));
+    if (!accum) BM_CK(cudaMemsetAsync(y, 0, (size_t)T * hd.D * 4, st));
+    BM_CK(launch_gemm_tc(0, L->map_in, p, sms, st, false));
+  } else if ((rc = launch_gemv_any(true, p, sms, st, pdl))) {
+    return rc;
+  }
   if ((rc = mark(2))) return rc;
-  if (G == 1) rc = launch_k2k3_tb<1>(p, sms, st, pdl, ev ? [&]() { return mark(3); } : std::function<int()>());
-  else if (G == 2) rc = launch_k2k3_tb<2>(p, sms, st, pdl, ev ? [&]() { return mark(3); } : std::function<int()>());
-  else rc = launch_k2k3_tb<4>(p, sms, st, pdl, ev ? [&]() { return mark(3); } : std::function<int()>());
+  {   // gate/up and down factors: the staged kernels, every routed expert's tokens in batches of 4
+    std::function<int()> between = ev ? std::function<int()>([&]() { return mark(3); }) : std::function<int()>();
+    const int A_max = std::min(hd.E, p.P);
+    if (G == 1) rc = launch_k2k3_dec<1, 4>(p, A_max, sms, st, pdl, between);
+    else if (G == 2) rc = launch_k2k3_dec<2, 4>(p, A_max, sms, st, pdl, between);
+    else rc = launch_k2k3_dec<4, 4>(p, A_max, sms, st, pdl, between);
+  }
   if (rc) return rc;
   if ((rc = mark(4))) return rc;
-  if ((rc = launch_gemv_any(false, p, sms, st, pdl))) return rc;
+  if (tc) BM_CK(launch_gemm_tc(1, L->map_out, p, sms, st, pdl));
+  else if ((rc = launch_gemv_any(false, p, sms, st, pdl))) return rc;
   return mark(5);
 }
 
@@ -1793,6 +1839,11 @@ int upload(std::vector<uint8_t>&& img, int device, bitsmoe_layer** out) {
   L->d_cst = reinterpret_cast<const CStage*>(ds);
   L->d_dst = reinterpret_cast<const DStage*>(ds + cst_bytes);
   L->stage_bytes = cst_bytes + dst_bytes;
+  {
+    const ImageHeader* h = header_of(img.data());
+    L->maps = make_basis_map(L->map_in, d + h->off_basis_in, 2 * h->n, h->D_pad) &&
+              make_basis_map(L->map_out, d + h->off_basis_out, h->D, h->n_pad);
+  }
   const ImageHeader* hd = header_of(img.data());
   const size_t meta_end = hd->off_basis_in;   // header + descriptors + segments
   L->device = device;
