@@ -57,6 +57,23 @@ def measured_peaks():
         return {"hbm_gbs": FALLBACK_HBM_GBS}, "fallback"
 
 
+def measured_traffic(profile, sources):
+    """DRAM bytes per launch of a kernel from a committed ncu summary, or None when
+    the kernel's sources changed since that capture (the summary records their hash)."""
+    import hashlib
+    try:
+        lines = open(os.path.join(ROOT, "profiles", profile)).read().splitlines()
+        kv = dict(l.split(":", 1) for l in lines if ":" in l and not l.startswith("#"))
+        h = hashlib.sha256()
+        for src in sources:
+            h.update(open(os.path.join(ROOT, "paper_2606_00079_gb300", "csrc", src), "rb").read())
+        if kv.get("source_sha256", "").strip() != h.hexdigest():
+            return None
+        return int(kv["dram_bytes_per_launch"].strip())
+    except Exception:
+        return None
+
+
 def dist_env():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -461,8 +478,10 @@ def main():
         # one fused kernel does the whole step: its average duration is at most the timed region per
         # step (which also holds the gap between launches), so this is a lower bound
         achieved = (total_bytes / args.steps) / (ms / args.steps / 1e3) / 1e9
+        traffic = measured_traffic("ncu_full_k_fused_qw3_T1.txt", ("fused.cu", "device.cuh", "format.h"))
         roofline = {"bound": "hbm", "kernel": "k_fused (whole single-token forward)", "achieved": achieved,
-                    "peak": peak, "peak_source": peak_src, "unit": "GB/s", "frac": achieved / peak, "traffic": None,
+                    "peak": peak, "peak_source": peak_src, "unit": "GB/s", "frac": achieved / peak,
+                    "traffic": traffic,
                     "bytes_per_launch": total_bytes / args.steps,
                     "duration_us": ms / args.steps * 1e3,
                     "duration_source": "CUDA events over the timed region / steps",

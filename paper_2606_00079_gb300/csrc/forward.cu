@@ -1,24 +1,26 @@
-// BitsMoE quantized MoE-layer forward on sm_103a (GB300).
+// BitsMoE quantized MoE-layer forward on sm_103a (GB300): the kernel chains
+// and the C ABI.
 //
 // Stage 3 of the method (Fig. 1; "Inference Efficiency", Sec. Experiments):
 // the activation is projected once onto the shared bases, then each routed
 // expert's packed spectral factors are unpacked and applied inside the kernels
-// without rebuilding the expert weights.  Phases, one kernel each, chained on
-// the caller's stream with programmatic dependent launch (PDL) so that a
-// kernel's prologue overlaps the tail of the previous one:
+// without rebuilding the expert weights.  A call runs one of three plans
+// (forward_impl), kernels chained on the caller's stream with programmatic
+// dependent launch (PDL) so that a kernel's prologue overlaps the tail of the
+// previous one:
 //
-//   K0 k_router     top-k over the logits, softmax over the selected k, and
-//                   token -> expert grouping (counts, offsets, pair lists)
-//   K1 k_gemv<P>    z_g = Phi_g^T x, z_u = Phi_u^T x (bf16 rows streamed with
-//                   128-bit loads); zeroes the accumulators; then prefetches
-//                   the routed experts' packed factors and Phi_dn into L2
-//   K2 k_gateup     gate/up = P_hat (alpha * z): mixed-bit dequant-GEMV over
-//                   bucketed uniform-bit streams; in-register unpacking and
-//                   dp2a integer dot products (int16 activation operand),
-//                   fp32 partials reduced with vector red.add
-//   K3 k_down       h = SiLU(gate) * up (fused into the prologue), then
-//                   s += w_e * alpha_dn * (P_hat_dn^T h) per unit
-//   K4 k_gemv<O>    y = Phi_dn s (fp32 out)
+//   one token      k_fused (fused.cu): the whole layer in one persistent kernel
+//   2 .. 8 tokens  k_route_publish   routing by one block, published with a flag
+//                  k_gemv_bulk<P>    z_g = Phi_g^T x, z_u = Phi_u^T x (rows through
+//                                    a bulk-copy ring); zeroes the accumulators
+//                  k_gateup_dec      gate/up = P_hat (alpha * z): dp2a over
+//                                    bucketed uniform-bit streams staged per warp
+//                                    item, int16 activation operand, vector red.add
+//                  k_down_dec        h = SiLU(gate) * up, then
+//                                    s += w_e * alpha_dn * (P_hat_dn^T h) per unit
+//                  k_gemv_bulk<O>    y = Phi_dn s (fp32 out)
+//   more tokens    k_router (multi-block), k_gemm_tc (gemm.cu: tensor cores) for
+//                  both projections, the same gate/up and down kernels
 //
 // The identity behind the association is Eq. app_normalized_decomposition
 // (W = P A Phi^T for gate/up, W = Phi A P^T for down); summing the experts'
@@ -647,176 +649,12 @@ __global__ void __launch_bounds__(kThreads) k_gemv_bulk(Fwd p, int stage_rows) {
 // The lane owns 4 rows; c of the segment's units is quantised to int16 with
 // one scale per (item, token), so the inner loop is dp2a over unpacked code
 // bytes; the zero-point term sum_j c_jg zero_jg is applied once per item.
-// ---------------------------------------------------------------------------
-struct Range {
-  int bi;     // bucket index in the expert descriptor
-  int lo, hi; // bucket-local tile range
-  int ls0;    // local slot base of this range in the item's c table
-};
-
-
-template <int G, int TB>
-__global__ void __launch_bounds__(kThreads) k_gateup(Fwd p) {
-  pdl_trigger();
-  pdl_wait();
-  extern __shared__ int4 smem_k2[];
-  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-  int16_t* cq = reinterpret_cast<int16_t*>(smem_k2) + (size_t)wid * G * TB * p.s16;
-  const int A = p.active[0];
-  const int per_e = 2 * p.NRB * p.nseg;
-  const int total = A * per_e;
-  const int gl_lane = G == 1 ? 0 : (4 * lane) / p.group;   // lane's group inside the row block
-  for (int item = blockIdx.x * kWarps + wid; item < total; item += gridDim.x * kWarps) {
-    const int a = item / per_e;
-    int r = item - a * per_e;
-    const int h = r / (p.NRB * p.nseg);
-    r -= h * p.NRB * p.nseg;
-    const int rb = r / p.nseg, sg = r - rb * p.nseg;
-    const int e = p.active[1 + a];
-    const int32_t* segp = p.seg + ((size_t)h * p.E + e) * (p.nseg + 1);
-    const int t0 = segp[sg], t1 = segp[sg + 1];
-    if (t0 >= t1) continue;
-    const ExpertDesc& xd = p.desc[h * p.E + e];
-    const int32_t* unit = reinterpret_cast<const int32_t*>(p.img + xd.unit_off);
-    const float* alpha = reinterpret_cast<const float*>(p.img + xd.alpha_off);
-    // tile ranges of this item, per bucket
-    Range rg[kNumBk];
-    int nr = 0, nls = 0;
-    for (int bi = 0; bi < xd.nbk; ++bi) {
-      const BucketDesc& bd = xd.bk[bi];
-      const int lo = max(t0, bd.tile0) - bd.tile0, hi = min(t1, bd.tile0 + bd.ntiles) - bd.tile0;
-      if (lo < hi) {
-        rg[nr] = Range{bi, lo, hi, nls};
-        if (bd.bits < 16) nls += (hi - lo) * rl_units(bd.bits);
-        ++nr;
-      }
-    }
-    const int g_base = (rb * kRows) / p.group;
-    const int ntok = p.expert_count[e], pst = p.expert_start[e];
-    for (int tb0 = 0; tb0 < ntok; tb0 += TB) {
-      const int tb = min(TB, ntok - tb0);
-      int pair[TB];
-      const float* zrow[TB];
-#pragma unroll
-      for (int tt = 0; tt < TB; ++tt) {
-        pair[tt] = p.pair_list[pst + tb0 + min(tt, tb - 1)];
-        zrow[tt] = p.z + ((size_t)h * p.T + pair[tt] / p.k) * p.n_pad;
-      }
-      // pass 1: max |c| per token over the item's quantised units
-      float mx[TB];
-#pragma unroll
-      for (int tt = 0; tt < TB; ++tt) mx[tt] = 0.f;
-      for (int ri = 0; ri < nr; ++ri) {
-        const BucketDesc& bd = xd.bk[rg[ri].bi];
-        if (bd.bits == 16) continue;
-        const int U = rl_units(bd.bits), s0 = rg[ri].lo * U, ns = (rg[ri].hi - rg[ri].lo) * U;
-        const uint32_t* sz = reinterpret_cast<const uint32_t*>(p.img + bd.sz_off);
-        for (int i = lane; i < ns; i += 32) {
-          const int bs = s0 + i, gs = bd.slot0 + bs;
-          const int j = unit[gs];
-          const float al = alpha[gs];
-#pragma unroll
-          for (int gl = 0; gl < G; ++gl) {
-            const float sc = __half2float(__ushort_as_half((unsigned short)(sz[(size_t)(g_base + gl) * xd.nslots + bs] & 0xFFFFu)));
-#pragma unroll
-            for (int tt = 0; tt < TB; ++tt) mx[tt] = fmaxf(mx[tt], fabsf(al * sc * zrow[tt][j]));
-          }
-        }
-      }
-      float inv[TB], scl[TB];
-#pragma unroll
-      for (int tt = 0; tt < TB; ++tt) {
-        mx[tt] = warp_max(mx[tt]);
-        inv[tt] = mx[tt] > 0.f ? 32767.f / mx[tt] : 0.f;
-        scl[tt] = mx[tt] * (1.f / 32767.f);
-      }
-      // pass 2: quantise into shared memory, zero-point correction per group
-      float corr[G][TB];
-#pragma unroll
-      for (int gl = 0; gl < G; ++gl)
-#pragma unroll
-        for (int tt = 0; tt < TB; ++tt) corr[gl][tt] = 0.f;
-      for (int ri = 0; ri < nr; ++ri) {
-        const BucketDesc& bd = xd.bk[rg[ri].bi];
-        if (bd.bits == 16) continue;
-        const int U = rl_units(bd.bits), s0 = rg[ri].lo * U, ns = (rg[ri].hi - rg[ri].lo) * U;
-        const uint32_t* sz = reinterpret_cast<const uint32_t*>(p.img + bd.sz_off);
-        for (int i = lane; i < ns; i += 32) {
-          const int bs = s0 + i, gs = bd.slot0 + bs;
-          const int j = unit[gs];
-          const float al = alpha[gs];
-#pragma unroll
-          for (int gl = 0; gl < G; ++gl) {
-            const uint32_t szw = sz[(size_t)(g_base + gl) * xd.nslots + bs];
-            const float sc = __half2float(__ushort_as_half((unsigned short)(szw & 0xFFFFu)));
-            const float zp = __half2float(__ushort_as_half((unsigned short)(szw >> 16)));
-#pragma unroll
-            for (int tt = 0; tt < TB; ++tt) {
-              const int ci = __float2int_rn(al * sc * zrow[tt][j] * inv[tt]);
-              cq[(size_t)(gl * TB + tt) * p.s16 + rg[ri].ls0 + i] = (int16_t)ci;
-              corr[gl][tt] = fmaf((float)ci, zp, corr[gl][tt]);
-            }
-          }
-        }
-      }
-#pragma unroll
-      for (int gl = 0; gl < G; ++gl)
-#pragma unroll
-        for (int tt = 0; tt < TB; ++tt) corr[gl][tt] = warp_sum(corr[gl][tt]);
-      __syncwarp();
-      // main loop over the item's tiles
-      float accf[4][TB], acc16[4][TB];
-#pragma unroll
-      for (int w = 0; w < 4; ++w)
-#pragma unroll
-        for (int tt = 0; tt < TB; ++tt) accf[w][tt] = acc16[w][tt] = 0.f;
-      const int* cq32 = reinterpret_cast<const int*>(cq + (size_t)gl_lane * TB * p.s16);
-      const int tstride = p.s16 / 2;
-      for (int ri = 0; ri < nr; ++ri) {
-        const BucketDesc& bd = xd.bk[rg[ri].bi];
-        const int ntl = rg[ri].hi - rg[ri].lo;
-        const uint8_t* code = p.img + xd.code_base + (size_t)rb * xd.rb_stride + bd.code_off +
-                              (size_t)rg[ri].lo * rl_chunks(bd.bits) * kChunkBytes + lane * 16;
-        const int* cp = cq32 + rg[ri].ls0 / 2;
-        switch (bd.bits) {
-          case 1: rl_range<1, TB>(code, ntl, cp, tstride, accf); break;
-          case 2: rl_range<2, TB>(code, ntl, cp, tstride, accf); break;
-          case 3: rl_range<3, TB>(code, ntl, cp, tstride, accf); break;
-          case 4: rl_range<4, TB>(code, ntl, cp, tstride, accf); break;
-          case 6: rl_range<6, TB>(code, ntl, cp, tstride, accf); break;
-          case 8: rl_range<8, TB>(code, ntl, cp, tstride, accf); break;
-          default: {
-            const int gs0 = bd.slot0 + rg[ri].lo * 4;
-            rl_range16<TB>(code, ntl, unit + gs0, alpha + gs0, zrow, acc16);
-          }
-        }
-      }
-      // write partial sums of the lane's 4 rows
-      const int row = rb * kRows + 4 * lane;
-#pragma unroll
-      for (int tt = 0; tt < TB; ++tt) {
-        if (tt < tb) {
-          float cl = corr[0][tt];
-#pragma unroll
-          for (int gl = 1; gl < G; ++gl)
-            if (gl == gl_lane) cl = corr[gl][tt];
-          float o[4];
-#pragma unroll
-          for (int w = 0; w < 4; ++w) o[w] = fmaf(scl[tt], accf[w][tt] - cl, acc16[w][tt]);
-          red_add_v4(p.gu + ((size_t)pair[tt] * 2 + h) * p.I_pad + row, o[0], o[1], o[2], o[3]);
-        }
-      }
-      __syncwarp();
-    }
-  }
-}
-
-// ---------------------------------------------------------------------------
+//
 // K3: down factor.  h = SiLU(gate) * up for the block's rows (quantised to
 // int16 with one scale per token), then per unit j (one per lane):
 //   d_j = sum_g s_jg (sum_{i in g} q_ij h_i - zero_jg * sum_{i in g} h_i)
 //   s[t][j] += w_(t,e) * alpha_j * d_j
-// A block item is (routed expert, 8 UL tiles, up to 8 row blocks).
+// A block item is (routed expert, one UL tile per warp, a chunk of row blocks).
 // ---------------------------------------------------------------------------
 
 // scale/zero of group g of the lane's unit: sz[(g - szg0) * szstride + szcol]
@@ -884,128 +722,6 @@ __device__ __forceinline__ void ul_tile(const Fwd& p, const uint8_t* code, int r
         float d = (float)tot;
         if (starts) d = fmaf(-zp, (float)Hg[tt * 64 + hgi], d);
         accf[tt] = fmaf(sc, d, accf[tt]);
-      }
-    }
-  }
-}
-
-template <int G, int TB>
-__global__ void __launch_bounds__(kThreads) k_down(Fwd p) {
-  pdl_trigger();
-  pdl_wait();
-  extern __shared__ int4 smem_k3[];
-  const int rbc = p.rbc;
-  const int nrows_max = rbc * kRows;
-  float* hf = reinterpret_cast<float*>(smem_k3);                       // [TB][nrows_max]
-  int16_t* hq = reinterpret_cast<int16_t*>(hf + TB * nrows_max);       // [TB][nrows_max]
-  int* Hg = reinterpret_cast<int*>(hq + TB * nrows_max);               // [TB][64]
-  float* red = reinterpret_cast<float*>(Hg + TB * 64);                 // [kWarps][TB]
-  float* shs = red + kWarps * TB;                                      // [TB] scales
-  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-  const int A = p.active[0];
-  const int ntg = (p.ul_max_tiles + kK3Tiles - 1) / kK3Tiles;
-  const int nrc = (p.NRB + rbc - 1) / rbc;
-  const int total = A * ntg * nrc;
-  const int gshift = 31 - __clz(p.group);
-  for (int item = blockIdx.x; item < total; item += gridDim.x) {
-    const int a = item / (ntg * nrc);
-    const int r = item - a * ntg * nrc;
-    const int tg = r / nrc, rc = r - tg * nrc;
-    const int e = p.active[1 + a];
-    const ExpertDesc& xd = p.desc[2 * p.E + e];
-    if (tg * kK3Tiles >= xd.ntiles) continue;
-    const int rb0 = rc * rbc, rb1 = min(p.NRB, rb0 + rbc);
-    const int row0 = rb0 * kRows, nrows = (rb1 - rb0) * kRows;
-    const int ntok = p.expert_count[e], pst = p.expert_start[e];
-    // this warp's tile and bucket
-    const int tile = tg * kK3Tiles + wid;
-    int bi = -1;
-    if (tile < xd.ntiles)
-      for (int q = 0; q < xd.nbk; ++q)
-        if (tile >= xd.bk[q].tile0 && tile < xd.bk[q].tile0 + xd.bk[q].ntiles) bi = q;
-    for (int tb0 = 0; tb0 < ntok; tb0 += TB) {
-      const int tb = min(TB, ntok - tb0);
-      __syncthreads();
-      // h = SiLU(gate) * up for the rows of this block
-      float mx[TB];
-#pragma unroll
-      for (int tt = 0; tt < TB; ++tt) mx[tt] = 0.f;
-      for (int i = threadIdx.x; i < nrows; i += blockDim.x) {
-#pragma unroll
-        for (int tt = 0; tt < TB; ++tt) {
-          float hv = 0.f;
-          if (tt < tb) {
-            const int pr = p.pair_list[pst + tb0 + tt];
-            const float g = p.gu[((size_t)pr * 2) * p.I_pad + row0 + i];
-            const float u = p.gu[((size_t)pr * 2 + 1) * p.I_pad + row0 + i];
-            hv = g / (1.f + __expf(-g)) * u;
-          }
-          hf[tt * nrows_max + i] = hv;
-          mx[tt] = fmaxf(mx[tt], fabsf(hv));
-        }
-      }
-#pragma unroll
-      for (int tt = 0; tt < TB; ++tt) {
-        const float m = warp_max(mx[tt]);
-        if (lane == 0) red[wid * TB + tt] = m;
-      }
-      __syncthreads();
-      if (threadIdx.x < TB) {
-        float m = 0.f;
-        for (int w = 0; w < kWarps; ++w) m = fmaxf(m, red[w * TB + threadIdx.x]);
-        shs[threadIdx.x] = m;
-      }
-      __syncthreads();
-      for (int i = threadIdx.x; i < nrows; i += blockDim.x) {
-#pragma unroll
-        for (int tt = 0; tt < TB; ++tt) {
-          const float m = shs[tt];
-          const float inv = m > 0.f ? 32767.f / m : 0.f;
-          hq[tt * nrows_max + i] = (int16_t)__float2int_rn(hf[tt * nrows_max + i] * inv);
-        }
-      }
-      __syncthreads();
-      // group sums of the quantised h (groups lie inside the block's rows)
-      const int ngr = nrows >> gshift;
-      for (int q = wid; q < TB * ngr; q += kWarps) {
-        const int tt = q / ngr, g = q - tt * ngr;
-        int sacc = 0;
-        for (int i = lane; i < p.group; i += 32) sacc += hq[tt * nrows_max + (g << gshift) + i];
-#pragma unroll
-        for (int o = 16; o; o >>= 1) sacc += __shfl_xor_sync(0xFFFFFFFFu, sacc, o);
-        if (lane == 0) Hg[tt * 64 + g] = sacc;
-      }
-      __syncthreads();
-      if (bi < 0) continue;
-      const BucketDesc& bd = xd.bk[bi];
-      const int bs = (tile - bd.tile0) * 32 + lane;     // bucket-local slot
-      const int gs = bd.slot0 + bs;
-      const int j = reinterpret_cast<const int32_t*>(p.img + xd.unit_off)[gs];
-      const float al = reinterpret_cast<const float*>(p.img + xd.alpha_off)[gs];
-      const uint8_t* code = p.img + xd.code_base + bd.code_off +
-                            ((size_t)(tile - bd.tile0) * p.NRB + rb0) * ul_chunks(bd.bits) * kChunkBytes + lane * 16;
-      const uint32_t* sz = reinterpret_cast<const uint32_t*>(p.img + bd.sz_off);
-      float accf[TB];
-#pragma unroll
-      for (int tt = 0; tt < TB; ++tt) accf[tt] = 0.f;
-      switch (bd.bits) {
-        case 1: ul_tile<1, G, TB>(p, code, rb0, rb1, hq, nrows_max, Hg, sz, xd.nslots, 0, bs, accf); break;
-        case 2: ul_tile<2, G, TB>(p, code, rb0, rb1, hq, nrows_max, Hg, sz, xd.nslots, 0, bs, accf); break;
-        case 3: ul_tile<3, G, TB>(p, code, rb0, rb1, hq, nrows_max, Hg, sz, xd.nslots, 0, bs, accf); break;
-        case 4: ul_tile<4, G, TB>(p, code, rb0, rb1, hq, nrows_max, Hg, sz, xd.nslots, 0, bs, accf); break;
-        case 6: ul_tile<6, G, TB>(p, code, rb0, rb1, hq, nrows_max, Hg, sz, xd.nslots, 0, bs, accf); break;
-        case 8: ul_tile<8, G, TB>(p, code, rb0, rb1, hq, nrows_max, Hg, sz, xd.nslots, 0, bs, accf); break;
-        default: ul_tile<16, G, TB>(p, code, rb0, rb1, hq, nrows_max, Hg, sz, xd.nslots, 0, bs, accf); break;
-      }
-      if (al != 0.f) {
-#pragma unroll
-        for (int tt = 0; tt < TB; ++tt) {
-          if (tt < tb) {
-            const int pr = p.pair_list[pst + tb0 + tt];
-            const float scale = shs[tt] * (1.f / 32767.f);
-            atomicAdd(p.s + (size_t)(pr / p.k) * p.n_pad + j, p.pair_weight[pr] * al * scale * accf[tt]);
-          }
-        }
       }
     }
   }
@@ -1544,19 +1260,6 @@ int launch_gemv_any(bool proj, const Fwd& p, int sms, cudaStream_t st, bool pdl)
   return launch_gemv<8>(proj, p, sms, st, pdl);
 }
 
-template <int G, int TB>
-int launch_k2k3(const Fwd& p, int sms, cudaStream_t st, bool pdl, const std::function<int()>& between) {
-  int rc;
-  const size_t sm2 = (size_t)kWarps * G * TB * p.s16 * 2;
-  if ((rc = set_smem(k_gateup<G, TB>, sm2))) return rc;
-  if ((rc = launch(k_gateup<G, TB>, dim3(sms * 2), dim3(kThreads), sm2, st, pdl, p))) return rc;
-  if (between && (rc = between())) return rc;
-  const size_t nrm = (size_t)p.rbc * kRows;
-  const size_t sm3 = TB * nrm * 4 + TB * nrm * 2 + TB * 64 * 4 + kWarps * TB * 4 + TB * 4;
-  if ((rc = set_smem(k_down<G, TB>, sm3))) return rc;
-  return launch(k_down<G, TB>, dim3(sms * 2), dim3(kThreads), sm3, st, pdl, p);
-}
-
 template <int TB>
 int launch_gemv_bulk_tb(bool proj, const Fwd& p, int sms, cudaStream_t st, bool pdl) {
   const int ld = proj ? p.D_pad : p.n_pad;
@@ -1629,11 +1332,6 @@ int launch_k2k3_dec(const Fwd& p, int A_max, int sms, cudaStream_t st, bool pdl,
   const int nrc = (p.NRB + p.rbc - 1) / p.rbc;
   if ((rc = set_smem(k_down_dec<G, TB>, sm3))) return rc;
   return launch(k_down_dec<G, TB>, dim3(std::max(1, A_max * ntg * nrc)), dim3(kK3DecWarps * 32), sm3, st, pdl, p);
-}
-
-template <int G>
-int launch_k2k3_tb(const Fwd& p, int sms, cudaStream_t st, bool pdl, const std::function<int()>& between) {
-  return p.T == 1 ? launch_k2k3<G, 1>(p, sms, st, pdl, between) : launch_k2k3<G, 4>(p, sms, st, pdl, between);
 }
 
 bool aligned(const void* ptr, size_t a) { return ((uintptr_t)ptr % a) == 0; }
