@@ -48,25 +48,38 @@ __device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t* ptr) {
   return v;
 }
 
-// All blocks of the grid arrive on `cnt` (zero at kernel start) and wait
-// until every block has arrived.  The block's writes before the barrier are
-// ordered before its arrival (bar.sync, then a release reduction), and the
-// waiting side acquires; data written before the barrier is read with
-// L2-coherent loads after it.
-__device__ __forceinline__ void grid_barrier(uint32_t* cnt, uint32_t nblocks, int* status) {
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(cnt) : "memory");
+// Grid barrier on a counter that is zero at kernel start.  Arrival: thread 0
+// of a block, after the block's (or a warp group's) bar.sync has ordered the
+// writes to publish, adds 1 with release semantics.  Wait: lane 0 of warps
+// 0..3 poll with acquire loads, starting about 100 ns apart so that the
+// polls interleave, until one of them sees every block; then the whole block
+// synchronises.  Data written before the barrier is read with L2-coherent
+// loads after it.
+__device__ __forceinline__ void grid_arrive(uint32_t* cnt) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(cnt) : "memory");
+}
+__device__ __forceinline__ void grid_wait(uint32_t* cnt, uint32_t nblocks, int* status, volatile int* seen) {
+  const int wid = threadIdx.x >> 5;
+  if ((threadIdx.x & 31) == 0 && wid < 4) {
+    if (wid) __nanosleep(100 * wid);
     const long long t0 = clock64();
-    while (ld_acquire_u32(cnt) < nblocks) {
+    while (!*seen) {
+      if (ld_acquire_u32(cnt) >= nblocks) {
+        *seen = 1;
+        break;
+      }
       if (clock64() - t0 > kSpin) {
-        atomicCAS(status, 0, BITSMOE_ERR_TIMEOUT);
+        if (wid == 0) atomicCAS(status, 0, BITSMOE_ERR_TIMEOUT);
         break;
       }
     }
-    __threadfence();
   }
   __syncthreads();
+}
+__device__ __forceinline__ void grid_barrier(uint32_t* cnt, uint32_t nblocks, int* status, volatile int* seen) {
+  __syncthreads();
+  if (threadIdx.x == 0) grid_arrive(cnt);
+  grid_wait(cnt, nblocks, status, seen);
 }
 
 __device__ __forceinline__ void prefetch_run(const uint8_t* p, uint64_t bytes) {
@@ -493,6 +506,7 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
   int* sel_e = reinterpret_cast<int*>(keys + p.E);                     // [k] expert of routing rank a
   float* sel_w = reinterpret_cast<float*>(sel_e + p.k);                // [k] its gate weight
   float* part = reinterpret_cast<float*>(fsm + f.off_part);           // [kFWarps][32] down partial sums
+  volatile int* seen = reinterpret_cast<volatile int*>(bar_d + kFWarps);   // [3] grid barriers passed
   const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
   const int nb = gridDim.x, blk = blockIdx.x;
   const uint32_t row_in = (uint32_t)p.D_pad * 2, row_out = (uint32_t)p.n_pad * 2;
@@ -518,6 +532,7 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
   };
   if (tid == 0) {
     for (int i = 0; i < kMaxBStages + 1 + 2 * kFWarps; ++i) mbar_init(bar_b + i);
+    seen[0] = seen[1] = seen[2] = 0;
     issue_b(0, nst_pre);
   } else if (tid == 32) {   // this block's share of the staging tables into L2
     const uint64_t per = (f.tab_bytes / nb + 15) / 16 * 16;
@@ -603,6 +618,9 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
         p.z[(size_t)h * p.n_pad + j] = acc;
       }
     }
+    // the block's z rows are written: arrive at barrier 1 without waiting for the control warps
+    asm volatile("bar.sync 3, %0;" ::"r"(kBW * 32) : "memory");
+    if (tid == 0) grid_arrive(f.cnt + 0);
   } else {
     // ---- routing of the token: k largest logits (ties to the lower index), softmax over the k
     const int ct = tid - kBW * 32;
@@ -661,30 +679,17 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
         const int i = blk + m * nb, a = i / f.ul_max_tiles, tile = i - a * f.ul_max_tiles;
         const DStage r = load_drec(f.dst + (size_t)sel_e[a] * f.ul_max_tiles + tile);
         if (m == s) drec[s] = r;
-        if (r.bits) prefetch_run(p.img + r.code, (uint64_t)p.NRB * ul_chunks((int)r.bits) * kChunkBytes);
+        else if (r.bits) prefetch_run(p.img + r.code, (uint64_t)p.NRB * ul_chunks((int)r.bits) * kChunkBytes);
       }
-    } else if (ct == 64 && e1 > e0) {
-      prefetch_run(reinterpret_cast<const uint8_t*>(p.basis_out) + (size_t)e0 * row_out, (uint64_t)(e1 - e0) * row_out);
     }
   }
-  __syncthreads();   // projection rows consumed, routing and first staging records in shared memory
+  grid_wait(f.cnt + 0, nb, p.status, seen + 0);
+  // The projection rows are consumed; their buffer receives the first down tiles
+  // (each staged by its slot's warp once that warp's gate/up items are done, so
+  // that the copies do not delay the latency-bound z gathers) and, once the
+  // first down tiles are done, this block's rows of Phi_dn.
   uint8_t* ers = r1;                       // [e1 - e0][n_pad] bf16
   uint8_t* dslots = r1 + f.off_d;          // [nslot_d][slot_d]
-  if (tid == 0) {
-    fence_proxy_async();   // generic reads of the rows above, then async writes
-    if (e1 > e0) {
-      mbar_expect_tx(bar_e, (uint32_t)(e1 - e0) * row_out);
-      bulk_run(ers, reinterpret_cast<const uint8_t*>(p.basis_out) + (size_t)e0 * row_out,
-               (uint32_t)(e1 - e0) * row_out, bar_e);
-    }
-  } else if (tid >= 32 && tid < 32 + f.nslot_d) {
-    const int s = tid - 32;
-    if (s < md && drec[s].bits) {
-      fence_proxy_async();
-      d_stage(p, f, drec[s], dslots + (size_t)s * f.slot_d, bar_d + s);
-    }
-  }
-  grid_barrier(f.cnt + 0, nb, p.status);
 
   // ---- C: gate/up items
   if (wid < f.nslot_c) {
@@ -715,7 +720,11 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
       ++nst;
     }
   }
-  grid_barrier(f.cnt + 1, nb, p.status);
+  if (lane == 0 && wid < f.nslot_d && wid < md && drec[wid].bits) {
+    fence_proxy_async();   // generic reads of the projection rows (before barrier 1), then async writes
+    d_stage(p, f, drec[wid], dslots + (size_t)wid * f.slot_d, bar_d + wid);
+  }
+  grid_barrier(f.cnt + 1, nb, p.status, seen + 1);
 
   // ---- D: down tiles, s += w * alpha * P_dn^T h.  Warp w works on slot w % nslot_d
   // over row blocks w / nslot_d, + nsub, ...; the slot's partial sums meet in shared memory.
@@ -727,6 +736,16 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
     float* hsc = reinterpret_cast<float*>(hqs + p.I_pad);
     int* hsum = reinterpret_cast<int*>(hsc + p.NRB);
     const int rounds = (md + f.nslot_d - 1) / f.nslot_d;
+    // this block's rows of Phi_dn: once the first down tiles have read h (or now, without down tiles)
+    auto issue_e = [&]() {
+      if (tid == 0 && e1 > e0) {
+        fence_proxy_async();
+        mbar_expect_tx(bar_e, (uint32_t)(e1 - e0) * row_out);
+        bulk_run(ers, reinterpret_cast<const uint8_t*>(p.basis_out) + (size_t)e0 * row_out,
+                 (uint32_t)(e1 - e0) * row_out, bar_e);
+      }
+    };
+    if (rounds == 0) issue_e();
     int staged = 0, cur_a = -1;
     for (int rd = 0; rd < rounds; ++rd) {
       const int m = sl + rd * f.nslot_d;
@@ -759,6 +778,7 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
       }
       part[wid * 32 + lane] = acc;
       __syncthreads();
+      if (rd == 0) issue_e();
       if (r.bits && sub == 0) {
         float t = 0.f;
         for (int q = 0; q < nsub; ++q) t += part[(sl + q * f.nslot_d) * 32 + lane];
@@ -769,7 +789,7 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
       __syncthreads();
     }
   }
-  grid_barrier(f.cnt + 2, nb, p.status);
+  grid_barrier(f.cnt + 2, nb, p.status, seen + 2);
   pdl_trigger();   // every block is past its last wait on other blocks
 
   // ---- E: y = Phi_dn s for rows [e0, e1)
