@@ -337,7 +337,7 @@ def run_stack(args, spec, T, torch, bm, dev, rank, world, local):
         "e2e": {"value": world * ne * T / e2e_s, "unit": "tokens/s", "steps": ne,
                 "h2d_bytes_per_step": T * spec.D * 4, "d2h_bytes_per_step": T * spec.D * 4},
         "clocks": clocks,
-        "gpu_launches": args.steps * spec.layers * (bm.bitsmoe_forward_launches(layers[0], T, k) + 1),
+        "gpu_launches": args.steps * spec.layers * bm.bitsmoe_block_forward_launches(layers[0], T, k),
     }
     if rank == 0:
         print(json.dumps(line), flush=True)

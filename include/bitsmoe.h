@@ -147,6 +147,11 @@ size_t bitsmoe_workspace_bytes(const bitsmoe_layer* layer, int T, int top_k);
  * arguments. */
 int bitsmoe_forward_launches(const bitsmoe_layer* layer, int T, int top_k);
 
+/* Kernels one bitsmoe_moe_block_forward call launches: 1 when the fused
+ * single-token kernel runs (it computes the pre-norm and router too),
+ * otherwise the norm/router kernel plus bitsmoe_forward_launches. */
+int bitsmoe_block_forward_launches(const bitsmoe_layer* layer, int T, int top_k);
+
 /* The quantised MoE-layer forward, asynchronous on `stream`:
  *   x       device, T x D bf16 bit patterns (row-major), 16-byte aligned
  *   logits  device, T x E fp32 router logits (row-major), 16-byte aligned
@@ -193,7 +198,11 @@ int bitsmoe_rmsnorm_router(const float* h, const void* w_router, float eps, int 
 /* One pre-norm MoE block in place: h += MoE(x, logits) with x, logits from
  * bitsmoe_rmsnorm_router(h, w_router, eps) and MoE the quantised MoE-layer
  * forward of `layer`.  Workspace and errors as bitsmoe_moe_forward (the
- * normalised activations and logits live in the workspace).  Asynchronous. */
+ * normalised activations and logits live in the workspace).  Asynchronous.
+ * When the forward runs as the fused single-token kernel, that kernel also
+ * computes the norm and the router logits (in the same arithmetic order as
+ * bitsmoe_rmsnorm_router, so x and logits are the same bits); otherwise the
+ * norm/router kernel runs first. */
 int bitsmoe_moe_block_forward(float* h, const void* w_router, float eps, int T, int top_k,
                               const bitsmoe_layer* layer, void* ws, size_t ws_bytes, void* stream);
 

@@ -56,6 +56,7 @@ SIGNATURES = {
     "bitsmoe_profile_forward": (_I, [_P, _P, _I, _I, _P, _P, _P, _SZ, _P, ctypes.POINTER(ctypes.c_float)]),
     "bitsmoe_workspace_bytes": (_SZ, [_P, _I, _I]),
     "bitsmoe_forward_launches": (_I, [_P, _I, _I]),
+    "bitsmoe_block_forward_launches": (_I, [_P, _I, _I]),
     "bitsmoe_moe_forward": (_I, [_P, _P, _I, _I, _P, _P, _P, _SZ, _P]),
     "bitsmoe_moe_forward_host": (_I, [_P, _P, _I, _I, _P, _P, _P, _SZ, _P]),
     "bitsmoe_moe_forward_noalloc": (_I, [_P, _P, _I, _I, _P, _P, _P]),
@@ -233,6 +234,14 @@ def bitsmoe_forward_launches(layer: Layer, T: int, top_k: int) -> int:
     n = int(_lib().bitsmoe_forward_launches(layer.handle, T, top_k))
     if n < 0:
         raise BitsMoEError(n, "bitsmoe_forward_launches")
+    return n
+
+
+def bitsmoe_block_forward_launches(layer: Layer, T: int, top_k: int) -> int:
+    """Kernels one block forward launches (1: the fused kernel with its pre-norm; else norm/router + chain)."""
+    n = int(_lib().bitsmoe_block_forward_launches(layer.handle, T, top_k))
+    if n < 0:
+        raise BitsMoEError(n, "bitsmoe_block_forward_launches")
     return n
 
 

@@ -80,6 +80,10 @@ struct FusedArgs {
   const CStage* cst; // [2][E][nseg]
   const DStage* dst; // [E][ul_max_tiles] (directly after cst)
   uint64_t tab_bytes;  // bytes of both tables
+  const float* hn;     // norm mode (pre-norm block): hidden state h [D] to normalise; y = h accumulates
+  const uint16_t* wr;  // norm mode: router matrix [E][D] bf16
+  float eps;           // norm mode: RMSNorm epsilon
+  int norm;            // 1: compute x = bf16(RMSNorm(h)) and the router logits in the kernel
   int b_per, b_stage, b_nst, e_per;     // basis rows per block, rows per stage, stages; output rows per block
   int nslot_c, slot_c, nslot_d, slot_d; // gate/up and down staging slots (count, bytes)
   int off_route, off_xs, off_r1, off_d, off_rc, off_cq, off_rec, off_part, smem;

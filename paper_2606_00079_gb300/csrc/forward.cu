@@ -1370,8 +1370,11 @@ int num_sms_current(int* sms) {
 }
 
 
+// norm != nullptr: a pre-norm block (y = h accumulates); x and logits are the workspace buffers that
+// the norm/router step fills, either as its own kernel or inside the one-token fused kernel.
 int forward_impl(const void* x, const float* logits, int T, int top_k, const bitsmoe_layer* L, float* y,
-                 void* ws, size_t ws_bytes, cudaStream_t st, cudaEvent_t* ev = nullptr, bool accum = false) {
+                 void* ws, size_t ws_bytes, cudaStream_t st, cudaEvent_t* ev = nullptr, bool accum = false,
+                 const NormArgs* norm = nullptr) {
   const ImageHeader& hd = L->hd();
   const bool pdl = ev == nullptr;   // profiling runs the phases back to back without overlap
   const WsLayout w = ws_layout(hd, T, top_k);
@@ -1429,6 +1432,12 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
     fa.cst = L->d_cst;
     fa.dst = L->d_dst;
     fa.tab_bytes = L->stage_bytes;
+    if (norm) {
+      fa.norm = 1;
+      fa.hn = norm->h;
+      fa.wr = norm->w;
+      fa.eps = norm->eps;
+    }
     if ((rc = mark(0))) return rc;
     const cudaError_t e = launch_fused(p, fa, sms, st, pdl);
     if (e != cudaSuccess) return cuda_fail(e);
@@ -1436,6 +1445,7 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
       if ((rc = mark(i))) return rc;
     return BITSMOE_OK;
   }
+  if (norm && (rc = launch_norm_router(*norm, sms, st))) return rc;
   if (p.decode) {
     const int A_max = std::min(hd.E, p.P);
     const size_t rsm = (size_t)route_words(p.T, hd.E, p.P) * 4 + 16;
@@ -1684,6 +1694,11 @@ int bitsmoe_forward_launches(const bitsmoe_layer* L, int T, int top_k) {
   return 5;
 }
 
+int bitsmoe_block_forward_launches(const bitsmoe_layer* L, int T, int top_k) {
+  const int n = bitsmoe_forward_launches(L, T, top_k);
+  return n > 1 ? n + 1 : n;
+}
+
 size_t bitsmoe_workspace_bytes(const bitsmoe_layer* L, int T, int top_k) {
   if (!L || T < 0 || top_k < 1 || top_k > std::min(L->hd().E, 32)) return 0;
   return ws_layout(L->hd(), T, top_k).total;
@@ -1791,9 +1806,8 @@ int bitsmoe_moe_block_forward(float* h, const void* w_router, float eps, int T, 
   uint8_t* wb = static_cast<uint8_t*>(ws);
   NormArgs a{h, static_cast<const uint16_t*>(w_router), eps, T, hd.D, hd.E, hd.D_pad,
              reinterpret_cast<uint16_t*>(wb + w.x_stage), reinterpret_cast<float*>(wb + w.logits_stage)};
-  if ((rc = launch_norm_router(a, L->num_sms, st))) return rc;
   return forward_impl(wb + w.x_stage, reinterpret_cast<const float*>(wb + w.logits_stage), T, top_k, L, h, ws,
-                      ws_bytes, st, nullptr, true);
+                      ws_bytes, st, nullptr, true, &a);
 }
 
 int bitsmoe_last_device_status(void* ws, void* stream) {

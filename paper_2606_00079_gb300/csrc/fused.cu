@@ -76,6 +76,25 @@ __device__ __forceinline__ void grid_wait(uint32_t* cnt, uint32_t nblocks, int* 
   }
   __syncthreads();
 }
+// The same wait for the control warps only (lane 0 of each polls; then they sync on barrier 2).
+__device__ __forceinline__ void grid_wait_ctl(uint32_t* cnt, uint32_t nblocks, int* status, volatile int* seen,
+                                              int cw, int nthreads) {
+  if ((threadIdx.x & 31) == 0) {
+    if (cw) __nanosleep(100 * cw);
+    const long long t0 = clock64();
+    while (!*seen) {
+      if (ld_acquire_u32(cnt) >= nblocks) {
+        *seen = 1;
+        break;
+      }
+      if (clock64() - t0 > kSpin) {
+        if (cw == 0) atomicCAS(status, 0, BITSMOE_ERR_TIMEOUT);
+        break;
+      }
+    }
+  }
+  asm volatile("bar.sync 2, %0;" ::"r"(nthreads) : "memory");
+}
 __device__ __forceinline__ void grid_barrier(uint32_t* cnt, uint32_t nblocks, int* status, volatile int* seen) {
   __syncthreads();
   if (threadIdx.x == 0) grid_arrive(cnt);
@@ -532,8 +551,11 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
   };
   if (tid == 0) {
     for (int i = 0; i < kMaxBStages + 1 + 2 * kFWarps; ++i) mbar_init(bar_b + i);
-    seen[0] = seen[1] = seen[2] = 0;
+    seen[0] = seen[1] = seen[2] = seen[3] = 0;
     issue_b(0, nst_pre);
+  } else if (tid == 64 && f.norm) {   // this block's router rows (norm mode) into L2
+    const int epb = (p.E + nb - 1) / nb, r0 = min(p.E, blk * epb), r1e = min(p.E, r0 + epb);
+    if (r1e > r0) prefetch_run(reinterpret_cast<const uint8_t*>(f.wr + (size_t)r0 * p.D), (uint64_t)(r1e - r0) * p.D * 2);
   } else if (tid == 32) {   // this block's share of the staging tables into L2
     const uint64_t per = (f.tab_bytes / nb + 15) / 16 * 16;
     const uint64_t o = (uint64_t)blk * per;
@@ -562,13 +584,41 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
     }
     __syncthreads();   // part[] is reused below
   }
+  uint16_t* xs = reinterpret_cast<uint16_t*>(fsm + f.off_xs);
+  if (f.norm) {
+    // pre-norm of the block: x = bf16(h / sqrt(mean(h^2) + eps)) (unit weight), in the same
+    // arithmetic order as the separate norm/router kernel: 256 strided partial sums, warp sums,
+    // eight warp totals in order
+    float* red = part;
+    if (tid < 256) {
+      float ss = 0.f;
+      for (int d = tid; d < p.D; d += 256) {
+        const float v = f.hn[d];
+        ss = fmaf(v, v, ss);
+      }
+      ss = warp_sum(ss);
+      if (lane == 0) red[wid] = ss;
+    }
+    __syncthreads();
+    float sum = 0.f;
+    for (int w = 0; w < 8; ++w) sum += red[w];
+    const float iv = rsqrtf(sum / (float)p.D + f.eps);
+    for (int d = tid; d < p.D_pad; d += kFThreads) {
+      uint32_t u32 = 0;
+      if (d < p.D) {   // round to bf16, nearest even
+        u32 = __float_as_uint(f.hn[d] * iv);
+        u32 = (u32 + 0x7FFFu + ((u32 >> 16) & 1u)) & 0xFFFF0000u;
+      }
+      xs[d] = (uint16_t)(u32 >> 16);
+    }
+    __syncthreads();
+  }
 
   const int ndi = p.k * f.ul_max_tiles;   // down items of all blocks (some past an expert's tiles)
   const int md = ndi > blk ? (ndi - blk + nb - 1) / nb : 0;   // this block's: i = blk + m * nb
   if (wid < kBW) {
-    // ---- x into shared memory, zero gate/up and s
-    uint16_t* xs = reinterpret_cast<uint16_t*>(fsm + f.off_xs);
-    for (int i = tid; i < p.D_pad / 8; i += kBW * 32) {
+    // ---- x into shared memory (unless the block normalised h itself), zero gate/up and s
+    for (int i = tid; i < (f.norm ? 0 : p.D_pad / 8); i += kBW * 32) {
       uint4 v = make_uint4(0, 0, 0, 0);
       if (8 * i + 8 <= p.D) {
         v = *reinterpret_cast<const uint4*>(p.x + 8 * i);
@@ -622,9 +672,43 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
     asm volatile("bar.sync 3, %0;" ::"r"(kBW * 32) : "memory");
     if (tid == 0) grid_arrive(f.cnt + 0);
   } else {
-    // ---- routing of the token: k largest logits (ties to the lower index), softmax over the k
     const int ct = tid - kBW * 32;
-    for (int i = ct; i < p.E; i += kCT) keys[i] = order_key(p.logits[i]);
+    if (f.norm) {
+      // this block's router logits (rows blk * epb ..), one control warp per row, the lane's
+      // 16-byte chunks in the same order as the separate norm/router kernel; then every
+      // block's logits are published through grid counter 4
+      const int epb = (p.E + nb - 1) / nb, cw = ct >> 5, nch = p.D >> 3;
+      for (int j = cw; j < epb; j += kCT / 32) {
+        const int e = blk * epb + j;
+        if (e >= p.E) break;
+        const uint4* rp = reinterpret_cast<const uint4*>(f.wr + (size_t)e * p.D);
+        float acc = 0.f;
+        for (int c0 = 0; c0 < nch; c0 += 256) {
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const int c = c0 + u * 32 + lane;
+            if (c < nch) {
+              const uint4 v = __ldg(rp + c), xv = *reinterpret_cast<const uint4*>(xs + c * 8);
+              acc = fmaf(bf16lo(v.x), bf16lo(xv.x), acc);
+              acc = fmaf(bf16hi(v.x), bf16hi(xv.x), acc);
+              acc = fmaf(bf16lo(v.y), bf16lo(xv.y), acc);
+              acc = fmaf(bf16hi(v.y), bf16hi(xv.y), acc);
+              acc = fmaf(bf16lo(v.z), bf16lo(xv.z), acc);
+              acc = fmaf(bf16hi(v.z), bf16hi(xv.z), acc);
+              acc = fmaf(bf16lo(v.w), bf16lo(xv.w), acc);
+              acc = fmaf(bf16hi(v.w), bf16hi(xv.w), acc);
+            }
+          }
+        }
+        acc = warp_sum(acc);
+        if (lane == 0) const_cast<float*>(p.logits)[e] = acc;
+      }
+      asm volatile("bar.sync 2, %0;" ::"r"(kCT) : "memory");
+      if (ct == 0) grid_arrive(f.cnt + 4);
+      grid_wait_ctl(f.cnt + 4, nb, p.status, seen + 3, cw, kCT);
+    }
+    // ---- routing of the token: k largest logits (ties to the lower index), softmax over the k
+    for (int i = ct; i < p.E; i += kCT) keys[i] = order_key(__ldcg(p.logits + i));
     asm volatile("bar.sync 2, %0;" ::"r"(kCT) : "memory");
     for (int i = ct; i < p.E; i += kCT) {
       const uint32_t key = keys[i];
@@ -830,6 +914,7 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
       f.cnt[0] = 0u;
       f.cnt[1] = 0u;
       f.cnt[2] = 0u;
+      f.cnt[4] = 0u;
       __threadfence();
       f.cnt[3] = 0u;
     }

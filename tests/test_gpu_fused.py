@@ -175,3 +175,39 @@ def test_fused_plan_taken_for_qw3_dims_not_for_d4096(env):
     big = synth.scaled_spec(synth.WORKLOADS["mixtral"], E=2, I=128, top_k=1)
     Lb = bm.bitsmoe_pack(synth.make_layer(big, seed=1), device=0)
     assert bm.bitsmoe_forward_launches(Lb, 1, 1) == 5
+
+
+@pytest.mark.parametrize("E,top_k", [(4, 2), (200, 8)])
+def test_block_forward_fused_norm(env, E, top_k):
+    """A one-token pre-norm block runs as the single fused kernel, which also
+    computes the RMSNorm and the router logits (E = 200 > blocks: two router
+    rows on some blocks).  Its update must match the two-step path
+    (norm/router kernel, then the forward) up to the order of the float
+    atomics, and the oracle's MoE on the same x and logits."""
+    torch, bm = env
+    spec = small(E=E, top_k=top_k, n=72)
+    layer = synth.make_layer(spec, seed=5)
+    L = bm.bitsmoe_pack(layer, device=0)
+    assert bm.bitsmoe_block_forward_launches(L, 1, top_k) == 1
+    assert bm.bitsmoe_block_forward_launches(L, 2, top_k) == bm.bitsmoe_forward_launches(L, 2, top_k) + 1
+    wr = torch.from_numpy(synth.make_router_weight(spec, seed=5).view(np.int16)).cuda()
+    h0 = torch.from_numpy(synth.make_hidden(spec, 1, seed=5)).cuda() * 3.0
+    eps, st = 1e-6, torch.cuda.current_stream().cuda_stream
+    ws = bm.Workspace(L, 1, top_k)
+    x = torch.empty((1, spec.D), dtype=torch.int16, device="cuda")
+    lg = torch.empty((1, spec.E), dtype=torch.float32, device="cuda")
+    bm.bitsmoe_rmsnorm_router(h0.data_ptr(), wr.data_ptr(), eps, 1, spec.D, spec.E, x.data_ptr(), lg.data_ptr(), st)
+    y2 = bm.moe_forward(L, x, lg, top_k, ws=ws)
+    torch.cuda.synchronize()
+    for rep in range(3):   # the same workspace, repeatedly
+        h = h0.clone()
+        bm.bitsmoe_moe_block_forward(h.data_ptr(), wr.data_ptr(), eps, 1, top_k, L, ws.ptr, ws.nbytes, st)
+        torch.cuda.synchronize()
+        assert bm.bitsmoe_last_device_status(ws.ptr) == 0
+        two_step = (h0 + y2).cpu().numpy().astype(np.float64)   # the same fp32 add as the kernel's
+        ymax, hmax = float(y2.abs().max()), float(h0.abs().max())
+        assert np.max(np.abs(h.cpu().numpy() - two_step)) <= 1e-5 * ymax + 2.4e-7 * hmax
+        upd = (h - h0).cpu().numpy().astype(np.float64)
+    xo = x.cpu().numpy().view(np.uint16)
+    ref = oracle.moe_forward_factored(layer, xo, lg.cpu().numpy().astype(np.float64), top_k)
+    assert rel_err(upd, ref) <= TOL
