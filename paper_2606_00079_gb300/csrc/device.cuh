@@ -240,6 +240,7 @@ __device__ __forceinline__ float warp_max(float v) {
 __device__ __forceinline__ uint32_t order_key(float f) {
   const uint32_t u = __float_as_uint(f);
   if ((u & 0x7FFFFFFFu) > 0x7F800000u) return 0u;
+  if (u == 0x80000000u) return 0x80000000u;   // -0 and +0 are equal logits: they tie
   return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 

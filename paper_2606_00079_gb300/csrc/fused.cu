@@ -512,6 +512,47 @@ __device__ void d_stage(const Fwd& p, const FusedArgs& f, const DStage& r, uint8
 constexpr int kBW = 12;
 constexpr int kCT = (kFWarps - kBW) * 32;   // control threads
 
+// Routing of the token by the kCT control threads: the k largest logits (ties to the
+// lower index) into sel_e, their softmax into sel_w.  Out of line so that one copy of
+// the code exists: the kernel runs it once on dummy keys (logits == nullptr) while it
+// waits for the previous kernel, which brings the code into the instruction cache.
+__device__ __noinline__ void route_token(const float* logits, int E, int k, uint32_t* keys, int* sel_e,
+                                         float* sel_w, int ct) {
+  for (int i = ct; i < E; i += kCT) keys[i] = logits ? order_key(__ldcg(logits + i)) : 0u;
+  asm volatile("bar.sync 2, %0;" ::"r"(kCT) : "memory");
+  for (int i = ct; i < E; i += kCT) {
+    const uint32_t key = keys[i];
+    int rank = 0;
+    int f2 = 0;
+    for (; f2 + 4 <= E; f2 += 4) {
+      const uint4 o = *reinterpret_cast<const uint4*>(keys + f2);
+      rank += (o.x > key) | ((o.x == key) & (f2 < i));
+      rank += (o.y > key) | ((o.y == key) & (f2 + 1 < i));
+      rank += (o.z > key) | ((o.z == key) & (f2 + 2 < i));
+      rank += (o.w > key) | ((o.w == key) & (f2 + 3 < i));
+    }
+    for (; f2 < E; ++f2) {
+      const uint32_t o = keys[f2];
+      rank += (o > key) | ((o == key) & (f2 < i));
+    }
+    if (rank < k) {
+      sel_e[rank] = i;
+      sel_w[rank] = key ? __uint_as_float((key & 0x80000000u) ? (key & 0x7FFFFFFFu) : ~key)
+                        : __int_as_float(0x7FC00000);   // key 0: a NaN logit
+    }
+  }
+  asm volatile("bar.sync 2, %0;" ::"r"(kCT) : "memory");
+  if (ct < 32) {
+    const float m = sel_w[0];
+    const float ev = ct < k ? expf(sel_w[ct] - m) : 0.f;
+    float sum = ev;
+#pragma unroll
+    for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
+    __syncwarp();   // every lane has read sel_w[0]
+    if (ct < k) sel_w[ct] = ev * (1.f / sum);
+  }
+}
+
 template <int G>
 __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
   extern __shared__ __align__(128) uint8_t fsm[];
@@ -562,6 +603,7 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
     if (o < f.tab_bytes)
       prefetch_run(reinterpret_cast<const uint8_t*>(f.cst) + o, min(per, f.tab_bytes - o));
   }
+  if (wid >= kBW) route_token(nullptr, p.E, p.k, keys, sel_e, sel_w, tid - kBW * 32);   // code warm-up
   __syncthreads();
   pdl_wait();   // x, logits, y and the workspace belong to earlier kernels until here
 
@@ -707,40 +749,8 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
       if (ct == 0) grid_arrive(f.cnt + 4);
       grid_wait_ctl(f.cnt + 4, nb, p.status, seen + 3, cw, kCT);
     }
-    // ---- routing of the token: k largest logits (ties to the lower index), softmax over the k
-    for (int i = ct; i < p.E; i += kCT) keys[i] = order_key(__ldcg(p.logits + i));
-    asm volatile("bar.sync 2, %0;" ::"r"(kCT) : "memory");
-    for (int i = ct; i < p.E; i += kCT) {
-      const uint32_t key = keys[i];
-      int rank = 0;
-      int f2 = 0;
-      for (; f2 + 4 <= p.E; f2 += 4) {
-        const uint4 o = *reinterpret_cast<const uint4*>(keys + f2);
-        rank += (o.x > key) | ((o.x == key) & (f2 < i));
-        rank += (o.y > key) | ((o.y == key) & (f2 + 1 < i));
-        rank += (o.z > key) | ((o.z == key) & (f2 + 2 < i));
-        rank += (o.w > key) | ((o.w == key) & (f2 + 3 < i));
-      }
-      for (; f2 < p.E; ++f2) {
-        const uint32_t o = keys[f2];
-        rank += (o > key) | ((o == key) & (f2 < i));
-      }
-      if (rank < p.k) {
-        sel_e[rank] = i;
-        sel_w[rank] = key ? __uint_as_float((key & 0x80000000u) ? (key & 0x7FFFFFFFu) : ~key)
-                          : __int_as_float(0x7FC00000);   // key 0: a NaN logit
-      }
-    }
-    asm volatile("bar.sync 2, %0;" ::"r"(kCT) : "memory");
-    if (ct < 32) {
-      const float m = sel_w[0];
-      const float ev = ct < p.k ? expf(sel_w[ct] - m) : 0.f;
-      float sum = ev;
-#pragma unroll
-      for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
-      __syncwarp();   // every lane has read sel_w[0]
-      if (ct < p.k) sel_w[ct] = ev * (1.f / sum);
-    }
+    // ---- routing of the token
+    route_token(p.logits, p.E, p.k, keys, sel_e, sel_w, ct);
     // ---- staging: control thread s < nslot_c stages gate/up slot s; 32 + s < 32 + nslot_d prefetches down slot s
     const int A = p.k;
     const int nci = A * 2 * p.NRB * p.nseg;

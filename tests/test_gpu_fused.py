@@ -103,6 +103,22 @@ def test_fused_top1_and_all_experts(env):
         check(env, layer, x, logits, k, L=L)
 
 
+@pytest.mark.parametrize("E", [33, 200, 256])
+def test_fused_routing_ties_many_experts(env, E):
+    """Routing inside the fused kernel with several keys per lane (E > 32), ragged
+    E, many exact ties and signed zeros: the k largest logits, ties to the lower index."""
+    spec = small(E=E, n=40, I=128)
+    layer = synth.make_layer(spec, seed=E)
+    x, _ = synth.make_inputs(spec, 1, seed=E)
+    rng = np.random.default_rng(E)
+    logits = rng.integers(-2, 3, size=(1, E)).astype(np.float32)
+    logits[0, rng.integers(0, E, size=4)] = -0.0
+    torch, bm = env
+    L = bm.bitsmoe_pack(layer, device=0)
+    for k in (1, 8, 32):
+        check(env, layer, x, logits, k, L=L)
+
+
 def test_fused_consecutive_calls_layers_and_workspace_state(env):
     torch, bm = env
     spec = synth.scaled_spec(synth.WORKLOADS["qw3"], D=512, E=32, I=384, n=512, top_k=4)
