@@ -147,6 +147,15 @@ size_t bitsmoe_workspace_bytes(const bitsmoe_layer* layer, int T, int top_k);
  * arguments. */
 int bitsmoe_forward_launches(const bitsmoe_layer* layer, int T, int top_k);
 
+/* How a forward of T tokens runs on this layer, as a bit set:
+ *   1  the fused single-token kernel
+ *   2  the small-batch decode chain (2 <= T <= 8)
+ *   4  tensor-core (tcgen05) shared-basis projections
+ *   8  tensor-core gate/up factors (layers without 16-bit units whose group is
+ *      a multiple of 128 rows; otherwise the dp2a kernel)
+ * Returns a negative error code for invalid arguments; 0 for T == 0. */
+int bitsmoe_forward_plan(const bitsmoe_layer* layer, int T, int top_k);
+
 /* Kernels one bitsmoe_moe_block_forward call launches: 1 when the fused
  * single-token kernel runs (it computes the pre-norm and router too),
  * otherwise the norm/router kernel plus bitsmoe_forward_launches. */

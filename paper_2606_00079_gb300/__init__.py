@@ -57,6 +57,7 @@ SIGNATURES = {
     "bitsmoe_workspace_bytes": (_SZ, [_P, _I, _I]),
     "bitsmoe_forward_launches": (_I, [_P, _I, _I]),
     "bitsmoe_block_forward_launches": (_I, [_P, _I, _I]),
+    "bitsmoe_forward_plan": (_I, [_P, _I, _I]),
     "bitsmoe_moe_forward": (_I, [_P, _P, _I, _I, _P, _P, _P, _SZ, _P]),
     "bitsmoe_moe_forward_host": (_I, [_P, _P, _I, _I, _P, _P, _P, _SZ, _P]),
     "bitsmoe_moe_forward_noalloc": (_I, [_P, _P, _I, _I, _P, _P, _P]),
@@ -234,6 +235,18 @@ def bitsmoe_forward_launches(layer: Layer, T: int, top_k: int) -> int:
     n = int(_lib().bitsmoe_forward_launches(layer.handle, T, top_k))
     if n < 0:
         raise BitsMoEError(n, "bitsmoe_forward_launches")
+    return n
+
+
+PLAN_FUSED, PLAN_DECODE_CHAIN, PLAN_TC_PROJECTIONS, PLAN_TC_GATE_UP = 1, 2, 4, 8
+
+
+def bitsmoe_forward_plan(layer: Layer, T: int, top_k: int) -> int:
+    """Bit set of how a T-token forward runs: PLAN_FUSED, PLAN_DECODE_CHAIN, PLAN_TC_PROJECTIONS,
+    PLAN_TC_GATE_UP."""
+    n = int(_lib().bitsmoe_forward_plan(layer.handle, T, top_k))
+    if n < 0:
+        raise BitsMoEError(n, "bitsmoe_forward_plan")
     return n
 
 

@@ -101,7 +101,11 @@ cudaError_t launch_fused(const Fwd& p, const FusedArgs& f, int sms, cudaStream_t
 // y += Phi_dn s (mode 1) for all T tokens of p (z, resp. y, zeroed before
 // unless y carries a residual).
 bool make_basis_map(void* map_out, const void* base, int rows, int cols_pad);
-cudaError_t launch_gemm_tc(int mode, const void* map, const Fwd& p, int sms, cudaStream_t st, bool pdl);
+cudaError_t launch_gemm_tc(int mode, const void* map, const Fwd& p, int sms, cudaStream_t st, bool pdl,
+                           bool zt = false);
+// Tensor-core gate/up factors of every routed expert (z stored [2][n_pad][T]); the
+// layer's most row-lane tiles and slots of any gate/up (h, e) size the shared memory.
+cudaError_t launch_gu_tc(const Fwd& p, int max_tiles, int max_slots, cudaStream_t st, bool pdl);
 // Staging records of a packed image (host side, at upload).
 void build_stage_tables(const uint8_t* img, std::vector<CStage>& cst, std::vector<DStage>& dst);
 

@@ -52,6 +52,9 @@ struct bitsmoe_layer {
   alignas(64) uint8_t map_in[128];    // TMA maps of the two input bases and of the output basis
   alignas(64) uint8_t map_out[128];
   bool maps = false;
+  bool tcx = false;            // gate/up factors on tensor cores: no 16-bit units, groups of whole row blocks
+  int rl_max_tiles = 0;        // most row-lane tiles and slots of any gate/up (h, e)
+  int rl_max_slots = 0;
   std::vector<uint8_t> meta;   // host copy of header + descriptors + segment table
   int seg_bytes = 0;           // largest gate/up item: code bytes inside one row block
   int ul_max_chunks = 1;       // largest 16-byte chunks per row block of any down unit
@@ -1309,20 +1312,24 @@ int launch_gemv_bulk(bool proj, const Fwd& p, int sms, cudaStream_t st, bool pdl
   return launch_gemv_bulk_tb<8>(proj, p, sms, st, pdl);
 }
 
+// parts: 1 the gate/up kernel, 2 the down kernel, 3 both
 template <int G, int TB>
 int launch_k2k3_dec(const Fwd& p, int A_max, int sms, cudaStream_t st, bool pdl,
-                    const std::function<int()>& between) {
+                    const std::function<int()>& between, int parts = 3) {
   int rc;
   const size_t rbytes = 0;
-  const size_t smax = (size_t)p.s16 - 8;
-  const size_t pw2 = (size_t)p.seg_bytes + smax * 4 * (2 + G) + (size_t)G * TB * p.s16 * 2 + 16;
-  const size_t sm2 = rbytes + kK2DecWarps * pw2;
-  const int items2 = A_max * 2 * p.NRB * p.nseg;
-  if ((rc = set_smem(k_gateup_dec<G, TB>, sm2))) return rc;
-  if ((rc = launch(k_gateup_dec<G, TB>, dim3((items2 + kK2DecWarps - 1) / kK2DecWarps), dim3(kK2DecWarps * 32), sm2,
-                   st, pdl, p)))
-    return rc;
+  if (parts & 1) {
+    const size_t smax = (size_t)p.s16 - 8;
+    const size_t pw2 = (size_t)p.seg_bytes + smax * 4 * (2 + G) + (size_t)G * TB * p.s16 * 2 + 16;
+    const size_t sm2 = rbytes + kK2DecWarps * pw2;
+    const int items2 = A_max * 2 * p.NRB * p.nseg;
+    if ((rc = set_smem(k_gateup_dec<G, TB>, sm2))) return rc;
+    if ((rc = launch(k_gateup_dec<G, TB>, dim3((items2 + kK2DecWarps - 1) / kK2DecWarps), dim3(kK2DecWarps * 32),
+                     sm2, st, pdl, p)))
+      return rc;
+  }
   if (between && (rc = between())) return rc;
+  if (!(parts & 2)) return BITSMOE_OK;
   const size_t nrm = (size_t)p.rbc * kRows;
   const int ngc_max = std::max(1, (int)(nrm / p.group));
   const size_t pw3 = (size_t)p.ul_bytes + (size_t)ngc_max * 32 * 4 + 16;
@@ -1479,23 +1486,30 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
   if ((rc = launch(k_router, dim3((T + tpb - 1) / tpb), dim3(1024), router_smem, st, false, p))) return rc;
   if ((rc = mark(1))) return rc;
   const bool tc = L->maps;   // tensor-core projections for multi-token calls
+  const bool tcx = tc && L->tcx;   // and tensor-core gate/up factors (z then stored token-fastest)
   if (tc) {
     // the projection, the gate/up and the down kernels add into z, gu and s (adjacent in
     // the workspace); the output basis adds into y (which keeps the residual when accumulating)
     BM_CK(cudaMemsetAsync(p.z, 0, (size_t)(reinterpret_cast<uint8_t*>(p.s) - reinterpret_cast<uint8_t*>(p.z)) +
                                       (size_t)T * hd.n_pad * 4, st));
     if (!accum) BM_CK(cudaMemsetAsync(y, 0, (size_t)T * hd.D * 4, st));
-    BM_CK(launch_gemm_tc(0, L->map_in, p, sms, st, false));
+    BM_CK(launch_gemm_tc(0, L->map_in, p, sms, st, false, tcx));
   } else if ((rc = launch_gemv_any(true, p, sms, st, pdl))) {
     return rc;
   }
   if ((rc = mark(2))) return rc;
-  {   // gate/up and down factors: the staged kernels, every routed expert's tokens in batches of 4
+  {   // gate/up factors (tensor cores, or the staged dp2a kernel over batches of 4 tokens), then down
     std::function<int()> between = ev ? std::function<int()>([&]() { return mark(3); }) : std::function<int()>();
     const int A_max = std::min(hd.E, p.P);
-    if (G == 1) rc = launch_k2k3_dec<1, 4>(p, A_max, sms, st, pdl, between);
-    else if (G == 2) rc = launch_k2k3_dec<2, 4>(p, A_max, sms, st, pdl, between);
-    else rc = launch_k2k3_dec<4, 4>(p, A_max, sms, st, pdl, between);
+    if (tcx) {
+      BM_CK(launch_gu_tc(p, L->rl_max_tiles, L->rl_max_slots, st, pdl));
+      if ((rc = mark(3))) return rc;
+      between = std::function<int()>();
+    }
+    const int parts = tcx ? 2 : 3;
+    if (G == 1) rc = launch_k2k3_dec<1, 4>(p, A_max, sms, st, pdl, between, parts);
+    else if (G == 2) rc = launch_k2k3_dec<2, 4>(p, A_max, sms, st, pdl, between, parts);
+    else rc = launch_k2k3_dec<4, 4>(p, A_max, sms, st, pdl, between, parts);
   }
   if (rc) return rc;
   if ((rc = mark(4))) return rc;
@@ -1551,6 +1565,15 @@ int upload(std::vector<uint8_t>&& img, int device, bitsmoe_layer** out) {
     const ImageHeader* h = header_of(img.data());
     L->maps = make_basis_map(L->map_in, d + h->off_basis_in, 2 * h->n, h->D_pad) &&
               make_basis_map(L->map_out, d + h->off_basis_out, h->D, h->n_pad);
+    bool ok16 = h->group % kRows == 0;
+    const ExpertDesc* xd = desc_of(img.data());
+    for (int i = 0; i < 2 * h->E; ++i) {
+      for (int k = 0; k < xd[i].nbk; ++k)
+        if (xd[i].bk[k].bits >= 16) ok16 = false;
+      L->rl_max_tiles = std::max(L->rl_max_tiles, (int)xd[i].ntiles);
+      L->rl_max_slots = std::max(L->rl_max_slots, (int)xd[i].nslots);
+    }
+    L->tcx = ok16;
   }
   const ImageHeader* hd = header_of(img.data());
   const size_t meta_end = hd->off_basis_in;   // header + descriptors + segments
@@ -1692,6 +1715,15 @@ int bitsmoe_forward_launches(const bitsmoe_layer* L, int T, int top_k) {
   const int s16 = (int)align_up(std::max(hd.seg_max_slots, 8), 64) + 8;
   if (decode && fused_plan(hd, T, top_k, L->seg_bytes, L->ul_max_chunks, s16, L->num_sms, &fa)) return 1;
   return 5;
+}
+
+int bitsmoe_forward_plan(const bitsmoe_layer* L, int T, int top_k) {
+  const int n = bitsmoe_forward_launches(L, T, top_k);
+  if (n <= 0) return n;
+  if (n == 1) return 1;
+  const ImageHeader& hd = L->hd();
+  if (T <= 8 && T * hd.E <= 4096) return 2;
+  return L->maps ? (L->tcx ? 4 | 8 : 4) : 0;
 }
 
 int bitsmoe_block_forward_launches(const bitsmoe_layer* L, int T, int top_k) {

@@ -23,6 +23,7 @@
 #include <mutex>
 
 #include "device.cuh"
+#include "tc.cuh"
 
 namespace {
 
@@ -30,46 +31,11 @@ constexpr int kGThreads = 128;
 constexpr int kKB = 64;                    // K elements per stage (one 128-byte swizzle row of bf16)
 constexpr uint32_t kATile = 128 * kKB * 2; // bytes of an A stage (128 rows)
 
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
-  uint64_t d = 0;
-  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);   // start address
-  d |= (uint64_t)1 << 16;                      // leading byte offset (unused for swizzled K-major)
-  d |= (uint64_t)(1024 >> 4) << 32;            // stride byte offset: 8 rows x 128 bytes
-  d |= (uint64_t)1 << 46;                      // descriptor version
-  d |= (uint64_t)2 << 61;                      // 128-byte swizzle
-  return d;
-}
-
-// kind::f16 instruction descriptor: bf16 x bf16 -> f32, both K-major, M = 128, N.
-__host__ __device__ constexpr uint32_t idesc_bf16(int n) {
-  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
-}
-
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
   asm volatile(
       "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
       : "memory");
-}
-
-__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
-      "l"(a), "l"(b), "r"(idesc), "r"(acc)
-      : "memory");
-}
-
-__device__ __forceinline__ void mma_commit(uint64_t* bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
-               : "memory");
-}
-
-__device__ __forceinline__ void mbar_init_n(uint64_t* bar, uint32_t n) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(n) : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }
 
 struct GemmArgs {
@@ -87,7 +53,8 @@ struct GemmArgs {
   int D;             // mode 1: output row length
   const uint16_t* x; // mode 0: [T][D] bf16 bits
   const float* s;    // mode 1: [T][n_pad]
-  float* z;          // mode 0: [2][T][n_pad], zeroed before
+  int zt;            // mode 0: z stored [2][n_pad][T] (token fastest) instead of [2][T][n_pad]
+  float* z;          // mode 0: zeroed before
   float* y;          // mode 1: [T][D], zeroed before unless accumulating
   int* status;
 };
@@ -225,7 +192,7 @@ __global__ void __launch_bounds__(kGThreads, 1) k_gemm_tc(const __grid_constant_
           const float v = __uint_as_float(r[q]);
           if (g.mode == 0) {
             const int h = m >= g.n, j = m - h * g.n;
-            atomicAdd(g.z + ((size_t)h * g.T + t) * g.n_pad + j, v);
+            atomicAdd(g.z + (g.zt ? ((size_t)h * g.n_pad + j) * g.T + t : ((size_t)h * g.T + t) * g.n_pad + j), v);
           } else {
             atomicAdd(g.y + (size_t)t * g.D + m, v);
           }
@@ -279,7 +246,7 @@ bool make_basis_map(void* map_out, const void* base, int rows, int cols_pad) {
 
 // mode 0: z += Phi_{g,u}^T x for all T tokens; mode 1: y += Phi_dn s.  The
 // target must hold zeros (or the residual, for y) before the launch.
-cudaError_t launch_gemm_tc(int mode, const void* map, const Fwd& p, int sms, cudaStream_t st, bool pdl) {
+cudaError_t launch_gemm_tc(int mode, const void* map, const Fwd& p, int sms, cudaStream_t st, bool pdl, bool zt) {
   static_assert(sizeof(CUtensorMap) == 128, "tensor map size");
   GemmArgs g;
   std::memset(&g, 0, sizeof(g));
@@ -297,6 +264,7 @@ cudaError_t launch_gemm_tc(int mode, const void* map, const Fwd& p, int sms, cud
   g.z = p.z;
   g.y = p.y;
   g.status = p.status;
+  g.zt = zt ? 1 : 0;
   CUtensorMap amap;
   std::memcpy(&amap, map, sizeof(amap));
   static std::mutex mu;
