@@ -151,8 +151,9 @@ int bitsmoe_forward_launches(const bitsmoe_layer* layer, int T, int top_k);
  *   1  the fused single-token kernel
  *   2  the small-batch decode chain (2 <= T <= 8)
  *   4  tensor-core (tcgen05) shared-basis projections
- *   8  tensor-core gate/up factors (layers without 16-bit units whose group is
- *      a multiple of 128 rows; otherwise the dp2a kernel)
+ *   8  tensor-core gate/up factors (layers without 16-bit gate/up units whose
+ *      group is a multiple of 128 rows; otherwise the dp2a kernel)
+ *  16  tensor-core down factor (the same condition on the down units)
  * Returns a negative error code for invalid arguments; 0 for T == 0. */
 int bitsmoe_forward_plan(const bitsmoe_layer* layer, int T, int top_k);
 

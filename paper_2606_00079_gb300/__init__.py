@@ -238,12 +238,12 @@ def bitsmoe_forward_launches(layer: Layer, T: int, top_k: int) -> int:
     return n
 
 
-PLAN_FUSED, PLAN_DECODE_CHAIN, PLAN_TC_PROJECTIONS, PLAN_TC_GATE_UP = 1, 2, 4, 8
+PLAN_FUSED, PLAN_DECODE_CHAIN, PLAN_TC_PROJECTIONS, PLAN_TC_GATE_UP, PLAN_TC_DOWN = 1, 2, 4, 8, 16
 
 
 def bitsmoe_forward_plan(layer: Layer, T: int, top_k: int) -> int:
     """Bit set of how a T-token forward runs: PLAN_FUSED, PLAN_DECODE_CHAIN, PLAN_TC_PROJECTIONS,
-    PLAN_TC_GATE_UP."""
+    PLAN_TC_GATE_UP, PLAN_TC_DOWN."""
     n = int(_lib().bitsmoe_forward_plan(layer.handle, T, top_k))
     if n < 0:
         raise BitsMoEError(n, "bitsmoe_forward_plan")

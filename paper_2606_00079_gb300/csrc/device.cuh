@@ -106,6 +106,9 @@ cudaError_t launch_gemm_tc(int mode, const void* map, const Fwd& p, int sms, cud
 // Tensor-core gate/up factors of every routed expert (z stored [2][n_pad][T]); the
 // layer's most row-lane tiles and slots of any gate/up (h, e) size the shared memory.
 cudaError_t launch_gu_tc(const Fwd& p, int max_tiles, int max_slots, cudaStream_t st, bool pdl);
+// Tensor-core down factor of every routed expert into s (zeroed before); ul_max_tiles:
+// the layer's most unit-lane tiles of any expert.
+cudaError_t launch_dn_tc(const Fwd& p, int ul_max_tiles, cudaStream_t st, bool pdl);
 // Staging records of a packed image (host side, at upload).
 void build_stage_tables(const uint8_t* img, std::vector<CStage>& cst, std::vector<DStage>& dst);
 

@@ -384,6 +384,321 @@ __global__ void __launch_bounds__(kXThreads, 2) k_gu_tc(Fwd p, XArgs xa) {
   if (wid == 1) tmem_dealloc(tmem, ncols);
 }
 
+// ---------------------------------------------------------------------------
+// Down factor on tensor cores (Eq. 3's down projection, summed over the routed
+// experts before the output basis):
+//
+//   s[t][j] += g_{t,e} * alpha_{dn,e,j} * sum_i p_hat[i, j] * h_{t,e}[i]
+//   p_hat[i, j] = scale_{j,g(i)} * (q_ij - zero_{j,g(i)}),   h = SiLU(gate) * up
+//
+// One block per (routed expert, 128 down slots = four unit-lane tiles); the K
+// dimension is the expert's rows i, one row block (two K-blocks) per step:
+//   A[slot][i] = q_ij (bf16, exact), decoded from the unit-lane streams (a lane owns a
+//                unit and its codes run along i);
+//   B[t][i]    = h_t[i] as a bf16 pair hi + lo;
+//   per group: P = A B in TMEM; out[slot][t] += scale * (P - zero * H_g[t]) in
+//              registers, H_g[t] = sum over the group's rows of h_t[i];
+//   finally s[t][unit] += g_{t,e} * alpha * out with fp32 reductions (experts meet in s).
+// ---------------------------------------------------------------------------
+constexpr int kDNT = 64;   // largest token tile of the down kernel
+
+struct DArgs {
+  int NTmax;   // 16 .. 64, power of two
+  int mt_max;  // 128-slot tiles of the largest down (e)
+};
+
+// 4 codes of rows 4k .. 4k + 3 -> A[slot = row][K = kk .. kk + 3] (kk: row inside the row block)
+__device__ __forceinline__ void store_a4(uint8_t* sa, int row, int kk, uint2 v) {
+  const uint32_t off = (uint32_t)(kk >> 6) * kXATile + (uint32_t)(row >> 3) * 1024u + (uint32_t)(row & 7) * 128u +
+                       ((uint32_t)(((kk & 63) >> 3) ^ (row & 7)) << 4) + ((uint32_t)((kk >> 2) & 1) << 3);
+  *reinterpret_cast<uint2*>(sa + off) = v;
+}
+
+// Rows 64 hp .. 64 hp + 63 of one unit's staged row block (its 16-byte chunks at
+// `ln`, chunk c at ln + 512 c) into A row `row`.
+template <int B>
+__device__ __forceinline__ void decode_ul(const uint8_t* ln, int hp, int row, uint8_t* sa) {
+  if (B == 3) {   // low 2-bit plane: chunk hp, word w = rows 64 hp + 16 w ..; high bit: chunk 2, word = row / 32
+    const uint8_t* lo = ln + hp * kChunkBytes;
+    const uint8_t* hi = ln + 2 * kChunkBytes;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+      const uint32_t wl = lds32(lo + 4 * w), wh = lds32(hi + 4 * (2 * hp + (w >> 1)));
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const uint32_t q = ((wl >> (2 * k)) & 0x03030303u) | (((wh >> (4 * (w & 1) + k)) & 0x01010101u) << 2);
+        store_a4(sa, row, 64 * hp + 16 * w + 4 * k, codes_bf16(q, 3));
+      }
+    }
+  } else if (B == 6) {   // low 4-bit plane: chunks 2hp, 2hp+1 (rows 32c + 8w ..); high 2 bits: chunk 4 + hp (16 rows a word)
+#pragma unroll
+    for (int cc = 0; cc < 2; ++cc) {
+      const uint8_t* lo = ln + (2 * hp + cc) * kChunkBytes;
+#pragma unroll
+      for (int w = 0; w < 4; ++w) {
+        const int r0 = 32 * cc + 8 * w;   // row inside this half
+        const uint32_t wl = lds32(lo + 4 * w), wh = lds32(ln + (4 + hp) * kChunkBytes + 4 * (r0 >> 4));
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+          const int rr = r0 + 4 * k;
+          const uint32_t q = ((wl >> (4 * k)) & 0x0F0F0F0Fu) | (((wh >> (2 * ((rr & 15) >> 2))) & 0x03030303u) << 4);
+          store_a4(sa, row, 64 * hp + rr, codes_bf16(q, 6));
+        }
+      }
+    }
+  } else {   // 1, 2, 4, 8: chunk c covers rows 128c/B .., word 32/B rows, group k at bit B*k
+    constexpr int RPW = 32 / B;   // rows per word
+    constexpr uint32_t kMask = B == 1 ? 0x01010101u : B == 2 ? 0x03030303u : B == 4 ? 0x0F0F0F0Fu : 0xFFFFFFFFu;
+#pragma unroll
+    for (int wi = 0; wi < 2 * B; ++wi) {   // the 2B words of rows 64 hp ..
+      const int gw = 2 * B * hp + wi;      // word index over the row block
+      const uint32_t wv = lds32(ln + (gw >> 2) * kChunkBytes + 4 * (gw & 3));
+#pragma unroll
+      for (int k = 0; k < RPW / 4; ++k) store_a4(sa, row, gw * RPW + 4 * k, codes_bf16((wv >> (B * k)) & kMask, B));
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kXThreads, 2) k_dn_tc(Fwd p, DArgs da) {
+  extern __shared__ uint8_t dsm_raw[];
+  uint8_t* dsm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(dsm_raw) + 1023) & ~(uintptr_t)1023);
+  constexpr uint32_t kCodeBuf = 4 * 8 * kChunkBytes;              // four tiles of at most 8 chunks
+  uint8_t* sa = dsm;                                                // [2 K-blocks][128 x 128 B]
+  uint8_t* sb = sa + 2 * kXATile;                                   // hi [2][NT x 128 B], then lo
+  const uint32_t b_half = 2u * da.NTmax * 128u;
+  uint8_t* cbuf = sb + 2 * (size_t)b_half;                          // [2][kCodeBuf]
+  uint32_t* szb = reinterpret_cast<uint32_t*>(cbuf + 2 * kCodeBuf); // [2][128] scale | zero of the group
+  int* su = reinterpret_cast<int*>(szb + 256);                      // [128] unit of each slot
+  float* sal = reinterpret_cast<float*>(su + 128);                  // [128] alpha
+  float* hs = sal + 128;                                            // [2][kDNT] group sums of h per token
+  int* tok = reinterpret_cast<int*>(hs + 2 * kDNT);                 // [kDNT]
+  float* pw = reinterpret_cast<float*>(tok + kDNT);                 // [kDNT] gate weight of the pair
+  int* pairs = reinterpret_cast<int*>(pw + kDNT);                   // [kDNT]
+  int* tq = pairs + kDNT;                                           // [4] bits | [4] buffer offset | [4] stream offset
+  uint64_t* cbar = reinterpret_cast<uint64_t*>(tq + 12);            // [2]
+  uint64_t* bar = cbar + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar + 1);
+  const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+
+  pdl_trigger();
+  const int mt = blockIdx.x % da.mt_max, a = blockIdx.x / da.mt_max;
+  pdl_wait();   // routing and gate/up come from earlier kernels
+  if (a >= p.active[0]) return;
+  const int e = p.active[1 + a];
+  const int ntok = p.expert_count[e], pst = p.expert_start[e];
+  const ExpertDesc& xd = p.desc[2 * p.E + e];
+  const int m0 = mt * 128;
+  if (ntok <= 0 || m0 >= xd.nslots) return;
+  const int nslots = xd.nslots, nsl = min(128, nslots - m0), nq = nsl / 32;
+  const int nt_need = min(da.NTmax, max(16, (ntok + 15) & ~15));
+  int NT = 16;
+  while (NT < nt_need) NT <<= 1;
+  const uint32_t ncols = NT < 32 ? 32u : (uint32_t)NT;
+  const int lgNT = 31 - __clz(NT);
+
+  if (tid < 4) {   // the block's unit-lane tiles: bits, offset in the code buffer, stream offset of row block 0
+    const int t = 4 * mt + tid;
+    int bits = 0, src = 0;
+    if (tid < nq) {
+      int k = 0;
+      for (int q = 1; q < xd.nbk; ++q)
+        if (t >= xd.bk[q].tile0) k = q;
+      bits = xd.bk[k].bits;
+      src = (int)xd.bk[k].code_off + (t - xd.bk[k].tile0) * p.NRB * bits * kChunkBytes;
+    }
+    tq[tid] = bits;
+    tq[8 + tid] = src;
+  }
+  if (tid < 128) {
+    su[tid] = tid < nsl ? reinterpret_cast<const int*>(p.img + xd.unit_off)[m0 + tid] : 0;
+    sal[tid] = tid < nsl ? reinterpret_cast<const float*>(p.img + xd.alpha_off)[m0 + tid] : 0.f;
+  }
+  if (tid < 2 * kDNT) hs[tid] = 0.f;
+  if (tid == 0) {
+    mbar_init_n(bar, 1);
+    mbar_init(cbar);
+    mbar_init(cbar + 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (wid == 1) tmem_alloc(tmem_slot, ncols);
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  if (tid == 0) {
+    int o = 0;
+    for (int q = 0; q < 4; ++q) {
+      tq[4 + q] = o;
+      o += tq[q] * kChunkBytes;
+    }
+  }
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t idesc = idesc_bf16(NT);
+  const uint8_t* code = p.img + xd.code_base;
+  const uint32_t* szg = reinterpret_cast<const uint32_t*>(p.img + xd.sz_off);
+
+  // row block r of the four tiles (each tile's B chunks are contiguous per row block) and
+  // the scale/zero of its group, into buffer r & 1 (one thread)
+  auto issue = [&](int r) {
+    if (r >= p.NRB) return;
+    const int buf = r & 1, g = (r * kRows) / p.group;
+    uint32_t bytes = (uint32_t)nsl * 4;
+    for (int q = 0; q < nq; ++q) bytes += (uint32_t)tq[q] * kChunkBytes;
+    fence_proxy_async();
+    mbar_expect_tx(cbar + buf, bytes);
+    for (int q = 0; q < nq; ++q)
+      bulk_g2s(cbuf + (size_t)buf * kCodeBuf + tq[4 + q], code + tq[8 + q] + (size_t)r * tq[q] * kChunkBytes,
+               (uint32_t)tq[q] * kChunkBytes, cbar + buf);
+    bulk_g2s(szb + buf * 128, szg + (size_t)g * nslots + m0, (uint32_t)nsl * 4, cbar + buf);
+  };
+
+  float out[kDNT];
+  uint32_t ncommit = 0, cuse = 0;
+  bool ok = true;
+  for (int tt0 = 0; tt0 < ntok; tt0 += NT) {
+    const int nt = min(NT, ntok - tt0);
+#pragma unroll
+    for (int q = 0; q < kDNT; ++q) out[q] = 0.f;
+    __syncthreads();   // the previous tile's scatter has read tok / pw
+    for (int t = tid; t < NT; t += kXThreads) {
+      const int q = t < nt ? p.pair_list[pst + tt0 + t] : 0;
+      pairs[t] = q;
+      tok[t] = q / p.k;
+      pw[t] = t < nt ? p.pair_weight[q] : 0.f;
+    }
+    if (tid < 2 * kDNT) hs[tid] = 0.f;
+    __syncthreads();
+    if (tid == 32) issue(0);
+    for (int r = 0; r < p.NRB; ++r) {
+      const int buf = r & 1, g = (r * kRows) / p.group;
+      const bool gfirst = (r * kRows) % p.group == 0, glast = ((r + 1) * kRows) % p.group == 0 || r == p.NRB - 1;
+      if (tid == 0) {
+        if (ncommit > 0) ok &= mbar_wait(bar, (ncommit - 1) & 1u);
+        ok &= mbar_wait(cbar + buf, (cuse >> buf) & 1u);
+      }
+      cuse ^= 1u << buf;
+      asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+      __syncthreads();
+      asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+      if (tid == 32) issue(r + 1);
+      // A: thread = (slot, half of the rows); a warp holds 32 slots of one tile
+      {
+        const int m = tid & 127, hp = tid >> 7, q = m >> 5;
+        const int bits = tq[q];
+        const uint8_t* ln = cbuf + (size_t)buf * kCodeBuf + tq[4 + q] + (m & 31) * 16;
+        switch (bits) {
+          case 1: decode_ul<1>(ln, hp, m, sa); break;
+          case 2: decode_ul<2>(ln, hp, m, sa); break;
+          case 3: decode_ul<3>(ln, hp, m, sa); break;
+          case 4: decode_ul<4>(ln, hp, m, sa); break;
+          case 6: decode_ul<6>(ln, hp, m, sa); break;
+          case 8: decode_ul<8>(ln, hp, m, sa); break;
+          default: {   // slots past the expert's last tile: zeros
+#pragma unroll
+            for (int kk = 0; kk < 64; kk += 4) store_a4(sa, m, 64 * hp + kk, make_uint2(0u, 0u));
+          }
+        }
+      }
+      // B: thread (token row t, 8-row chunk c) with t fixed per thread; h = SiLU(gate) * up
+      {
+        const int t = tid & (NT - 1);
+        const bool live = t < nt;
+        const float* gp = p.gu + (size_t)pairs[t] * 2 * p.I_pad + (size_t)r * kRows;
+        float hsum = 0.f;
+        for (int item = tid; item < NT * 16; item += kXThreads) {
+          const int c = item >> lgNT;
+          float hv[8];
+          if (live) {
+            const float4 g0 = __ldcg(reinterpret_cast<const float4*>(gp + 8 * c));
+            const float4 g1 = __ldcg(reinterpret_cast<const float4*>(gp + 8 * c + 4));
+            const float4 u0 = __ldcg(reinterpret_cast<const float4*>(gp + p.I_pad + 8 * c));
+            const float4 u1 = __ldcg(reinterpret_cast<const float4*>(gp + p.I_pad + 8 * c + 4));
+            const float gg[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+            const float uu[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+#pragma unroll
+            for (int u = 0; u < 8; ++u) hv[u] = gg[u] / (1.f + __expf(-gg[u])) * uu[u];
+          } else {
+#pragma unroll
+            for (int u = 0; u < 8; ++u) hv[u] = 0.f;
+          }
+          uint32_t hw[4], lw[4];
+#pragma unroll
+          for (int m2 = 0; m2 < 4; ++m2) {
+            const float v0 = hv[2 * m2], v1 = hv[2 * m2 + 1];
+            hsum += v0 + v1;
+            const uint32_t h0 = __float_as_uint(v0) & 0xFFFF0000u, h1 = __float_as_uint(v1) & 0xFFFF0000u;
+            hw[m2] = __byte_perm(h0, h1, 0x7632);
+            const __nv_bfloat162 bl = __floats2bfloat162_rn(v0 - __uint_as_float(h0), v1 - __uint_as_float(h1));
+            lw[m2] = *reinterpret_cast<const uint32_t*>(&bl);
+          }
+          const uint32_t off = (uint32_t)(c >> 3) * (uint32_t)NT * 128u + sw_off(t, c & 7);
+          *reinterpret_cast<uint4*>(sb + off) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+          *reinterpret_cast<uint4*>(sb + b_half + off) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+        }
+        if (live && hsum != 0.f) atomicAdd(hs + (g & 1) * kDNT + t, hsum);
+      }
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+      __syncthreads();
+      if (tid == 0) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+#pragma unroll
+        for (int kb = 0; kb < 2; ++kb) {
+          const uint32_t a0 = smem_u32(sa + (size_t)kb * kXATile);
+          const uint32_t b0 = smem_u32(sb + (size_t)kb * NT * 128);
+#pragma unroll
+          for (int k16 = 0; k16 < 4; ++k16) {
+            const uint64_t ad = sw128_desc(a0 + k16 * 32);
+            mma_bf16(tmem, ad, sw128_desc(b0 + k16 * 32), idesc, (!gfirst || kb || k16) ? 1u : 0u);
+            mma_bf16(tmem, ad, sw128_desc(b0 + b_half + k16 * 32), idesc, 1u);
+          }
+        }
+        mma_commit(bar);
+      }
+      ++ncommit;
+      if (glast) {   // the group's partial sums: out += scale * (P - zero * H)
+        if (tid == 0) ok &= mbar_wait(bar, (ncommit - 1) & 1u);
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        __syncthreads();
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        if (wid < 4) {
+          const int m = 32 * wid + lane;
+          const uint32_t szw = szb[buf * 128 + m];
+          const float sc = m < nsl ? __half2float(__ushort_as_half((unsigned short)(szw & 0xFFFFu))) : 0.f;
+          const float zp = m < nsl ? __half2float(__ushort_as_half((unsigned short)(szw >> 16))) : 0.f;
+          const float* hg = hs + (g & 1) * kDNT;
+#pragma unroll
+          for (int c0 = 0; c0 < kDNT; c0 += 8) {
+            if (c0 < nt) {
+              uint32_t rr[8];
+              tmem_ld8(tmem + ((uint32_t)(32 * wid) << 16) + (uint32_t)c0, rr);
+#pragma unroll
+              for (int q = 0; q < 8; ++q) out[c0 + q] = fmaf(sc, __uint_as_float(rr[q]) - zp * hg[c0 + q], out[c0 + q]);
+            }
+          }
+        } else {   // the other warps clear the next group's sums
+          for (int t = tid - 128; t < kDNT; t += 128) hs[((g + 1) & 1) * kDNT + t] = 0.f;
+        }
+      }
+    }
+    // s[t][unit] += g_{t,e} * alpha * out (experts meet in s: fp32 reductions)
+    if (wid < 4) {
+      const int m = 32 * wid + lane;
+      const float al = sal[m];
+      if (m < nsl && al != 0.f) {
+        float* sp = p.s + su[m];
+#pragma unroll
+        for (int q = 0; q < kDNT; ++q)
+          if (q < nt) atomicAdd(sp + (size_t)tok[q] * p.n_pad, pw[q] * al * out[q]);
+      }
+    }
+  }
+  if (!ok && tid == 0) atomicCAS(p.status, 0, BITSMOE_ERR_TIMEOUT);
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  if (wid == 1) tmem_dealloc(tmem, ncols);
+}
+
 }  // namespace
 
 namespace bmoe {
@@ -427,6 +742,38 @@ cudaError_t launch_gu_tc(const Fwd& p, int max_tiles, int max_slots, cudaStream_
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, k_gu_tc, p, xa);
+}
+
+cudaError_t launch_dn_tc(const Fwd& p, int ul_max_tiles, cudaStream_t st, bool pdl) {
+  DArgs da;
+  int nt = 16;
+  while (nt < p.T && nt < kDNT) nt <<= 1;   // experts with more tokens take several token tiles
+  da.NTmax = nt;
+  da.mt_max = std::max(1, (ul_max_tiles + 3) / 4);
+  const size_t smem = 1024 + 2 * (size_t)kXATile + 4 * (size_t)nt * 128 + 2 * 4 * 8 * kChunkBytes + 256 * 4 +
+                      128 * 8 + 2 * kDNT * 4 + 3 * kDNT * 4 + 12 * 4 + 3 * 8 + 16;
+  static std::mutex mu;
+  static size_t done = 0;
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    if (smem > done) {
+      const cudaError_t r = cudaFuncSetAttribute(k_dn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (r != cudaSuccess) return r;
+      done = smem;
+    }
+  }
+  const int A_max = std::min(p.E, p.P);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(A_max * da.mt_max));
+  cfg.blockDim = dim3(kXThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, k_dn_tc, p, da);
 }
 
 }  // namespace bmoe

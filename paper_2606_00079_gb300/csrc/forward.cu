@@ -53,6 +53,7 @@ struct bitsmoe_layer {
   alignas(64) uint8_t map_out[128];
   bool maps = false;
   bool tcx = false;            // gate/up factors on tensor cores: no 16-bit units, groups of whole row blocks
+  bool tcd = false;            // down factor on tensor cores: the same conditions for the down units
   int rl_max_tiles = 0;        // most row-lane tiles and slots of any gate/up (h, e)
   int rl_max_slots = 0;
   std::vector<uint8_t> meta;   // host copy of header + descriptors + segment table
@@ -1501,15 +1502,20 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
   {   // gate/up factors (tensor cores, or the staged dp2a kernel over batches of 4 tokens), then down
     std::function<int()> between = ev ? std::function<int()>([&]() { return mark(3); }) : std::function<int()>();
     const int A_max = std::min(hd.E, p.P);
+    const bool tcd = tc && L->tcd;
     if (tcx) {
       BM_CK(launch_gu_tc(p, L->rl_max_tiles, L->rl_max_slots, st, pdl));
       if ((rc = mark(3))) return rc;
       between = std::function<int()>();
     }
-    const int parts = tcx ? 2 : 3;
-    if (G == 1) rc = launch_k2k3_dec<1, 4>(p, A_max, sms, st, pdl, between, parts);
-    else if (G == 2) rc = launch_k2k3_dec<2, 4>(p, A_max, sms, st, pdl, between, parts);
-    else rc = launch_k2k3_dec<4, 4>(p, A_max, sms, st, pdl, between, parts);
+    const int parts = (tcx ? 0 : 1) | (tcd ? 0 : 2);
+    if (parts) {
+      if (G == 1) rc = launch_k2k3_dec<1, 4>(p, A_max, sms, st, pdl, between, parts);
+      else if (G == 2) rc = launch_k2k3_dec<2, 4>(p, A_max, sms, st, pdl, between, parts);
+      else rc = launch_k2k3_dec<4, 4>(p, A_max, sms, st, pdl, between, parts);
+      if (rc) return rc;
+    }
+    if (tcd) BM_CK(launch_dn_tc(p, hd.ul_max_tiles, st, pdl));
   }
   if (rc) return rc;
   if ((rc = mark(4))) return rc;
@@ -1574,6 +1580,11 @@ int upload(std::vector<uint8_t>&& img, int device, bitsmoe_layer** out) {
       L->rl_max_slots = std::max(L->rl_max_slots, (int)xd[i].nslots);
     }
     L->tcx = ok16;
+    bool okd = h->group % kRows == 0;
+    for (int i = 2 * h->E; i < 3 * h->E; ++i)
+      for (int k = 0; k < xd[i].nbk; ++k)
+        if (xd[i].bk[k].bits >= 16) okd = false;
+    L->tcd = okd;
   }
   const ImageHeader* hd = header_of(img.data());
   const size_t meta_end = hd->off_basis_in;   // header + descriptors + segments
@@ -1723,7 +1734,7 @@ int bitsmoe_forward_plan(const bitsmoe_layer* L, int T, int top_k) {
   if (n == 1) return 1;
   const ImageHeader& hd = L->hd();
   if (T <= 8 && T * hd.E <= 4096) return 2;
-  return L->maps ? (L->tcx ? 4 | 8 : 4) : 0;
+  return L->maps ? 4 | (L->tcx ? 8 : 0) | (L->tcd ? 16 : 0) : 0;
 }
 
 int bitsmoe_block_forward_launches(const bitsmoe_layer* L, int T, int top_k) {

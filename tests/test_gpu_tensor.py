@@ -65,14 +65,15 @@ TC_BITS = {0: 0.1, 1: 0.15, 2: 0.2, 3: 0.15, 4: 0.15, 6: 0.15, 8: 0.1}
     (130, 4, 2, 96, 72, 512, 256),    # group of two row blocks
     (600, 4, 2, 64, 40, 256, 128),    # experts with more than 256 tokens: two token tiles
 ])
-def test_tensor_gate_up_factors(env, T, E, k, D, n, I, group):
-    """Gate/up factors on tcgen05 (codes decoded once per row block into bf16 tiles,
-    scale * alpha * z as a bf16 pair): every bit-width below 16."""
+def test_tensor_expert_factors(env, T, E, k, D, n, I, group):
+    """Gate/up and down factors on tcgen05 (codes decoded once into bf16 tiles; gate/up:
+    scale * alpha * z as a bf16 pair; down: h as a bf16 pair, group scales applied to the
+    per-group partial sums): every bit-width below 16."""
     torch, bm = env
     spec = synth.scaled_spec(synth.WORKLOADS["tiny"], D=D, E=E, I=I, n=n, group=group, top_k=k)
     layer = synth.make_layer(spec, seed=T + n, bits_dist=TC_BITS, alpha_scale=4.0)
     L = bm.bitsmoe_pack(layer, device=0)
-    assert bm.bitsmoe_forward_plan(L, T, k) == bm.PLAN_TC_PROJECTIONS | bm.PLAN_TC_GATE_UP
+    assert bm.bitsmoe_forward_plan(L, T, k) == bm.PLAN_TC_PROJECTIONS | bm.PLAN_TC_GATE_UP | bm.PLAN_TC_DOWN
     x, logits = synth.make_inputs(spec, T, seed=T)
     ws = bm.Workspace(L, T, k)
     y = bm.moe_forward(L, torch.from_numpy(x.view(np.int16)).cuda(), torch.from_numpy(logits).cuda(), k, ws=ws)
@@ -88,7 +89,7 @@ def test_tensor_path_qw3_dims_ragged_tokens(env):
     layer = synth.make_layer(spec, seed=72)
     L = bm.bitsmoe_pack(layer, device=0)
     T = 40
-    assert bm.bitsmoe_forward_plan(L, T, spec.top_k) == bm.PLAN_TC_PROJECTIONS | bm.PLAN_TC_GATE_UP
+    assert bm.bitsmoe_forward_plan(L, T, spec.top_k) == bm.PLAN_TC_PROJECTIONS | bm.PLAN_TC_GATE_UP | bm.PLAN_TC_DOWN
     x, logits = synth.make_inputs(spec, T, seed=72)
     y = bm.moe_forward(L, torch.from_numpy(x.view(np.int16)).cuda(), torch.from_numpy(logits).cuda(), spec.top_k)
     torch.cuda.synchronize()
