@@ -143,8 +143,8 @@ size_t bitsmoe_workspace_bytes(const bitsmoe_layer* layer, int T, int top_k);
  * (no counterpart in the paper: for callers that capture the forward into a
  * CUDA graph or count launches).  A single token runs as one fused persistent
  * kernel (1) when the layer's per-block shares of the bases and factors fit
- * in shared memory; otherwise the forward is a chain of 5 kernels.  Returns a negative error code for invalid
- * arguments. */
+ * in shared memory; otherwise the forward is a chain of 5 to 7 kernels (see
+ * bitsmoe_forward_plan).  Returns a negative error code for invalid arguments. */
 int bitsmoe_forward_launches(const bitsmoe_layer* layer, int T, int top_k);
 
 /* How a forward of T tokens runs on this layer, as a bit set:

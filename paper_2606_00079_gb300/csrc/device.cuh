@@ -42,6 +42,9 @@ struct Fwd {
   float* z;         // [2][T][n_pad]
   float* gu;        // [P][2][I_pad]
   float* s;         // [T][n_pad]
+  float* zT;        // [2][n_pad][T]: z again, token fastest (written for the tensor-core gate/up kernel)
+  int tc_gu_min;    // > 0: the tensor-core gate/up kernel takes the experts with at least this many
+  int tc_dn_min;    //      tokens and the dp2a kernel the rest (likewise for the down factor)
 };
 
 // Staging records of the fused single-token kernel, derived from the image
@@ -102,8 +105,8 @@ cudaError_t launch_fused(const Fwd& p, const FusedArgs& f, int sms, cudaStream_t
 // unless y carries a residual).
 bool make_basis_map(void* map_out, const void* base, int rows, int cols_pad);
 cudaError_t launch_gemm_tc(int mode, const void* map, const Fwd& p, int sms, cudaStream_t st, bool pdl,
-                           bool zt = false);
-// Tensor-core gate/up factors of every routed expert (z stored [2][n_pad][T]); the
+                           float* zT = nullptr);
+// Tensor-core gate/up factors of every routed expert (reads zT); the
 // layer's most row-lane tiles and slots of any gate/up (h, e) size the shared memory.
 cudaError_t launch_gu_tc(const Fwd& p, int max_tiles, int max_slots, cudaStream_t st, bool pdl);
 // Tensor-core down factor of every routed expert into s (zeroed before); ul_max_tiles:

@@ -21,8 +21,8 @@
 // B, and one thread issues the range's MMAs, whose commit frees A and B.  Each
 // (pair, h, row) is written by exactly one block: plain stores, no atomics.
 // Requires: every unit below 16 bits and the group a multiple of 128 rows (the
-// host checks the layer once at upload), and z stored [2][n_pad][T] (token
-// fastest, as the tensor-core projection writes it for this kernel).
+// host checks the layer once at upload), and zT = z stored [2][n_pad][T] (token
+// fastest, which the tensor-core projection writes for this kernel).
 #include <cuda_bf16.h>
 
 #include <algorithm>
@@ -141,7 +141,7 @@ __global__ void __launch_bounds__(kXThreads, 2) k_gu_tc(Fwd p, XArgs xa) {
   if (a >= p.active[0]) return;
   const int e = p.active[1 + a];
   const int ntok = p.expert_count[e], pst = p.expert_start[e];
-  if (ntok <= 0) return;
+  if (ntok <= 0 || ntok < p.tc_gu_min) return;   // fewer tokens: the dp2a kernel's expert
   const ExpertDesc& xd = p.desc[h * p.E + e];
   const int nslots = xd.nslots, nbk = xd.nbk;
   const int g = (rb * kRows) / p.group;
@@ -308,7 +308,7 @@ __global__ void __launch_bounds__(kXThreads, 2) k_gu_tc(Fwd p, XArgs xa) {
       // B: thread (token row t, 8-slot chunk c); a thread keeps one t over its items
       {
         const int t = tid & (NT - 1);
-        const float* zrow = p.z + (size_t)h * p.n_pad * p.T + (t < nt ? tok[t] : 0);
+        const float* zrow = p.zT + (size_t)h * p.n_pad * p.T + (t < nt ? tok[t] : 0);
         const uint32_t T32 = (uint32_t)p.T;
         float cs = 0.f;
         for (int item = tid; item < NT * (R / 8); item += kXThreads) {
@@ -488,7 +488,7 @@ __global__ void __launch_bounds__(kXThreads, 2) k_dn_tc(Fwd p, DArgs da) {
   const int ntok = p.expert_count[e], pst = p.expert_start[e];
   const ExpertDesc& xd = p.desc[2 * p.E + e];
   const int m0 = mt * 128;
-  if (ntok <= 0 || m0 >= xd.nslots) return;
+  if (ntok <= 0 || ntok < p.tc_dn_min || m0 >= xd.nslots) return;   // fewer tokens: the dp2a kernel's expert
   const int nslots = xd.nslots, nsl = min(128, nslots - m0), nq = nsl / 32;
   const int nt_need = min(da.NTmax, max(16, (ntok + 15) & ~15));
   int NT = 16;

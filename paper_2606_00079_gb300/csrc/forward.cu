@@ -781,7 +781,7 @@ __global__ void __launch_bounds__(kK2DecWarps * 32) k_gateup_dec(Fwd p) {
   const ExpertDesc& xd = p.desc[h * p.E + e];
   const ItemRec it = p.items[((size_t)h * p.E + e) * p.nseg + sg];
   const int ntok = p.expert_count[e], pst = p.expert_start[e];
-  if (it.nr == 0) {
+  if (it.nr == 0 || (p.tc_gu_min > 0 && ntok >= p.tc_gu_min)) {   // empty, or the tensor-core kernel's
     pdl_wait();
     return;
   }
@@ -1009,7 +1009,7 @@ __global__ void __launch_bounds__(kK3DecWarps * 32) k_down_dec(Fwd p) {
   const int r = item - a * ntg * nrc;
   const int tg = r / nrc, rc = r - tg * nrc;
   const ExpertDesc& xd = p.desc[2 * p.E + e];
-  if (tg * kK3DecWarps >= xd.ntiles) {
+  if (tg * kK3DecWarps >= xd.ntiles || (p.tc_dn_min > 0 && p.expert_count[e] >= p.tc_dn_min)) {
     pdl_wait();
     return;
   }
@@ -1171,7 +1171,7 @@ __global__ void __launch_bounds__(kK3DecWarps * 32) k_down_dec(Fwd p) {
 // host side
 // ---------------------------------------------------------------------------
 struct WsLayout {
-  size_t status, pair_expert, pair_weight, expert_count, expert_start, pair_list, active, z, gu, s;
+  size_t status, pair_expert, pair_weight, expert_count, expert_start, pair_list, active, z, gu, s, zt;
   size_t x_stage, logits_stage, y_stage;
   size_t sync;   // fused single-token kernel: grid-barrier counters
   size_t total;
@@ -1196,6 +1196,7 @@ WsLayout ws_layout(const ImageHeader& hd, int T, int k) {
   w.z = take(2 * (size_t)T * hd.n_pad * 4);
   w.gu = take(P * 2 * hd.I_pad * 4);
   w.s = take((size_t)T * hd.n_pad * 4);
+  w.zt = take(2 * (size_t)T * hd.n_pad * 4);   // z again, token fastest (tensor-core gate/up)
   w.x_stage = take((size_t)T * hd.D * 2);
   w.logits_stage = take((size_t)T * hd.E * 4);
   w.y_stage = take((size_t)T * hd.D * 4);
@@ -1380,6 +1381,11 @@ int num_sms_current(int* sms) {
 
 // norm != nullptr: a pre-norm block (y = h accumulates); x and logits are the workspace buffers that
 // the norm/router step fills, either as its own kernel or inside the one-token fused kernel.
+#ifndef BITSMOE_TC_MIN_TOKENS
+#define BITSMOE_TC_MIN_TOKENS 8
+#endif
+constexpr int kTcMinTokens = BITSMOE_TC_MIN_TOKENS;   // tokens from which an expert's factors use tensor cores
+
 int forward_impl(const void* x, const float* logits, int T, int top_k, const bitsmoe_layer* L, float* y,
                  void* ws, size_t ws_bytes, cudaStream_t st, cudaEvent_t* ev = nullptr, bool accum = false,
                  const NormArgs* norm = nullptr) {
@@ -1426,6 +1432,7 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
   p.z = reinterpret_cast<float*>(wb + w.z);
   p.gu = reinterpret_cast<float*>(wb + w.gu);
   p.s = reinterpret_cast<float*>(wb + w.s);
+  p.zT = reinterpret_cast<float*>(wb + w.zt);
   const int sms = L->num_sms;
   int rc;
   auto mark = [&](int i) -> int {
@@ -1491,10 +1498,13 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
   if (tc) {
     // the projection, the gate/up and the down kernels add into z, gu and s (adjacent in
     // the workspace); the output basis adds into y (which keeps the residual when accumulating)
-    BM_CK(cudaMemsetAsync(p.z, 0, (size_t)(reinterpret_cast<uint8_t*>(p.s) - reinterpret_cast<uint8_t*>(p.z)) +
-                                      (size_t)T * hd.n_pad * 4, st));
+    BM_CK(cudaMemsetAsync(p.z, 0,
+                          (size_t)((tcx ? reinterpret_cast<uint8_t*>(p.zT) : reinterpret_cast<uint8_t*>(p.s)) -
+                                   reinterpret_cast<uint8_t*>(p.z)) +
+                              (size_t)(tcx ? 2 : 1) * T * hd.n_pad * 4,
+                          st));
     if (!accum) BM_CK(cudaMemsetAsync(y, 0, (size_t)T * hd.D * 4, st));
-    BM_CK(launch_gemm_tc(0, L->map_in, p, sms, st, false, tcx));
+    BM_CK(launch_gemm_tc(0, L->map_in, p, sms, st, false, tcx ? p.zT : nullptr));
   } else if ((rc = launch_gemv_any(true, p, sms, st, pdl))) {
     return rc;
   }
@@ -1502,19 +1512,22 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
   {   // gate/up factors (tensor cores, or the staged dp2a kernel over batches of 4 tokens), then down
     std::function<int()> between = ev ? std::function<int()>([&]() { return mark(3); }) : std::function<int()>();
     const int A_max = std::min(hd.E, p.P);
+    // Experts with at least kTcMinTokens tokens go to the tensor-core kernels (their codes
+    // are decoded once for all tokens), the others to the dp2a kernels (whose cost follows
+    // the tokens): each kernel skips the other's experts.
     const bool tcd = tc && L->tcd;
-    if (tcx) {
-      BM_CK(launch_gu_tc(p, L->rl_max_tiles, L->rl_max_slots, st, pdl));
-      if ((rc = mark(3))) return rc;
-      between = std::function<int()>();
-    }
-    const int parts = (tcx ? 0 : 1) | (tcd ? 0 : 2);
-    if (parts) {
-      if (G == 1) rc = launch_k2k3_dec<1, 4>(p, A_max, sms, st, pdl, between, parts);
-      else if (G == 2) rc = launch_k2k3_dec<2, 4>(p, A_max, sms, st, pdl, between, parts);
-      else rc = launch_k2k3_dec<4, 4>(p, A_max, sms, st, pdl, between, parts);
-      if (rc) return rc;
-    }
+    p.tc_gu_min = tcx ? kTcMinTokens : 0;
+    p.tc_dn_min = tcd ? kTcMinTokens : 0;
+    if (G == 1) rc = launch_k2k3_dec<1, 4>(p, A_max, sms, st, pdl, std::function<int()>(), 1);
+    else if (G == 2) rc = launch_k2k3_dec<2, 4>(p, A_max, sms, st, pdl, std::function<int()>(), 1);
+    else rc = launch_k2k3_dec<4, 4>(p, A_max, sms, st, pdl, std::function<int()>(), 1);
+    if (rc) return rc;
+    if (tcx) BM_CK(launch_gu_tc(p, L->rl_max_tiles, L->rl_max_slots, st, pdl));
+    if (between && (rc = between())) return rc;
+    if (G == 1) rc = launch_k2k3_dec<1, 4>(p, A_max, sms, st, pdl, std::function<int()>(), 2);
+    else if (G == 2) rc = launch_k2k3_dec<2, 4>(p, A_max, sms, st, pdl, std::function<int()>(), 2);
+    else rc = launch_k2k3_dec<4, 4>(p, A_max, sms, st, pdl, std::function<int()>(), 2);
+    if (rc) return rc;
     if (tcd) BM_CK(launch_dn_tc(p, hd.ul_max_tiles, st, pdl));
   }
   if (rc) return rc;
@@ -1725,7 +1738,8 @@ int bitsmoe_forward_launches(const bitsmoe_layer* L, int T, int top_k) {
   FusedArgs fa;
   const int s16 = (int)align_up(std::max(hd.seg_max_slots, 8), 64) + 8;
   if (decode && fused_plan(hd, T, top_k, L->seg_bytes, L->ul_max_chunks, s16, L->num_sms, &fa)) return 1;
-  return 5;
+  if (decode || !L->maps) return 5;
+  return 3 + (L->tcx ? 2 : 1) + (L->tcd ? 2 : 1);   // router, projection, gate/up, down, output basis
 }
 
 int bitsmoe_forward_plan(const bitsmoe_layer* L, int T, int top_k) {

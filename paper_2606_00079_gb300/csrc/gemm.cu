@@ -53,8 +53,8 @@ struct GemmArgs {
   int D;             // mode 1: output row length
   const uint16_t* x; // mode 0: [T][D] bf16 bits
   const float* s;    // mode 1: [T][n_pad]
-  int zt;            // mode 0: z stored [2][n_pad][T] (token fastest) instead of [2][T][n_pad]
-  float* z;          // mode 0: zeroed before
+  float* z;          // mode 0: [2][T][n_pad], zeroed before
+  float* zT;         // mode 0: null, or [2][n_pad][T] (token fastest), zeroed before: also written
   float* y;          // mode 1: [T][D], zeroed before unless accumulating
   int* status;
 };
@@ -192,7 +192,8 @@ __global__ void __launch_bounds__(kGThreads, 1) k_gemm_tc(const __grid_constant_
           const float v = __uint_as_float(r[q]);
           if (g.mode == 0) {
             const int h = m >= g.n, j = m - h * g.n;
-            atomicAdd(g.z + (g.zt ? ((size_t)h * g.n_pad + j) * g.T + t : ((size_t)h * g.T + t) * g.n_pad + j), v);
+            atomicAdd(g.z + ((size_t)h * g.T + t) * g.n_pad + j, v);
+            if (g.zT) atomicAdd(g.zT + ((size_t)h * g.n_pad + j) * g.T + t, v);
           } else {
             atomicAdd(g.y + (size_t)t * g.D + m, v);
           }
@@ -246,7 +247,7 @@ bool make_basis_map(void* map_out, const void* base, int rows, int cols_pad) {
 
 // mode 0: z += Phi_{g,u}^T x for all T tokens; mode 1: y += Phi_dn s.  The
 // target must hold zeros (or the residual, for y) before the launch.
-cudaError_t launch_gemm_tc(int mode, const void* map, const Fwd& p, int sms, cudaStream_t st, bool pdl, bool zt) {
+cudaError_t launch_gemm_tc(int mode, const void* map, const Fwd& p, int sms, cudaStream_t st, bool pdl, float* zT) {
   static_assert(sizeof(CUtensorMap) == 128, "tensor map size");
   GemmArgs g;
   std::memset(&g, 0, sizeof(g));
@@ -264,7 +265,7 @@ cudaError_t launch_gemm_tc(int mode, const void* map, const Fwd& p, int sms, cud
   g.z = p.z;
   g.y = p.y;
   g.status = p.status;
-  g.zt = zt ? 1 : 0;
+  g.zT = zT;
   CUtensorMap amap;
   std::memcpy(&amap, map, sizeof(amap));
   static std::mutex mu;

@@ -47,7 +47,7 @@ def small_layer(env):
 def test_tensor_path_token_counts(env, small_layer, T):
     torch, bm = env
     spec, layer, L = small_layer
-    assert bm.bitsmoe_forward_launches(L, T, spec.top_k) == 5
+    assert bm.bitsmoe_forward_launches(L, T, spec.top_k) == 5   # 16-bit units: the dp2a expert kernels
     assert bm.bitsmoe_forward_plan(L, T, spec.top_k) == bm.PLAN_TC_PROJECTIONS   # 16-bit units: dp2a gate/up
     x, logits = synth.make_inputs(spec, T, seed=T)
     y = bm.moe_forward(L, torch.from_numpy(x.view(np.int16)).cuda(), torch.from_numpy(logits).cuda(), spec.top_k)
@@ -80,6 +80,22 @@ def test_tensor_expert_factors(env, T, E, k, D, n, I, group):
     torch.cuda.synchronize()
     assert bm.bitsmoe_last_device_status(ws.ptr) == 0
     ref = oracle.moe_forward_factored(layer, x, logits, k)
+    assert rel_err(y.cpu().numpy().astype(np.float64), ref) <= TOL
+
+
+def test_tensor_and_dp2a_experts_in_one_call(env):
+    """Experts with many tokens take the tensor-core factor kernels and the others the dp2a
+    kernels in the same call (a biased logit sends every token to expert 0)."""
+    torch, bm = env
+    spec = synth.scaled_spec(synth.WORKLOADS["tiny"], D=128, E=8, I=384, n=120, group=128, top_k=2)
+    layer = synth.make_layer(spec, seed=81, bits_dist=TC_BITS, alpha_scale=4.0)
+    L = bm.bitsmoe_pack(layer, device=0)
+    T = 24
+    x, logits = synth.make_inputs(spec, T, seed=81)
+    logits[:, 0] += 20.0
+    y = bm.moe_forward(L, torch.from_numpy(x.view(np.int16)).cuda(), torch.from_numpy(logits).cuda(), 2)
+    torch.cuda.synchronize()
+    ref = oracle.moe_forward_factored(layer, x, logits, 2)
     assert rel_err(y.cpu().numpy().astype(np.float64), ref) <= TOL
 
 
