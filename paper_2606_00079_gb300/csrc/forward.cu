@@ -1496,14 +1496,14 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
   const bool tc = L->maps;   // tensor-core projections for multi-token calls
   const bool tcx = tc && L->tcx;   // and tensor-core gate/up factors (z then stored token-fastest)
   if (tc) {
-    // the projection, the gate/up and the down kernels add into z, gu and s (adjacent in
-    // the workspace); the output basis adds into y (which keeps the residual when accumulating)
+    // the gate/up and down kernels add into gu and s (cleared here with z and zT, which lie
+    // next to them); the projection stores z (and zT), the output basis stores y (or adds
+    // into it, when it holds the residual)
     BM_CK(cudaMemsetAsync(p.z, 0,
                           (size_t)((tcx ? reinterpret_cast<uint8_t*>(p.zT) : reinterpret_cast<uint8_t*>(p.s)) -
                                    reinterpret_cast<uint8_t*>(p.z)) +
                               (size_t)(tcx ? 2 : 1) * T * hd.n_pad * 4,
                           st));
-    if (!accum) BM_CK(cudaMemsetAsync(y, 0, (size_t)T * hd.D * 4, st));
     BM_CK(launch_gemm_tc(0, L->map_in, p, sms, st, false, tcx ? p.zT : nullptr));
   } else if ((rc = launch_gemv_any(true, p, sms, st, pdl))) {
     return rc;
