@@ -43,6 +43,9 @@ struct Fwd {
   float* gu;        // [P][2][I_pad]
   float* s;         // [T][n_pad]
   float* zT;        // [2][n_pad][T]: z again, token fastest (written for the tensor-core gate/up kernel)
+  uint16_t* hh;     // [P][I_pad] bf16 hi of h = SiLU(gate) * up (pairs of the tensor-core down kernel)
+  uint16_t* hl;     // [P][I_pad] bf16 lo (the rounded remainder)
+  float* hsum;      // [P][NG] sums of h over each quantisation group (zeroed before)
   int tc_gu_min;    // > 0: the tensor-core gate/up kernel takes the experts with at least this many
   int tc_dn_min;    //      tokens and the dp2a kernel the rest (likewise for the down factor)
 };
@@ -112,6 +115,8 @@ cudaError_t launch_gu_tc(const Fwd& p, int max_tiles, int max_slots, cudaStream_
 // Tensor-core down factor of every routed expert into s (zeroed before); ul_max_tiles:
 // the layer's most unit-lane tiles of any expert.
 cudaError_t launch_dn_tc(const Fwd& p, int ul_max_tiles, cudaStream_t st, bool pdl);
+// h of the pairs of the tensor-core down kernel, as its bf16 pair and group sums.
+cudaError_t launch_h_pack(const Fwd& p, cudaStream_t st, bool pdl);
 // Staging records of a packed image (host side, at upload).
 void build_stage_tables(const uint8_t* img, std::vector<CStage>& cst, std::vector<DStage>& dst);
 

@@ -598,43 +598,24 @@ __global__ void __launch_bounds__(kXThreads, 2) k_dn_tc(Fwd p, DArgs da) {
           }
         }
       }
-      // B: thread (token row t, 8-row chunk c) with t fixed per thread; h = SiLU(gate) * up
+      // B: h = SiLU(gate) * up of the expert's pairs for this row block, as the bf16 pair
+      // prepared once per pair (k_h_pack): thread (token row t, 8-row chunk c), t fixed per thread
       {
         const int t = tid & (NT - 1);
         const bool live = t < nt;
-        const float* gp = p.gu + (size_t)pairs[t] * 2 * p.I_pad + (size_t)r * kRows;
-        float hsum = 0.f;
+        const size_t hrow = (size_t)pairs[t] * p.I_pad + (size_t)r * kRows;
         for (int item = tid; item < NT * 16; item += kXThreads) {
           const int c = item >> lgNT;
-          float hv[8];
+          uint4 hw = make_uint4(0, 0, 0, 0), lw = make_uint4(0, 0, 0, 0);
           if (live) {
-            const float4 g0 = __ldcg(reinterpret_cast<const float4*>(gp + 8 * c));
-            const float4 g1 = __ldcg(reinterpret_cast<const float4*>(gp + 8 * c + 4));
-            const float4 u0 = __ldcg(reinterpret_cast<const float4*>(gp + p.I_pad + 8 * c));
-            const float4 u1 = __ldcg(reinterpret_cast<const float4*>(gp + p.I_pad + 8 * c + 4));
-            const float gg[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
-            const float uu[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
-#pragma unroll
-            for (int u = 0; u < 8; ++u) hv[u] = gg[u] / (1.f + __expf(-gg[u])) * uu[u];
-          } else {
-#pragma unroll
-            for (int u = 0; u < 8; ++u) hv[u] = 0.f;
-          }
-          uint32_t hw[4], lw[4];
-#pragma unroll
-          for (int m2 = 0; m2 < 4; ++m2) {
-            const float v0 = hv[2 * m2], v1 = hv[2 * m2 + 1];
-            hsum += v0 + v1;
-            const uint32_t h0 = __float_as_uint(v0) & 0xFFFF0000u, h1 = __float_as_uint(v1) & 0xFFFF0000u;
-            hw[m2] = __byte_perm(h0, h1, 0x7632);
-            const __nv_bfloat162 bl = __floats2bfloat162_rn(v0 - __uint_as_float(h0), v1 - __uint_as_float(h1));
-            lw[m2] = *reinterpret_cast<const uint32_t*>(&bl);
+            hw = __ldcg(reinterpret_cast<const uint4*>(p.hh + hrow + 8 * c));
+            lw = __ldcg(reinterpret_cast<const uint4*>(p.hl + hrow + 8 * c));
           }
           const uint32_t off = (uint32_t)(c >> 3) * (uint32_t)NT * 128u + sw_off(t, c & 7);
-          *reinterpret_cast<uint4*>(sb + off) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-          *reinterpret_cast<uint4*>(sb + b_half + off) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+          *reinterpret_cast<uint4*>(sb + off) = hw;
+          *reinterpret_cast<uint4*>(sb + b_half + off) = lw;
         }
-        if (live && hsum != 0.f) atomicAdd(hs + (g & 1) * kDNT + t, hsum);
+        if (gfirst && tid < NT) hs[(g & 1) * kDNT + tid] = tid < nt ? __ldcg(p.hsum + (size_t)pairs[tid] * p.NG + g) : 0.f;
       }
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -675,8 +656,6 @@ __global__ void __launch_bounds__(kXThreads, 2) k_dn_tc(Fwd p, DArgs da) {
               for (int q = 0; q < 8; ++q) out[c0 + q] = fmaf(sc, __uint_as_float(rr[q]) - zp * hg[c0 + q], out[c0 + q]);
             }
           }
-        } else {   // the other warps clear the next group's sums
-          for (int t = tid - 128; t < kDNT; t += 128) hs[((g + 1) & 1) * kDNT + t] = 0.f;
         }
       }
     }
@@ -697,6 +676,46 @@ __global__ void __launch_bounds__(kXThreads, 2) k_dn_tc(Fwd p, DArgs da) {
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   if (wid == 1) tmem_dealloc(tmem, ncols);
+}
+
+// h = SiLU(gate) * up of every routed pair whose expert takes the tensor-core down
+// kernel, once: as the bf16 pair hi (truncation) + lo (rounded remainder) that the
+// down kernel's B operand needs, and its sums over each quantisation group.  Thread =
+// 8 consecutive rows of one pair; the threads of a group meet by warp shuffles.
+__global__ void __launch_bounds__(256) k_h_pack(Fwd p) {
+  pdl_trigger();
+  const int per_pair = p.I_pad / 8;
+  const size_t idx = (size_t)blockIdx.x * 256 + threadIdx.x;
+  pdl_wait();   // gate/up come from the previous kernels
+  if (idx >= (size_t)p.P * per_pair) return;   // whole 16-thread groups: I_pad / 8 is a multiple of 16
+  const int q = (int)(idx / per_pair), c = (int)(idx - (size_t)q * per_pair);
+  const int e = p.pair_expert[q];
+  if (p.expert_count[e] < p.tc_dn_min) return;   // the dp2a down kernel's expert (whole pair: 16-thread groups)
+  const float* gp = p.gu + (size_t)q * 2 * p.I_pad + 8 * c;
+  const float4 g0 = __ldcg(reinterpret_cast<const float4*>(gp)), g1 = __ldcg(reinterpret_cast<const float4*>(gp + 4));
+  const float4 u0 = __ldcg(reinterpret_cast<const float4*>(gp + p.I_pad));
+  const float4 u1 = __ldcg(reinterpret_cast<const float4*>(gp + p.I_pad + 4));
+  const float gg[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+  const float uu[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+  uint32_t hw[4], lw[4];
+  float sum = 0.f;
+#pragma unroll
+  for (int m = 0; m < 4; ++m) {
+    const float v0 = gg[2 * m] / (1.f + __expf(-gg[2 * m])) * uu[2 * m];
+    const float v1 = gg[2 * m + 1] / (1.f + __expf(-gg[2 * m + 1])) * uu[2 * m + 1];
+    sum += v0 + v1;
+    const uint32_t h0 = __float_as_uint(v0) & 0xFFFF0000u, h1 = __float_as_uint(v1) & 0xFFFF0000u;
+    hw[m] = __byte_perm(h0, h1, 0x7632);
+    const __nv_bfloat162 bl = __floats2bfloat162_rn(v0 - __uint_as_float(h0), v1 - __uint_as_float(h1));
+    lw[m] = *reinterpret_cast<const uint32_t*>(&bl);
+  }
+  *reinterpret_cast<uint4*>(p.hh + (size_t)q * p.I_pad + 8 * c) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+  *reinterpret_cast<uint4*>(p.hl + (size_t)q * p.I_pad + 8 * c) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+  // 16 consecutive threads cover one 128-row block of one pair; a group is one or more blocks
+  const unsigned gm = __activemask();
+#pragma unroll
+  for (int o = 8; o; o >>= 1) sum += __shfl_xor_sync(gm, sum, o);
+  if ((threadIdx.x & 15) == 0) atomicAdd(p.hsum + (size_t)q * p.NG + (8 * c) / p.group, sum);
 }
 
 }  // namespace
@@ -742,6 +761,20 @@ cudaError_t launch_gu_tc(const Fwd& p, int max_tiles, int max_slots, cudaStream_
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, k_gu_tc, p, xa);
+}
+
+cudaError_t launch_h_pack(const Fwd& p, cudaStream_t st, bool pdl) {
+  const size_t nth = (size_t)p.P * (p.I_pad / 8);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)((nth + 255) / 256));
+  cfg.blockDim = dim3(256);
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, k_h_pack, p);
 }
 
 cudaError_t launch_dn_tc(const Fwd& p, int ul_max_tiles, cudaStream_t st, bool pdl) {

@@ -1171,7 +1171,7 @@ __global__ void __launch_bounds__(kK3DecWarps * 32) k_down_dec(Fwd p) {
 // host side
 // ---------------------------------------------------------------------------
 struct WsLayout {
-  size_t status, pair_expert, pair_weight, expert_count, expert_start, pair_list, active, z, gu, s, zt;
+  size_t status, pair_expert, pair_weight, expert_count, expert_start, pair_list, active, z, gu, s, zt, hsum, hh, hl;
   size_t x_stage, logits_stage, y_stage;
   size_t sync;   // fused single-token kernel: grid-barrier counters
   size_t total;
@@ -1197,6 +1197,9 @@ WsLayout ws_layout(const ImageHeader& hd, int T, int k) {
   w.gu = take(P * 2 * hd.I_pad * 4);
   w.s = take((size_t)T * hd.n_pad * 4);
   w.zt = take(2 * (size_t)T * hd.n_pad * 4);   // z again, token fastest (tensor-core gate/up)
+  w.hsum = take(P * hd.NG * 4);                 // group sums of h (tensor-core down)
+  w.hh = take(P * hd.I_pad * 2);                // h as a bf16 pair (tensor-core down)
+  w.hl = take(P * hd.I_pad * 2);
   w.x_stage = take((size_t)T * hd.D * 2);
   w.logits_stage = take((size_t)T * hd.E * 4);
   w.y_stage = take((size_t)T * hd.D * 4);
@@ -1433,6 +1436,9 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
   p.gu = reinterpret_cast<float*>(wb + w.gu);
   p.s = reinterpret_cast<float*>(wb + w.s);
   p.zT = reinterpret_cast<float*>(wb + w.zt);
+  p.hsum = reinterpret_cast<float*>(wb + w.hsum);
+  p.hh = reinterpret_cast<uint16_t*>(wb + w.hh);
+  p.hl = reinterpret_cast<uint16_t*>(wb + w.hl);
   const int sms = L->num_sms;
   int rc;
   auto mark = [&](int i) -> int {
@@ -1500,9 +1506,8 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
     // next to them); the projection stores z (and zT), the output basis stores y (or adds
     // into it, when it holds the residual)
     BM_CK(cudaMemsetAsync(p.z, 0,
-                          (size_t)((tcx ? reinterpret_cast<uint8_t*>(p.zT) : reinterpret_cast<uint8_t*>(p.s)) -
-                                   reinterpret_cast<uint8_t*>(p.z)) +
-                              (size_t)(tcx ? 2 : 1) * T * hd.n_pad * 4,
+                          (size_t)(reinterpret_cast<uint8_t*>(p.hsum) - reinterpret_cast<uint8_t*>(p.z)) +
+                              (size_t)T * top_k * hd.NG * 4,
                           st));
     BM_CK(launch_gemm_tc(0, L->map_in, p, sms, st, false, tcx ? p.zT : nullptr));
   } else if ((rc = launch_gemv_any(true, p, sms, st, pdl))) {
@@ -1528,7 +1533,10 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
     else if (G == 2) rc = launch_k2k3_dec<2, 4>(p, A_max, sms, st, pdl, std::function<int()>(), 2);
     else rc = launch_k2k3_dec<4, 4>(p, A_max, sms, st, pdl, std::function<int()>(), 2);
     if (rc) return rc;
-    if (tcd) BM_CK(launch_dn_tc(p, hd.ul_max_tiles, st, pdl));
+    if (tcd) {
+      BM_CK(launch_h_pack(p, st, pdl));
+      BM_CK(launch_dn_tc(p, hd.ul_max_tiles, st, pdl));
+    }
   }
   if (rc) return rc;
   if ((rc = mark(4))) return rc;
@@ -1739,7 +1747,7 @@ int bitsmoe_forward_launches(const bitsmoe_layer* L, int T, int top_k) {
   const int s16 = (int)align_up(std::max(hd.seg_max_slots, 8), 64) + 8;
   if (decode && fused_plan(hd, T, top_k, L->seg_bytes, L->ul_max_chunks, s16, L->num_sms, &fa)) return 1;
   if (decode || !L->maps) return 5;
-  return 3 + (L->tcx ? 2 : 1) + (L->tcd ? 2 : 1);   // router, projection, gate/up, down, output basis
+  return 3 + (L->tcx ? 2 : 1) + (L->tcd ? 3 : 1);   // router, projection, gate/up, [h pack,] down, output basis
 }
 
 int bitsmoe_forward_plan(const bitsmoe_layer* L, int T, int top_k) {
