@@ -149,8 +149,10 @@ int bitsmoe_forward_launches(const bitsmoe_layer* layer, int T, int top_k);
 
 /* How a forward of T tokens runs on this layer, as a bit set:
  *   1  the fused single-token kernel
- *   2  the small-batch decode chain (2 <= T <= 8)
- *   4  tensor-core (tcgen05) shared-basis projections
+ *   2  the small-batch decode chain (2 <= T <= 8, or a single token whose
+ *      layer does not fit the fused kernel)
+ *   4  tensor-core (tcgen05) shared-basis projections (every T > 8; the decode
+ *      chain from 4 tokens)
  *   8  tensor-core gate/up factors (layers without 16-bit gate/up units whose
  *      group is a multiple of 128 rows; otherwise the dp2a kernel)
  *  16  tensor-core down factor (the same condition on the down units)

@@ -108,7 +108,7 @@ cudaError_t launch_fused(const Fwd& p, const FusedArgs& f, int sms, cudaStream_t
 // unless y carries a residual).
 bool make_basis_map(void* map_out, const void* base, int rows, int cols_pad);
 cudaError_t launch_gemm_tc(int mode, const void* map, const Fwd& p, int sms, cudaStream_t st, bool pdl,
-                           float* zT = nullptr);
+                           float* zT = nullptr, void* zero = nullptr, size_t zero_bytes = 0);
 // Tensor-core gate/up factors of every routed expert (reads zT); the
 // layer's most row-lane tiles and slots of any gate/up (h, e) size the shared memory.
 cudaError_t launch_gu_tc(const Fwd& p, int max_tiles, int max_slots, cudaStream_t st, bool pdl);

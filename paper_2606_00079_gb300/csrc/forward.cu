@@ -1384,6 +1384,15 @@ int num_sms_current(int* sms) {
 
 // norm != nullptr: a pre-norm block (y = h accumulates); x and logits are the workspace buffers that
 // the norm/router step fills, either as its own kernel or inside the one-token fused kernel.
+#ifndef BITSMOE_DECODE_MAX_TOKENS
+#define BITSMOE_DECODE_MAX_TOKENS 8
+#endif
+// Small batches run the decode chain (every kernel routes all tokens itself; the
+// single token also the fused kernel), larger ones the tensor-core chain.
+inline bool decode_mode(const ImageHeader& hd, int T) {
+  return T <= BITSMOE_DECODE_MAX_TOKENS && T * hd.E <= 4096;
+}
+
 #ifndef BITSMOE_TC_MIN_TOKENS
 #define BITSMOE_TC_MIN_TOKENS 8
 #endif
@@ -1412,7 +1421,7 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
   p.rbc = k3_rbc(hd);
   p.seg_bytes = L->seg_bytes;
   // decode mode: every kernel can afford the routing of all tokens
-  p.decode = T <= 8 && T * hd.E <= 4096;
+  p.decode = decode_mode(hd, T);
   {   // down staging: keep a warp's tile within ~48 KB of shared memory
     const int need = std::max(1, hd.group / kRows);
     int rbc = std::min(p.rbc, std::max(1, (48 * 1024) / (L->ul_max_chunks * kChunkBytes)));
@@ -1474,7 +1483,14 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
     if ((rc = set_smem(k_route_publish, rsm))) return rc;
     if ((rc = launch(k_route_publish, dim3(1), dim3(kThreads), rsm, st, false, p))) return rc;
     if ((rc = mark(1))) return rc;
-    if ((rc = launch_gemv_bulk(true, p, sms, st, pdl))) return rc;
+    const bool tcp = L->maps && T >= 4;   // below 4 tokens the bulk-copy GEMV streams the bases faster
+    if (tcp) {   // tensor-core projection; it also clears gate/up and s for the expert kernels
+      const size_t zb = (size_t)(reinterpret_cast<uint8_t*>(p.s) - reinterpret_cast<uint8_t*>(p.gu)) +
+                        (size_t)T * hd.n_pad * 4;
+      BM_CK(launch_gemm_tc(0, L->map_in, p, sms, st, pdl, nullptr, p.gu, zb));
+    } else if ((rc = launch_gemv_bulk(true, p, sms, st, pdl))) {
+      return rc;
+    }
     if ((rc = mark(2))) return rc;
     std::function<int()> between = ev ? std::function<int()>([&]() { return mark(3); }) : std::function<int()>();
     if (T == 1) {
@@ -1488,7 +1504,8 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
     }
     if (rc) return rc;
     if ((rc = mark(4))) return rc;
-    if ((rc = launch_gemv_bulk(false, p, sms, st, pdl))) return rc;
+    if (tcp) BM_CK(launch_gemm_tc(1, L->map_out, p, sms, st, pdl));
+    else if ((rc = launch_gemv_bulk(false, p, sms, st, pdl))) return rc;
     return mark(5);
   }
   const int tpb = std::max(1, 1024 / hd.E);
@@ -1742,7 +1759,7 @@ int bitsmoe_forward_launches(const bitsmoe_layer* L, int T, int top_k) {
   const ImageHeader& hd = L->hd();
   if (top_k < 1 || top_k > std::min(hd.E, 32)) return BITSMOE_ERR_INVALID_ARG;
   if (T == 0) return 0;
-  const bool decode = T <= 8 && T * hd.E <= 4096;
+  const bool decode = decode_mode(hd, T);
   FusedArgs fa;
   const int s16 = (int)align_up(std::max(hd.seg_max_slots, 8), 64) + 8;
   if (decode && fused_plan(hd, T, top_k, L->seg_bytes, L->ul_max_chunks, s16, L->num_sms, &fa)) return 1;
@@ -1755,7 +1772,7 @@ int bitsmoe_forward_plan(const bitsmoe_layer* L, int T, int top_k) {
   if (n <= 0) return n;
   if (n == 1) return 1;
   const ImageHeader& hd = L->hd();
-  if (T <= 8 && T * hd.E <= 4096) return 2;
+  if (decode_mode(hd, T)) return 2 | (L->maps && T >= 4 ? 4 : 0);
   return L->maps ? 4 | (L->tcx ? 8 : 0) | (L->tcd ? 16 : 0) : 0;
 }
 

@@ -60,6 +60,8 @@ struct GemmArgs {
   float* z;          // mode 0: [2][T][n_pad]
   float* zT;         // mode 0: null, or [2][n_pad][T] (token fastest): also written
   float* y;          // mode 1: [T][D]
+  float4* zero;      // null, or a buffer of later kernels to clear (after the PDL wait)
+  size_t zero_n;     // its length in float4
   int* status;
 };
 
@@ -141,6 +143,11 @@ __global__ void __launch_bounds__(kGThreads, 1) k_gemm_tc(const __grid_constant_
     // are converted and stored (and before the wait for a ring slot).
     pdl_wait();   // activations come from earlier kernels
     const int bt = tid - 64;   // 0 .. kStagers - 1
+    if (g.zero) {   // a buffer that the following kernels accumulate into
+      const size_t nthr = (size_t)gridDim.x * gridDim.y * kStagers;
+      for (size_t i = ((size_t)blockIdx.y * gridDim.x + blockIdx.x) * kStagers + bt; i < g.zero_n; i += nthr)
+        g.zero[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
     const int nch = g.N * 8;
     auto load4 = [&](int i, int c0, float4 (&v)[4][2]) {
       const int kbase = (kb0 + i) * kKB;
@@ -335,7 +342,8 @@ bool make_basis_map(void* map_out, const void* base, int rows, int cols_pad) {
 
 // mode 0: z = Phi_{g,u}^T x (and zT, when given) for all T tokens; mode 1:
 // y = Phi_dn s, or y += Phi_dn s when p.accum.  Plain stores: nothing to clear.
-cudaError_t launch_gemm_tc(int mode, const void* map, const Fwd& p, int sms, cudaStream_t st, bool pdl, float* zT) {
+cudaError_t launch_gemm_tc(int mode, const void* map, const Fwd& p, int sms, cudaStream_t st, bool pdl, float* zT,
+                           void* zero, size_t zero_bytes) {
   static_assert(sizeof(CUtensorMap) == 128, "tensor map size");
   GemmArgs g;
   std::memset(&g, 0, sizeof(g));
@@ -353,6 +361,8 @@ cudaError_t launch_gemm_tc(int mode, const void* map, const Fwd& p, int sms, cud
   g.s = p.s;
   g.z = p.z;
   g.zT = zT;
+  g.zero = static_cast<float4*>(zero);
+  g.zero_n = zero_bytes / 16;
   g.y = p.y;
   g.status = p.status;
   CUtensorMap amap;

@@ -92,10 +92,15 @@ def test_all_bit_widths_groups_and_token_batches(env, group, I, T):
 
 @pytest.mark.parametrize("b", [1, 2, 3, 4, 6, 8, 16])
 def test_uniform_bit_width(env, b):
+    """Five tokens: the decode chain with the tensor-core projections."""
+    torch, bm = env
     spec = small(n=70)
     layer = synth.make_layer(spec, seed=b, bits_dist={b: 1.0}, alpha_scale=3.0)
+    L = bm.bitsmoe_pack(layer, device=0)
+    assert bm.bitsmoe_forward_plan(L, 5, spec.top_k) == bm.PLAN_DECODE_CHAIN | bm.PLAN_TC_PROJECTIONS
+    assert bm.bitsmoe_forward_plan(L, 3, spec.top_k) == bm.PLAN_DECODE_CHAIN
     x, logits = synth.make_inputs(spec, 5, seed=b)
-    check(env, layer, x, logits, spec.top_k)
+    check(env, layer, x, logits, spec.top_k, L=L)
 
 
 def set_unit(layer, h, e, j, b, rng):
