@@ -188,7 +188,10 @@ int bitsmoe_moe_forward(const void* x, const float* logits, int T, int top_k,
 /* Same forward from host buffers: copies x (T x D bf16) and logits (T x E fp32)
  * from host memory into the workspace, runs the forward, copies y (T x D fp32)
  * back to host memory and synchronises `stream`.  Pinned host memory gives
- * asynchronous copies; pageable memory works but is slower. */
+ * asynchronous copies; pageable memory works but is slower.  A single token
+ * on the fused kernel with all three buffers pinned (device-mapped, 16-byte
+ * aligned) skips the copies: the kernel reads x and the logits from, and
+ * writes y to, the host buffers directly. */
 int bitsmoe_moe_forward_host(const void* x_host, const float* logits_host, int T, int top_k,
                              const bitsmoe_layer* layer, float* y_host,
                              void* ws, size_t ws_bytes, void* stream);

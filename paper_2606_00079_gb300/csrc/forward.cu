@@ -1348,6 +1348,18 @@ int launch_k2k3_dec(const Fwd& p, int A_max, int sms, cudaStream_t st, bool pdl,
 
 bool aligned(const void* ptr, size_t a) { return ((uintptr_t)ptr % a) == 0; }
 
+// The device address of pinned, device-mapped host memory (null for anything else or when
+// not aligned to `a` bytes).
+const void* mapped_host(const void* p, size_t a) {
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  if (at.type != cudaMemoryTypeHost || !at.devicePointer || !aligned(at.devicePointer, a)) return nullptr;
+  return at.devicePointer;
+}
+
 template <int TB>
 int launch_norm_router_tb(const NormArgs& a, int sms, cudaStream_t st) {
   const size_t smem = (size_t)TB * a.D_pad8 * 4 + kWarps * TB * 4;
@@ -1816,6 +1828,20 @@ int bitsmoe_moe_forward_host(const void* x_host, const float* logits_host, int T
   if (rc) return rc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   uint8_t* wb = static_cast<uint8_t*>(ws);
+  if (T == 1 && bitsmoe_forward_launches(L, T, top_k) == 1) {
+    // One token on the fused kernel with pinned (device-mapped) host buffers: the kernel reads x
+    // and the logits and writes y through the unified address space (the bytes cross the
+    // host link inside the kernel), which saves the copy round trips of a few KB.
+    const void* xd = mapped_host(x_host, 16);
+    const void* ld = mapped_host(logits_host, 16);
+    void* yd = const_cast<void*>(mapped_host(y_host, 16));
+    if (xd && ld && yd) {
+      rc = forward_impl(xd, static_cast<const float*>(ld), T, top_k, L, static_cast<float*>(yd), ws, ws_bytes, st);
+      if (rc) return rc;
+      BM_CK(cudaStreamSynchronize(st));
+      return BITSMOE_OK;
+    }
+  }
   BM_CK(cudaMemcpyAsync(wb + w.x_stage, x_host, (size_t)T * hd.D * 2, cudaMemcpyHostToDevice, st));
   BM_CK(cudaMemcpyAsync(wb + w.logits_stage, logits_host, (size_t)T * hd.E * 4, cudaMemcpyHostToDevice, st));
   rc = forward_impl(wb + w.x_stage, reinterpret_cast<const float*>(wb + w.logits_stage), T, top_k, L,

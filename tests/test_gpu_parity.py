@@ -162,6 +162,33 @@ def test_host_buffer_entry_point_matches(env):
     assert bm.bitsmoe_last_device_status(ws.ptr, 0) == 0
 
 
+def test_host_buffer_single_token_pinned_and_pageable(env):
+    """One token on the fused kernel through the host-buffer entry point: pinned buffers are
+    read and written by the kernel in place, pageable ones are copied; both match."""
+    torch, bm = env
+    spec = small()
+    layer = synth.make_layer(spec, seed=12, alpha_scale=3.0)
+    L = bm.bitsmoe_pack(layer, device=0)
+    assert bm.bitsmoe_forward_launches(L, 1, spec.top_k) == 1
+    ws = bm.Workspace(L, 1, spec.top_k)
+    st = torch.cuda.current_stream().cuda_stream
+    for step in range(3):
+        x, logits = synth.make_inputs(spec, 1, seed=12, step=step)
+        ref = oracle.moe_forward_factored(layer, x, logits, spec.top_k)
+        y_page = bm.bitsmoe_moe_forward_host(x, logits, spec.top_k, L, ws.ptr, ws.nbytes, st)
+        xp = torch.from_numpy(x.view(np.int16)).pin_memory()
+        lp = torch.from_numpy(logits).pin_memory()
+        yp = torch.full((1, spec.D), float("nan"), dtype=torch.float32).pin_memory()
+        rc = bm._lib().bitsmoe_moe_forward_host(xp.data_ptr(), lp.data_ptr(), 1, spec.top_k, L.handle,
+                                                yp.data_ptr(), ws.ptr, ws.nbytes, st)
+        assert rc == 0
+        y_pin = yp.numpy().astype(np.float64)
+        assert rel_err(y_page.astype(np.float64), ref) <= TOL
+        assert rel_err(y_pin, ref) <= TOL
+        assert rel_err(y_pin, y_page.astype(np.float64)) <= 1e-5
+    assert bm.bitsmoe_last_device_status(ws.ptr, 0) == 0
+
+
 def test_blob_upload_and_device_unpack_roundtrip(env):
     torch, bm = env
     spec = small()
