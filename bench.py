@@ -81,6 +81,29 @@ def dist_env():
     return rank, world, local
 
 
+def rank_barrier(world):
+    """All ranks meet here (N > 1) before and after the timed region."""
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(ms, world, device):
+    """The slowest rank's time: the job's time for the units all ranks processed."""
+    if world <= 1:
+        return float(ms)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(world, steps, tokens, ms):
+    """Whole-job tokens/s: every rank processed steps x tokens in the slowest rank's time."""
+    return world * steps * tokens / (ms / 1e3)
+
+
 def host_route(logits, k):
     """Experts each token is routed to (k largest logits, ties to the lower index):
     used only to count the algorithmic bytes of a step."""
@@ -288,8 +311,7 @@ def run_stack(args, spec, T, torch, bm, dev, rank, world, local):
     stream.synchronize()
     clk = ClockSampler(local)
     clk.start()
-    if world > 1:
-        torch.distributed.barrier()
+    rank_barrier(world)
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     clk.mark("t0")
@@ -303,13 +325,10 @@ def run_stack(args, spec, T, torch, bm, dev, rank, world, local):
     e1.synchronize()
     clk.mark("t1")
     torch.cuda.synchronize()
-    ms = e0.elapsed_time(e1)
+    rank_barrier(world)
+    ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
     clocks = clk.stop()
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
-    value = world * args.steps * T / (ms / 1e3)
+    value = job_throughput(world, args.steps, T, ms)
     gbs = step_bytes * args.steps / (ms / 1e3) / 1e9
     peaks, peak_src = measured_peaks()
     peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
@@ -438,8 +457,7 @@ def main():
 
     clk = ClockSampler(local)
     clk.start()
-    if world > 1:
-        torch.distributed.barrier()
+    rank_barrier(world)
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     clk.mark("t0")
@@ -453,14 +471,11 @@ def main():
     e1.synchronize()
     clk.mark("t1")
     torch.cuda.synchronize()
-    ms = e0.elapsed_time(e1)
+    rank_barrier(world)
+    ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
     clocks = clk.stop()
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
     total_bytes = sum(step_bytes(i) for i in range(args.steps))
-    value = world * args.steps * T / (ms / 1e3)
+    value = job_throughput(world, args.steps, T, ms)
     fwd_gbs = total_bytes / (ms / 1e3) / 1e9
 
     # ---- roofline of the dominant kernel
