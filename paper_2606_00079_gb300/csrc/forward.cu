@@ -1274,7 +1274,10 @@ int launch_gemv_bulk_tb(bool proj, const Fwd& p, int sms, cudaStream_t st, bool 
   const int nrows = proj ? 2 * p.n : p.D;
   const size_t row_bytes = (size_t)ld * 2;
   const size_t vec = (size_t)TB * ld * 4;
-  const size_t budget = proj ? 64 * 1024 : (vec < 150 * 1024 ? 200 * 1024 - vec : 48 * 1024);
+#ifndef BITSMOE_GEMV_PROJ_KB
+#define BITSMOE_GEMV_PROJ_KB 128   // shared memory of the projection GEMV's two-stage ring (bytes in flight per SM)
+#endif
+  const size_t budget = proj ? BITSMOE_GEMV_PROJ_KB * 1024 : (vec < 150 * 1024 ? 200 * 1024 - vec : 48 * 1024);
   const int grid = std::min(nrows, sms);
   const int per = (nrows + grid - 1) / grid;
   int stage_rows = (int)std::max<size_t>(1, std::min<size_t>((budget / 2) / row_bytes, (size_t)(per + 1) / 2));
