@@ -143,14 +143,15 @@ size_t bitsmoe_workspace_bytes(const bitsmoe_layer* layer, int T, int top_k);
  * (no counterpart in the paper: for callers that capture the forward into a
  * CUDA graph or count launches).  A single token runs as one fused persistent
  * kernel (1) when the layer's per-block shares of the bases and factors fit
- * in shared memory; otherwise the forward is a chain of 5 to 7 kernels (see
+ * in shared memory, and up to 4 tokens as one such kernel per token (T);
+ * otherwise the forward is a chain of 5 to 8 kernels (see
  * bitsmoe_forward_plan).  Returns a negative error code for invalid arguments. */
 int bitsmoe_forward_launches(const bitsmoe_layer* layer, int T, int top_k);
 
 /* How a forward of T tokens runs on this layer, as a bit set:
- *   1  the fused single-token kernel
- *   2  the small-batch decode chain (2 <= T <= 8, or a single token whose
- *      layer does not fit the fused kernel)
+ *   1  the fused single-token kernel (once per token for up to 4 tokens)
+ *   2  the small-batch decode chain (T <= 8 on a layer that does not fit the
+ *      fused kernel, else 5 <= T <= 8)
  *   4  tensor-core (tcgen05) shared-basis projections (every T > 8; the decode
  *      chain from 4 tokens)
  *   8  tensor-core gate/up factors (layers without 16-bit gate/up units whose
@@ -159,8 +160,8 @@ int bitsmoe_forward_launches(const bitsmoe_layer* layer, int T, int top_k);
  * Returns a negative error code for invalid arguments; 0 for T == 0. */
 int bitsmoe_forward_plan(const bitsmoe_layer* layer, int T, int top_k);
 
-/* Kernels one bitsmoe_moe_block_forward call launches: 1 when the fused
- * single-token kernel runs (it computes the pre-norm and router too),
+/* Kernels one bitsmoe_moe_block_forward call launches: 1 a token when the
+ * fused single-token kernel runs (it computes the pre-norm and router too),
  * otherwise the norm/router kernel plus bitsmoe_forward_launches. */
 int bitsmoe_block_forward_launches(const bitsmoe_layer* layer, int T, int top_k);
 
@@ -226,8 +227,8 @@ int bitsmoe_moe_block_forward(float* h, const void* w_router, float eps, int T, 
  * and the call synchronises.  phase_ms[0..4] receive the durations of
  * routing, shared-basis projection (gate, up), gate/up factors + SwiGLU
  * inputs, down factor + weighted expert sum, output basis.  When the forward
- * runs as one fused kernel (see bitsmoe_forward_launches), its phases cannot
- * be separated: phase_ms[0] receives the whole forward and the others 0. */
+ * runs as fused kernels (see bitsmoe_forward_plan), its phases cannot be
+ * separated: phase_ms[0] receives the whole forward and the others 0. */
 int bitsmoe_profile_forward(const void* x, const float* logits, int T, int top_k,
                             const bitsmoe_layer* layer, float* y,
                             void* ws, size_t ws_bytes, void* stream, float phase_ms[5]);

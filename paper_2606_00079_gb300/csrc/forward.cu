@@ -1413,10 +1413,40 @@ inline bool decode_mode(const ImageHeader& hd, int T) {
 #endif
 constexpr int kTcMinTokens = BITSMOE_TC_MIN_TOKENS;   // tokens from which an expert's factors use tensor cores
 
+// Up to this many tokens run as one fused single-token forward per token when the layer
+// fits the fused kernel (T fused forwards beat the decode chain there).
+constexpr int kFusedMaxTokens = 4;
+
+bool fused_fits(const bitsmoe_layer* L, int top_k) {
+  const ImageHeader& hd = L->hd();
+  FusedArgs fa;
+  const int s16 = (int)align_up(std::max(hd.seg_max_slots, 8), 64) + 8;
+  return decode_mode(hd, 1) && fused_plan(hd, 1, top_k, L->seg_bytes, L->ul_max_chunks, s16, L->num_sms, &fa);
+}
+
 int forward_impl(const void* x, const float* logits, int T, int top_k, const bitsmoe_layer* L, float* y,
                  void* ws, size_t ws_bytes, cudaStream_t st, cudaEvent_t* ev = nullptr, bool accum = false,
                  const NormArgs* norm = nullptr) {
   const ImageHeader& hd = L->hd();
+  if (T > 1 && T <= kFusedMaxTokens && fused_fits(L, top_k)) {
+    // a few tokens: one fused forward each, on the same workspace (profiled as one phase)
+    if (ev) BM_CK(cudaEventRecord(ev[0], st));
+    for (int t = 0; t < T; ++t) {
+      NormArgs nt;
+      if (norm) {
+        nt = *norm;
+        nt.h = norm->h + (size_t)t * hd.D;
+        nt.T = 1;
+      }
+      const int rc = forward_impl(static_cast<const uint16_t*>(x) + (size_t)t * hd.D, logits + (size_t)t * hd.E, 1,
+                                  top_k, L, y + (size_t)t * hd.D, ws, ws_bytes, st, nullptr, accum,
+                                  norm ? &nt : nullptr);
+      if (rc) return rc;
+    }
+    if (ev)
+      for (int i = 1; i <= 5; ++i) BM_CK(cudaEventRecord(ev[i], st));
+    return BITSMOE_OK;
+  }
   const bool pdl = ev == nullptr;   // profiling runs the phases back to back without overlap
   const WsLayout w = ws_layout(hd, T, top_k);
   uint8_t* wb = static_cast<uint8_t*>(ws);
@@ -1778,6 +1808,7 @@ int bitsmoe_forward_launches(const bitsmoe_layer* L, int T, int top_k) {
   FusedArgs fa;
   const int s16 = (int)align_up(std::max(hd.seg_max_slots, 8), 64) + 8;
   if (decode && fused_plan(hd, T, top_k, L->seg_bytes, L->ul_max_chunks, s16, L->num_sms, &fa)) return 1;
+  if (T <= kFusedMaxTokens && fused_fits(L, top_k)) return T;   // one fused forward per token
   if (decode || !L->maps) return 5;
   return 3 + (L->tcx ? 2 : 1) + (L->tcd ? 3 : 1);   // router, projection, gate/up, [h pack,] down, output basis
 }
@@ -1785,7 +1816,7 @@ int bitsmoe_forward_launches(const bitsmoe_layer* L, int T, int top_k) {
 int bitsmoe_forward_plan(const bitsmoe_layer* L, int T, int top_k) {
   const int n = bitsmoe_forward_launches(L, T, top_k);
   if (n <= 0) return n;
-  if (n == 1) return 1;
+  if (T <= kFusedMaxTokens && fused_fits(L, top_k)) return 1;
   const ImageHeader& hd = L->hd();
   if (decode_mode(hd, T)) return 2 | (L->maps && T >= 4 ? 4 : 0);
   return L->maps ? 4 | (L->tcx ? 8 : 0) | (L->tcd ? 16 : 0) : 0;
@@ -1793,6 +1824,7 @@ int bitsmoe_forward_plan(const bitsmoe_layer* L, int T, int top_k) {
 
 int bitsmoe_block_forward_launches(const bitsmoe_layer* L, int T, int top_k) {
   const int n = bitsmoe_forward_launches(L, T, top_k);
+  if (n > 0 && T <= kFusedMaxTokens && fused_fits(L, top_k)) return n;   // the fused kernels norm in place
   return n > 1 ? n + 1 : n;
 }
 

@@ -660,9 +660,11 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
   const int md = ndi > blk ? (ndi - blk + nb - 1) / nb : 0;   // this block's: i = blk + m * nb
   if (wid < kBW) {
     // ---- x into shared memory (unless the block normalised h itself), zero gate/up and s
+    // a token row inside a batch starts at 2*D*t bytes: 16-byte loads only when x is 16-byte aligned
+    const bool x16 = (reinterpret_cast<uintptr_t>(p.x) & 15) == 0;
     for (int i = tid; i < (f.norm ? 0 : p.D_pad / 8); i += kBW * 32) {
       uint4 v = make_uint4(0, 0, 0, 0);
-      if (8 * i + 8 <= p.D) {
+      if (x16 && 8 * i + 8 <= p.D) {
         v = *reinterpret_cast<const uint4*>(p.x + 8 * i);
       } else {
         uint16_t t[8];

@@ -186,7 +186,8 @@ def test_fused_plan_taken_for_qw3_dims_not_for_d4096(env):
     qw3 = synth.scaled_spec(synth.WORKLOADS["qw3"], E=8, top_k=8)   # full qw3 dims, fewer experts
     L = bm.bitsmoe_pack(synth.make_layer(qw3, seed=1), device=0)
     assert bm.bitsmoe_forward_launches(L, 1, 8) == 1
-    assert bm.bitsmoe_forward_launches(L, 2, 8) == 5
+    assert bm.bitsmoe_forward_launches(L, 2, 8) == 2   # one fused forward per token
+    assert bm.bitsmoe_forward_launches(L, 5, 8) == 5
     # D = n = 4096: a block's share of the input bases (54 rows of 8 KB) exceeds shared memory
     big = synth.scaled_spec(synth.WORKLOADS["mixtral"], E=2, I=128, top_k=1)
     Lb = bm.bitsmoe_pack(synth.make_layer(big, seed=1), device=0)
@@ -205,7 +206,8 @@ def test_block_forward_fused_norm(env, E, top_k):
     layer = synth.make_layer(spec, seed=5)
     L = bm.bitsmoe_pack(layer, device=0)
     assert bm.bitsmoe_block_forward_launches(L, 1, top_k) == 1
-    assert bm.bitsmoe_block_forward_launches(L, 2, top_k) == bm.bitsmoe_forward_launches(L, 2, top_k) + 1
+    assert bm.bitsmoe_block_forward_launches(L, 2, top_k) == 2
+    assert bm.bitsmoe_block_forward_launches(L, 5, top_k) == bm.bitsmoe_forward_launches(L, 5, top_k) + 1
     wr = torch.from_numpy(synth.make_router_weight(spec, seed=5).view(np.int16)).cuda()
     h0 = torch.from_numpy(synth.make_hidden(spec, 1, seed=5)).cuda() * 3.0
     eps, st = 1e-6, torch.cuda.current_stream().cuda_stream
@@ -227,3 +229,38 @@ def test_block_forward_fused_norm(env, E, top_k):
     xo = x.cpu().numpy().view(np.uint16)
     ref = oracle.moe_forward_factored(layer, xo, lg.cpu().numpy().astype(np.float64), top_k)
     assert rel_err(upd, ref) <= TOL
+
+
+@pytest.mark.parametrize("T", [2, 3, 4])
+def test_few_tokens_as_fused_forwards(env, T):
+    """Two to four tokens run as one fused forward per token on one workspace: plain and
+    as a pre-norm block (norm mode), against the oracle and the two-step path."""
+    torch, bm = env
+    spec = small(E=8, top_k=3, n=72)
+    layer = synth.make_layer(spec, seed=30 + T, alpha_scale=3.0)
+    L = bm.bitsmoe_pack(layer, device=0)
+    assert bm.bitsmoe_forward_launches(L, T, spec.top_k) == T
+    assert bm.bitsmoe_forward_plan(L, T, spec.top_k) == bm.PLAN_FUSED
+    x, logits = synth.make_inputs(spec, T, seed=30 + T)
+    ws = bm.Workspace(L, T, spec.top_k)
+    y = bm.moe_forward(L, torch.from_numpy(x.view(np.int16)).cuda(), torch.from_numpy(logits).cuda(), spec.top_k,
+                       ws=ws)
+    torch.cuda.synchronize()
+    assert bm.bitsmoe_last_device_status(ws.ptr) == 0
+    ref = oracle.moe_forward_factored(layer, x, logits, spec.top_k)
+    assert rel_err(y.cpu().numpy().astype(np.float64), ref) <= TOL
+    # pre-norm block: h += MoE(RMSNorm(h)) token by token in the fused kernels
+    wr = torch.from_numpy(synth.make_router_weight(spec, seed=30 + T).view(np.int16)).cuda()
+    h0 = torch.from_numpy(synth.make_hidden(spec, T, seed=30 + T)).cuda()
+    st = torch.cuda.current_stream().cuda_stream
+    xb = torch.empty((T, spec.D), dtype=torch.int16, device="cuda")
+    lg = torch.empty((T, spec.E), dtype=torch.float32, device="cuda")
+    bm.bitsmoe_rmsnorm_router(h0.data_ptr(), wr.data_ptr(), 1e-6, T, spec.D, spec.E, xb.data_ptr(), lg.data_ptr(), st)
+    y2 = bm.moe_forward(L, xb, lg, spec.top_k, ws=ws)
+    h = h0.clone()
+    bm.bitsmoe_moe_block_forward(h.data_ptr(), wr.data_ptr(), 1e-6, T, spec.top_k, L, ws.ptr, ws.nbytes, st)
+    torch.cuda.synchronize()
+    assert bm.bitsmoe_last_device_status(ws.ptr) == 0
+    two_step = (h0 + y2).cpu().numpy().astype(np.float64)
+    ymax, hmax = float(y2.abs().max()), float(h0.abs().max())
+    assert np.max(np.abs(h.cpu().numpy() - two_step)) <= 1e-5 * ymax + 2.4e-7 * hmax

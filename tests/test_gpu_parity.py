@@ -98,7 +98,7 @@ def test_uniform_bit_width(env, b):
     layer = synth.make_layer(spec, seed=b, bits_dist={b: 1.0}, alpha_scale=3.0)
     L = bm.bitsmoe_pack(layer, device=0)
     assert bm.bitsmoe_forward_plan(L, 5, spec.top_k) == bm.PLAN_DECODE_CHAIN | bm.PLAN_TC_PROJECTIONS
-    assert bm.bitsmoe_forward_plan(L, 3, spec.top_k) == bm.PLAN_DECODE_CHAIN
+    assert bm.bitsmoe_forward_plan(L, 3, spec.top_k) == bm.PLAN_FUSED   # one fused forward per token
     x, logits = synth.make_inputs(spec, 5, seed=b)
     check(env, layer, x, logits, spec.top_k, L=L)
 
@@ -274,3 +274,16 @@ def test_mixtral_shape(env):
     for T in spec.tokens:
         x, logits = synth.make_inputs(spec, T, seed=0)
         check(env, layer, x, logits, spec.top_k, L=L)
+
+
+@pytest.mark.parametrize("T", [1, 2, 3])
+def test_decode_chain_without_fused_plan(env, T):
+    """A layer whose per-block shares do not fit the fused kernel (D = n = 4096): one to
+    three tokens take the decode chain with the bulk-copy GEMV projections."""
+    torch, bm = env
+    spec = synth.scaled_spec(synth.WORKLOADS["mixtral"], E=3, I=256, top_k=2)
+    layer = synth.make_layer(spec, seed=40 + T)
+    L = bm.bitsmoe_pack(layer, device=0)
+    assert bm.bitsmoe_forward_plan(L, T, spec.top_k) == bm.PLAN_DECODE_CHAIN
+    x, logits = synth.make_inputs(spec, T, seed=40 + T)
+    check(env, layer, x, logits, spec.top_k, L=L)
