@@ -253,3 +253,25 @@ def permute_units(layer: Dict[str, np.ndarray], perm: Sequence[int]) -> Dict[str
     for k in ("bits", "alpha", "codes", "scale", "zero"):
         out[k] = np.ascontiguousarray(layer[k][:, :, perm])
     return out
+
+
+def make_float_units(U: int, I: int, seed: int = 0, bits_dist: Optional[Dict[int, float]] = None,
+                     zero_groups: int = 0, group: int = 128) -> Tuple[np.ndarray, np.ndarray]:
+    """Unquantised spectral units for the quantiser: U unit-norm Gaussian directions of
+    length I (fp32, one per row, like the normalised spectral vectors of the method)
+    and a bit-width per unit drawn i.i.d. from `bits_dist` (default: mean 2.0 bits).
+    `zero_groups` groups of `group` elements are set to zero (edge cases)."""
+    rng = np.random.default_rng([seed, 43, U, I])
+    p = rng.standard_normal((U, I))
+    p /= np.maximum(np.linalg.norm(p, axis=1, keepdims=True), 1e-300)
+    p = p.astype(np.float32)
+    if zero_groups and U and I >= group:
+        ng = I // group
+        for _ in range(zero_groups):
+            u, g = int(rng.integers(U)), int(rng.integers(ng))
+            p[u, g * group:(g + 1) * group] = 0.0
+    dist = _dist(bits_dist if bits_dist is not None else DIST_MEAN_2_0)
+    vals = np.array([b for b, _ in dist], dtype=np.uint8)
+    probs = np.array([q for _, q in dist], dtype=np.float64)
+    bits = vals[rng.choice(len(vals), size=U, p=probs / probs.sum())]
+    return p, bits
