@@ -362,10 +362,143 @@ def run_stack(args, spec, T, torch, bm, dev, rank, world, local):
         print(json.dumps(line), flush=True)
 
 
+QUANT_METRIC = "spectral units quantised/s (per-unit Q_b into the stored format, MSE-optimal group scales)"
+# lane-instructions of the definition per (element, candidate) of the scale search: quotient as a
+# product, two clamp bounds, one rounding, fused product-difference, square, accumulate
+QUANT_OPS_PER_EVAL = 7
+FP32_LANES_PER_SM = 128
+
+
+def quant_inputs(torch, U, I, dist, seed, dev):
+    """Unit-norm Gaussian directions (fp32, U x I) and i.i.d. bit-widths, drawn on the device
+    from a seeded generator (the layer-sized input is 2.4 GB)."""
+    g = torch.Generator(device=dev)
+    g.manual_seed(seed)
+    P = torch.empty((U, I), dtype=torch.float32, device=dev)
+    for u0 in range(0, U, 65536):
+        blk = torch.randn((min(65536, U - u0), I), generator=g, device=dev, dtype=torch.float32)
+        P[u0:u0 + blk.shape[0]] = blk / blk.norm(dim=1, keepdim=True)
+    vals = torch.tensor([b for b, _ in dist], dtype=torch.uint8, device=dev)
+    probs = torch.tensor([p for _, p in dist], dtype=torch.float64, device=dev)
+    bits = vals[torch.multinomial(probs, U, replacement=True, generator=g)]
+    return P, bits.contiguous()
+
+
+def run_quantize(args, spec, rank, world, local):
+    """Quantiser of one Qwen3-shaped layer's spectral units (U = 3 E n units of length I, group
+    128, bits from the workload's distribution, 256 scale candidates): one
+    bitsmoe_quantize_units launch per step; input 2.4 GB >> L2."""
+    import torch
+    import paper_2606_00079_gb300 as bm
+    dev = torch.device("cuda", local)
+    U, I, group, grid = args.units or 3 * spec.E * spec.n, spec.I, spec.group, args.grid
+    P, bits = quant_inputs(torch, U, I, spec.bits_dist, 1000 + rank, dev)
+    ng = I // group
+    codes = torch.empty((U, I), dtype=torch.int16, device=dev)
+    scale = torch.empty((U, ng), dtype=torch.int16, device=dev)
+    zero = torch.empty((U, ng), dtype=torch.int16, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def step():
+        bm.bitsmoe_quantize_units(P.data_ptr(), bits.data_ptr(), U, I, group, grid, codes.data_ptr(),
+                                  scale.data_ptr(), zero.data_ptr(), status.data_ptr(), stream.cuda_stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(max(3, min(args.warmup, 5))):
+            step()
+    stream.synchronize()
+    if int(status.item()) != 0:
+        raise bm.BitsMoEError(int(status.item()), "bitsmoe_quantize_units")
+    clk = ClockSampler(local)
+    clk.start()
+    rank_barrier(world)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clk.mark("t0")
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    e1.synchronize()
+    clk.mark("t1")
+    torch.cuda.synchronize()
+    rank_barrier(world)
+    ms_own = e0.elapsed_time(e1)
+    ms = max_over_ranks(ms_own, world, dev)
+    clocks = clk.stop()
+    value = job_throughput(world, args.steps, U, ms)
+    # roofline: the search's lane-instructions against the fp32 lanes at the clock seen under load
+    low = ((bits >= 2) & (bits <= 4)).sum().item()
+    evals = float(low) * ng * group * grid
+    ops = evals * QUANT_OPS_PER_EVAL
+    sec = ms_own / args.steps / 1e3
+    peaks, _ = measured_peaks()
+    sm_mhz = clocks.get("sm_mhz") or float(peaks.get("sm_max_mhz", 2070.0))
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    peak = sms * FP32_LANES_PER_SM * sm_mhz * 1e6 / 1e12
+    peak_max = sms * FP32_LANES_PER_SM * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6 / 1e12
+    achieved = ops / sec / 1e12
+    hbm_bytes = U * I * 4.0 + U * I * 2.0 + U + 2.0 * U * ng * 2
+    roofline = {"bound": "alu", "kernel": "k_quantize (scale search of the 2-4 bit units)", "achieved": achieved,
+                "peak": peak, "unit": "T lane-instr/s", "frac": achieved / peak,
+                "peak_source": f"{sms} SMs x {FP32_LANES_PER_SM} fp32 lanes x {sm_mhz:.0f} MHz (median SM clock "
+                               "under load)",
+                "frac_at_max_clock": achieved / peak_max, "traffic": None,
+                "ops_per_eval": QUANT_OPS_PER_EVAL, "evals_per_launch": evals,
+                "hbm_gbs": hbm_bytes / sec / 1e9, "bytes_per_launch": hbm_bytes,
+                "duration_us": sec * 1e6}
+    # e2e: pinned host units in, codes / scales / zeros out, every step
+    ne = 3
+    Ph = P.cpu().pin_memory()
+    ch = torch.empty_like(codes, device="cpu").pin_memory()
+    sh = torch.empty_like(scale, device="cpu").pin_memory()
+    zh = torch.empty_like(zero, device="cpu").pin_memory()
+    t0 = time.perf_counter()
+    for _ in range(ne):
+        with torch.cuda.stream(stream):
+            P.copy_(Ph, non_blocking=True)
+            step()
+            ch.copy_(codes, non_blocking=True)
+            sh.copy_(scale, non_blocking=True)
+            zh.copy_(zero, non_blocking=True)
+        stream.synchronize()
+    e2e_s = time.perf_counter() - t0
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        from oracle import quantizer as Q
+        n_done, secs, chunk = 0, 0.0, 0
+        while secs < 12.0 and chunk < 64:   # chunks of 4096 units, about 12 s of CPU work
+            Pn, bn = synth.make_float_units(4096, I, seed=chunk, bits_dist=dict(spec.bits_dist))
+            t = time.perf_counter()
+            Q.quantize_units(Pn, bn, group, grid)
+            secs += time.perf_counter() - t
+            n_done += 4096
+            chunk += 1
+        cpu = {"value": n_done / secs, "unit": "units/s", "cores": cpu_cores(), "kind": "oracle",
+               "sample": f"{n_done} units of {I} (same bit distribution), fp32 numpy quantiser, {secs:.1f} s"}
+    if rank == 0:
+        line = {
+            "metric": QUANT_METRIC, "value": value, "unit": "units/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": f"quantiser: {spec.name} layer's spectral units (3 x {spec.E} x {spec.n} units "
+                                   f"of {I}, group {group}, mean {spec.mean_bits} bits, {grid} scale candidates)",
+                       "units": U, "unit_length": I, "group": group, "grid": grid,
+                       "l2": f"input {U * I * 4 / 1e9:.2f} GB per step (129 MB L2)"},
+            "roofline": roofline, "cpu_baseline": cpu,
+            "e2e": {"value": world * ne * U / e2e_s, "unit": "units/s", "steps": ne,
+                    "h2d_bytes_per_step": U * I * 4, "d2h_bytes_per_step": U * I * 2 + 2 * U * ng * 2},
+            "clocks": clocks, "gpu_launches": args.steps,
+        }
+        print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=None, help="default 20000 (one layer), 400 (layer stack)")
+    ap.add_argument("--steps", type=int, default=None,
+                    help="default 20000 (one layer), 400 (layer stack), 20 (--task quantize)")
     ap.add_argument("--warmup", type=int, default=200)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="qw3")
@@ -374,11 +507,16 @@ def main():
     ap.add_argument("--inputs", type=int, default=64)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--graph", type=int, default=256, help="forwards per captured CUDA graph")
+    ap.add_argument("--task", default="forward", choices=["forward", "quantize"],
+                    help="forward: the MoE-layer forward (default); quantize: the per-unit quantiser")
+    ap.add_argument("--grid", type=int, default=256, help="scale candidates of the quantiser (--task quantize)")
+    ap.add_argument("--units", type=int, default=None,
+                    help="units per quantiser step (--task quantize; default the whole layer, 3 E n)")
     args = ap.parse_args()
     spec = synth.WORKLOADS[args.workload]
     T = args.tokens or spec.tokens[0]
     if args.steps is None:
-        args.steps = 20000 if spec.layers == 1 else 400
+        args.steps = 20 if args.task == "quantize" else (20000 if spec.layers == 1 else 400)
     if args.impl == "reference":
         run_reference(args, spec, T)
         return
@@ -394,6 +532,12 @@ def main():
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
 
+    if args.task == "quantize":
+        run_quantize(args, spec, rank, world, local)
+        if world > 1:
+            torch.distributed.barrier()
+            torch.distributed.destroy_process_group()
+        return
     if spec.layers > 1:
         run_stack(args, spec, T, torch, bm, dev, rank, world, local)
         if world > 1:

@@ -260,6 +260,43 @@ int bitsmoe_profile_forward(const void* x, const float* logits, int T, int top_k
 int bitsmoe_moe_forward_noalloc(const void* x, const float* logits, int T, int top_k,
                                 const bitsmoe_layer* layer, float* y, void* stream);
 
+/* Quantise spectral units into the stored unit format above (the offline
+ * step that produces `codes`, `scale` and `zero` of bitsmoe_layer_host), on
+ * the GPU, asynchronously on `stream`.  BitsMoE quantises every normalised
+ * spectral vector p (a unit, length I) with its own bit-width b (appendix
+ * "Piecewise Reconstruction Error for Bit Allocation"), one scale per group
+ * of `group` consecutive elements (group 128 in the paper's experiments):
+ *   b = 2, 3, 4  symmetric uniform quantiser Q_b(p; s) = s clamp(round(p / s),
+ *                -2^(b-1), 2^(b-1) - 1) (Eq. app_scalar_quantization_uk) with
+ *                the MSE-optimal scale (Eq. app_low_bit_opt_scale), searched
+ *                over the fp16 candidates s_c = fp16(rho 2^(2-b) c / grid),
+ *                c = 1 .. grid, rho = max |p| over the group
+ *   b = 6, 8     Q_b with s = fp16(rho / (2^(b-1) - 1)) (Eq. app_uk_scale)
+ *   b = 1        sign quantiser mean|p| sign(p), sign(0) = +1
+ *                (Eq. app_one_bit_quantization)
+ *   b = 0        evicted (Eq. app_zero_bit_vector); b = 16: fp16 values.
+ * Stored: code = level + 2^(b-1), zero = 2^(b-1), scale = s (sign quantiser:
+ * code = [p >= 0], zero = 1/2, scale = 2 mean|p|); 0-bit units store zeros,
+ * 16-bit units the fp16 bit patterns and scale = zero = 0.  Arithmetic is
+ * fp32 with every operation rounded once, the quotient p / s taken as p times
+ * the rounded reciprocal of s, error sums in element order, ties to the
+ * smaller c; the result is deterministic.  A group with no usable scale (all
+ * zeros, or every candidate 0 or infinite in fp16) stores scale 0.
+ *   p       device, U x I fp32 (row u = unit u), 16-byte aligned, finite values
+ *   bits    device, U bit-widths
+ *   U       units (U == 0 is a successful no-op); I % group == 0
+ *   group   32, 64, 128 or 256
+ *   grid    candidates of the scale search: 32, 64, 128, 256, 512 or 1024
+ *   codes   device, U x I uint16 (written), 16-byte aligned
+ *   scale, zero  device, U x (I / group) fp16 bit patterns (written)
+ *   status  device int or NULL: a unit whose bit-width is not in
+ *           {0,1,2,3,4,6,8,16} gets zero outputs and, if status is not NULL
+ *           and holds 0, BITSMOE_ERR_UNSUPPORTED_BITS is written there
+ * Host-side checks only (INVALID_ARG, SHAPE, ALIGNMENT); never allocates,
+ * never synchronises.  One kernel launch. */
+int bitsmoe_quantize_units(const float* p, const uint8_t* bits, int64_t U, int I, int group, int grid,
+                           uint16_t* codes, uint16_t* scale, uint16_t* zero, int* status, void* stream);
+
 /* Synchronise `stream`, then read and clear the device status word kept in
  * `ws`: BITSMOE_OK, or the first device-side error recorded by the last
  * forward that used this workspace (each forward resets it when it starts). */

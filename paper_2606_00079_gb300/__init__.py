@@ -63,6 +63,7 @@ SIGNATURES = {
     "bitsmoe_moe_forward_noalloc": (_I, [_P, _P, _I, _I, _P, _P, _P]),
     "bitsmoe_rmsnorm_router": (_I, [_P, _P, ctypes.c_float, _I, _I, _I, _P, _P, _P]),
     "bitsmoe_moe_block_forward": (_I, [_P, _P, ctypes.c_float, _I, _I, _P, _P, _SZ, _P]),
+    "bitsmoe_quantize_units": (_I, [_P, _P, ctypes.c_int64, _I, _I, _I, _P, _P, _P, _P, _P]),
     "bitsmoe_last_device_status": (_I, [_P, _P]),
     "bitsmoe_free": (None, [_P]),
     "bitsmoe_strerror": (ctypes.c_char_p, [_I]),
@@ -308,6 +309,13 @@ def bitsmoe_profile_forward(x_ptr: int, logits_ptr: int, T: int, top_k: int, lay
     return [float(v) for v in ms]
 
 
+def bitsmoe_quantize_units(p_ptr: int, bits_ptr: int, U: int, I: int, group: int, grid: int, codes_ptr: int,
+                           scale_ptr: int, zero_ptr: int, status_ptr: int = 0, stream: int = 0) -> None:
+    """Quantise U float units (device U x I fp32) into codes / fp16 scale / fp16 zero (device)."""
+    _check(_lib().bitsmoe_quantize_units(p_ptr, bits_ptr, U, I, group, grid, codes_ptr, scale_ptr, zero_ptr,
+                                         status_ptr, stream), "bitsmoe_quantize_units")
+
+
 def bitsmoe_last_device_status(ws_ptr: int, stream: int = 0) -> int:
     return int(_lib().bitsmoe_last_device_status(ws_ptr, stream))
 
@@ -346,3 +354,21 @@ def moe_forward(layer: Layer, x_bits, logits, top_k: int, ws: Optional[Workspace
     bitsmoe_moe_forward(x_bits.data_ptr(), logits.data_ptr(), T, top_k, layer, y.data_ptr(),
                         ws.ptr, ws.nbytes, st.cuda_stream)
     return y
+
+
+def quantize_units(p, bits, group: int, grid: int = 256, stream=None):
+    """Quantise the units in the rows of `p` (torch fp32 U x I on the device) with per-unit
+    bit-widths `bits` (torch uint8, U) into the stored format; returns (codes uint16-as-int16
+    U x I, scale, zero fp16 bit patterns U x I/group, status int32 tensor of one element)."""
+    import torch
+    U, I = int(p.shape[0]), int(p.shape[1])
+    dev = p.device
+    codes = torch.empty((U, I), dtype=torch.int16, device=dev)
+    scale = torch.empty((U, I // group), dtype=torch.int16, device=dev)
+    zero = torch.empty((U, I // group), dtype=torch.int16, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    st = stream if stream is not None else torch.cuda.current_stream(dev)
+    bitsmoe_quantize_units(p.data_ptr(), bits.data_ptr(), U, I, group, grid, codes.data_ptr(), scale.data_ptr(),
+                           zero.data_ptr(), status.data_ptr(), st.cuda_stream)
+    return codes, scale, zero, status
+

@@ -1723,6 +1723,10 @@ int noalloc_scratch(int device, void** out) {
 
 }  // namespace
 
+namespace bmoe {
+int record_cuda_error(int cuda_error) { return cuda_fail(static_cast<cudaError_t>(cuda_error)); }
+}  // namespace bmoe
+
 extern "C" {
 
 int bitsmoe_moe_forward_noalloc(const void* x, const float* logits, int T, int top_k, const bitsmoe_layer* L,

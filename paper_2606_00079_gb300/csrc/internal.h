@@ -26,6 +26,10 @@ inline const ExpertDesc* desc_of(const uint8_t* img) {
   return reinterpret_cast<const ExpertDesc*>(img + header_of(img)->off_desc);
 }
 
+// Keep a failed CUDA call's error for bitsmoe_last_cuda_error (on this host
+// thread) and return BITSMOE_ERR_CUDA.
+int record_cuda_error(int cuda_error);
+
 // Supported quantisation groups and their checks.
 inline bool group_ok(int g) { return g == 32 || g == 64 || g == 128 || g == 256; }
 inline bool bits_ok(int b) {

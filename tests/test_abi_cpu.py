@@ -162,3 +162,22 @@ def test_malformed_blob_rejected(bm):
 def test_strerror(bm):
     assert bm.bitsmoe_strerror(0) == "ok"
     assert "workspace" in bm.bitsmoe_strerror(-4)
+
+
+def test_quantize_units_host_checks(bm):
+    """bitsmoe_quantize_units rejects bad arguments on the host, before any device work."""
+    lib = bm._lib()
+    A = 4096   # a 16-byte-aligned stand-in address (never dereferenced: the checks fail first)
+    q = lambda U, I, group, grid, p=A, codes=A, scale=A: lib.bitsmoe_quantize_units(
+        p, A, U, I, group, grid, codes, scale, A, 0, 0)
+    assert q(0, 128, 64, 256) == 0                                   # U == 0: no-op
+    assert q(-1, 128, 64, 256) == bm.ERR_CODE["INVALID_ARG"]
+    assert q(4, 0, 64, 256) == bm.ERR_CODE["INVALID_ARG"]
+    assert q(4, 96, 64, 256) == bm.ERR_CODE["SHAPE"]                 # I % group
+    assert q(4, 96, 48, 256) == bm.ERR_CODE["SHAPE"]                 # unsupported group
+    assert q(4, 128, 64, 100) == bm.ERR_CODE["INVALID_ARG"]          # grid not in the set
+    assert q(4, 128, 64, 2048) == bm.ERR_CODE["INVALID_ARG"]
+    assert q(4, 128, 64, 256, p=0) == bm.ERR_CODE["INVALID_ARG"]
+    assert q(4, 128, 64, 256, p=A + 4) == bm.ERR_CODE["ALIGNMENT"]
+    assert q(4, 128, 64, 256, codes=A + 8) == bm.ERR_CODE["ALIGNMENT"]
+    assert q(4, 128, 64, 256, scale=A + 1) == bm.ERR_CODE["ALIGNMENT"]
