@@ -494,6 +494,128 @@ def run_quantize(args, spec, rank, world, local):
         print(json.dumps(line), flush=True)
 
 
+ALLOC_METRIC = "spectral units allocated/s (per-projection bit allocation: costs, Lagrangian cut, greedy fill)"
+KAPPA_TABLE = (0.14949200, 0.04067890, 0.01184786)   # kappa_2, kappa_3, kappa_4 (Table kappa_values)
+
+
+def run_allocate(args, spec, rank, world, local):
+    """Bit allocation of one Qwen3-shaped layer: three projections of U = E n units of length I,
+    each under the paper's budget B_h = floor(E n b_eq - 16 n^2 / I) at b_eq = mean unit bits;
+    alpha_j = j^-1/2, beta log-normal, gamma 1/2.  A step is three bitsmoe_allocate_bits calls."""
+    import torch
+    import paper_2606_00079_gb300 as bm
+    dev = torch.device("cuda", local)
+    U, I = args.units or spec.E * spec.n, spec.I
+    P, _ = quant_inputs(torch, 3 * U, I, spec.bits_dist, 2000 + rank, dev)
+    g = torch.Generator(device=dev)
+    g.manual_seed(3000 + rank)
+    j = (torch.arange(3 * U, device=dev) % spec.n + 1).to(torch.float32)
+    alpha = j.pow(-0.5).contiguous()
+    beta = torch.exp(torch.randn(3 * U, generator=g, device=dev, dtype=torch.float32)).contiguous()
+    gamma = 0.5
+    from fractions import Fraction
+    budget = int((Fraction(U) * Fraction(str(spec.mean_bits)) * I - 16 * spec.n * spec.n) // I)
+    bits = torch.empty(3 * U, dtype=torch.uint8, device=dev)
+    nb = bm.bitsmoe_allocate_workspace_bytes(U)
+    wsb = torch.empty(nb + 256, dtype=torch.uint8, device=dev)
+    ws = (wsb.data_ptr() + 255) // 256 * 256
+    stream = torch.cuda.Stream(device=dev)
+
+    def call(h, profile=False):
+        o = h * U
+        return bm.bitsmoe_allocate_bits(P[o].data_ptr(), alpha[o:].data_ptr(), beta[o:].data_ptr(), gamma, U, I,
+                                        KAPPA_TABLE, budget, bits[o:].data_ptr(), ws, nb, stream.cuda_stream,
+                                        profile=profile)
+
+    def step():
+        for h in range(3):
+            call(h)
+
+    with torch.cuda.stream(stream):
+        for _ in range(max(3, min(args.warmup, 5))):
+            step()
+    stream.synchronize()
+    used = [int(bits[h * U:(h + 1) * U].to(torch.int64).sum().item()) for h in range(3)]
+    clk = ClockSampler(local)
+    clk.start()
+    rank_barrier(world)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clk.mark("t0")
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    e1.synchronize()
+    clk.mark("t1")
+    torch.cuda.synchronize()
+    rank_barrier(world)
+    ms_own = e0.elapsed_time(e1)
+    ms = max_over_ranks(ms_own, world, dev)
+    clocks = clk.stop()
+    value = job_throughput(world, args.steps, 3 * U, ms)
+    # roofline of the cost kernel (the one that streams the units), timed alone by the profiling call
+    nprof = 6
+    ph = np.zeros(3)
+    for i in range(nprof):
+        ph += np.array(call(i % 3, profile=True))
+    ph /= nprof
+    peaks, peak_src = measured_peaks()
+    peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    cost_bytes = U * (4.0 * I + 8.0)
+    achieved = cost_bytes / (ph[0] / 1e3) / 1e9
+    roofline = {"bound": "hbm", "kernel": "k_alloc_cost (distortions, costs and hull of every unit)",
+                "achieved": achieved, "peak": peak, "peak_source": peak_src, "unit": "GB/s",
+                "frac": achieved / peak, "traffic": None, "bytes_per_launch": cost_bytes,
+                "duration_us": ph[0] * 1e3, "duration_source": "CUDA events around the kernel (profiling call)",
+                "phase_ms": {"costs_and_hull": ph[0], "cut_and_result": ph[1], "fill": ph[2]},
+                "frac_of_8tbs": achieved / NOMINAL_HBM_GBS}
+    # e2e: pinned host units in, bit-widths out, every step
+    ne = 3
+    Ph = P.cpu().pin_memory()
+    bh = torch.empty_like(bits, device="cpu").pin_memory()
+    t0 = time.perf_counter()
+    for _ in range(ne):
+        with torch.cuda.stream(stream):
+            P.copy_(Ph, non_blocking=True)
+            step()
+            bh.copy_(bits, non_blocking=True)
+        stream.synchronize()
+    e2e_s = time.perf_counter() - t0
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        from oracle import allocator as Aor
+        kap = {2: KAPPA_TABLE[0], 3: KAPPA_TABLE[1], 4: KAPPA_TABLE[2]}
+        Pn, _ = synth.make_float_units(16384, I, seed=0)
+        an = (((np.arange(16384) % spec.n) + 1.0) ** -0.5).astype(np.float32)
+        n_done, secs, rep = 0, 0.0, 0
+        while secs < 12.0 and rep < 400:   # one chunk of 16384 units, new betas each time, ~12 s of CPU work
+            bn = np.random.default_rng([rep, 5]).lognormal(0.0, 1.0, 16384).astype(np.float32)
+            t = time.perf_counter()
+            Aor.allocate(Aor.costs(Pn, an, bn, gamma, kap), int(budget * 16384 / U))
+            secs += time.perf_counter() - t
+            n_done += 16384
+            rep += 1
+        cpu = {"value": n_done / secs, "unit": "units/s", "cores": cpu_cores(), "kind": "oracle",
+               "sample": f"{rep} allocations of a 16384-unit chunk of {I} (budget scaled, new betas each), "
+                         f"numpy, {secs:.1f} s"}
+    if rank == 0:
+        line = {
+            "metric": ALLOC_METRIC, "value": value, "unit": "units/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": f"bit allocation: {spec.name} layer, 3 projections x {U} units of {I}, budget "
+                                   f"B_h = {budget} (b_eq {spec.mean_bits}), gamma {gamma}",
+                       "units": 3 * U, "unit_length": I, "budget_per_projection": budget,
+                       "bits_used": used, "l2": f"input {3 * U * I * 4 / 1e9:.2f} GB per step (129 MB L2)"},
+            "roofline": roofline, "cpu_baseline": cpu,
+            "e2e": {"value": world * ne * 3 * U / e2e_s, "unit": "units/s", "steps": ne,
+                    "h2d_bytes_per_step": 3 * U * I * 4, "d2h_bytes_per_step": 3 * U},
+            "clocks": clocks, "gpu_launches": args.steps * 3 * 43,
+        }
+        print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -507,16 +629,18 @@ def main():
     ap.add_argument("--inputs", type=int, default=64)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--graph", type=int, default=256, help="forwards per captured CUDA graph")
-    ap.add_argument("--task", default="forward", choices=["forward", "quantize"],
-                    help="forward: the MoE-layer forward (default); quantize: the per-unit quantiser")
+    ap.add_argument("--task", default="forward", choices=["forward", "quantize", "allocate"],
+                    help="forward: the MoE-layer forward (default); quantize: the per-unit quantiser; "
+                         "allocate: the per-projection bit allocation")
     ap.add_argument("--grid", type=int, default=256, help="scale candidates of the quantiser (--task quantize)")
     ap.add_argument("--units", type=int, default=None,
-                    help="units per quantiser step (--task quantize; default the whole layer, 3 E n)")
+                    help="units per quantiser step (default the whole layer, 3 E n) or per allocated "
+                         "projection (default E n)")
     args = ap.parse_args()
     spec = synth.WORKLOADS[args.workload]
     T = args.tokens or spec.tokens[0]
     if args.steps is None:
-        args.steps = 20 if args.task == "quantize" else (20000 if spec.layers == 1 else 400)
+        args.steps = 20 if args.task != "forward" else (20000 if spec.layers == 1 else 400)
     if args.impl == "reference":
         run_reference(args, spec, T)
         return
@@ -532,8 +656,8 @@ def main():
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
 
-    if args.task == "quantize":
-        run_quantize(args, spec, rank, world, local)
+    if args.task != "forward":
+        (run_quantize if args.task == "quantize" else run_allocate)(args, spec, rank, world, local)
         if world > 1:
             torch.distributed.barrier()
             torch.distributed.destroy_process_group()

@@ -297,6 +297,51 @@ int bitsmoe_moe_forward_noalloc(const void* x, const float* logits, int T, int t
 int bitsmoe_quantize_units(const float* p, const uint8_t* bits, int64_t U, int I, int group, int grid,
                            uint16_t* codes, uint16_t* scale, uint16_t* zero, int* status, void* stream);
 
+/* Bit allocation for the units of one projection type (the offline step that
+ * produces `bits` of bitsmoe_layer_host), on the GPU, asynchronously on
+ * `stream`.  BitsMoE picks b_u in {0,1,2,3,4,6,8,16} for every unit u by the
+ * ILP of Eq. ilp_piecewise_eps: minimise sum_u C_u(b_u) subject to
+ * sum_u b_u <= budget, with C_u(b) = alpha_u^2 beta_u^gamma E_u(b) (Eq.
+ * app_component_loss_final) and the piecewise distortion of Eq.
+ * piecewise_expected_eps: E(0) = 1, E(1) = 1 - ||p_u||_1^2 / d,
+ * E(2|3|4) = kappa_2|3|4 (Table kappa_values: 0.14949200, 0.04067890,
+ * 0.01184786), E(6|8|16) = (d ||p_u||_inf^2 / 3) 2^(-2b).  The budget of the
+ * paper is B_h = floor(E n b_eq - 16 n^2 / m) (Eq.
+ * app_projection_normalized_budget) for E experts, rank n, unit length m.
+ * The ILP is solved by its Lagrangian relaxation plus a greedy fill: per unit
+ * the lower convex hull of (b, C(b)) from b = 0 (ties to the smaller b); hull
+ * increments taken in descending efficiency (ties to the lower unit index)
+ * while the bits fit, a group of equal efficiency within a unit whole or not
+ * at all (this part is an exact optimum for the bits it uses); then, while
+ * some unit's next increment fits the bits left, the most efficient one.
+ * Arithmetic is fp32, each operation rounded once (||p||_1 as an exact
+ * fixed-point sum of floor(|p_i| 2^40)); the result is deterministic.
+ *   p       device, U x d fp32 (row u = unit u, the normalised spectral
+ *           vector), 16-byte aligned, |p_i| < 2^20
+ *   alpha   device, U fp32 spectral energies; beta device, U fp32 importances
+ *           (beta_u = phi_u^T H phi_u, Eq. app_beta_vector_def), beta >= 0
+ *   gamma   smoothing exponent in [0, 1]; 0, 1/2 and 1 are exact (1, sqrt,
+ *           identity), other values use powf
+ *   U       units, 0 .. 2^32 - 2 (U == 0 is a successful no-op); d >= 1
+ *   kappa   host, 3 floats: the distortion of 2, 3 and 4 bits
+ *   budget  >= 0, in bits per unit element (sum of b_u)
+ *   bits    device, U bytes (written)
+ *   ws      device workspace of >= bitsmoe_allocate_workspace_bytes(U)
+ *           bytes, 256-byte aligned, caller-owned; no initialisation needed
+ * Host-side checks only (INVALID_ARG, SHAPE, ALIGNMENT,
+ * WORKSPACE_TOO_SMALL); never allocates, never synchronises.  43 kernel
+ * launches and one memset on `stream`. */
+size_t bitsmoe_allocate_workspace_bytes(int64_t U);
+int bitsmoe_allocate_bits(const float* p, const float* alpha, const float* beta, float gamma, int64_t U, int d,
+                          const float* kappa, int64_t budget, uint8_t* bits, void* ws, size_t ws_bytes,
+                          void* stream);
+/* Same, with the phases timed by CUDA events on `stream` and the call
+ * synchronised: phase_ms[0] the cost and hull kernel, [1] the selection of the
+ * cut and the per-unit result, [2] the fill. */
+int bitsmoe_profile_allocate_bits(const float* p, const float* alpha, const float* beta, float gamma, int64_t U,
+                                  int d, const float* kappa, int64_t budget, uint8_t* bits, void* ws,
+                                  size_t ws_bytes, void* stream, float phase_ms[3]);
+
 /* Synchronise `stream`, then read and clear the device status word kept in
  * `ws`: BITSMOE_OK, or the first device-side error recorded by the last
  * forward that used this workspace (each forward resets it when it starts). */

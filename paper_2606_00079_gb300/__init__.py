@@ -64,6 +64,12 @@ SIGNATURES = {
     "bitsmoe_rmsnorm_router": (_I, [_P, _P, ctypes.c_float, _I, _I, _I, _P, _P, _P]),
     "bitsmoe_moe_block_forward": (_I, [_P, _P, ctypes.c_float, _I, _I, _P, _P, _SZ, _P]),
     "bitsmoe_quantize_units": (_I, [_P, _P, ctypes.c_int64, _I, _I, _I, _P, _P, _P, _P, _P]),
+    "bitsmoe_allocate_workspace_bytes": (_SZ, [ctypes.c_int64]),
+    "bitsmoe_allocate_bits": (_I, [_P, _P, _P, ctypes.c_float, ctypes.c_int64, _I, ctypes.POINTER(ctypes.c_float),
+                                   ctypes.c_int64, _P, _P, _SZ, _P]),
+    "bitsmoe_profile_allocate_bits": (_I, [_P, _P, _P, ctypes.c_float, ctypes.c_int64, _I,
+                                           ctypes.POINTER(ctypes.c_float), ctypes.c_int64, _P, _P, _SZ, _P,
+                                           ctypes.POINTER(ctypes.c_float)]),
     "bitsmoe_last_device_status": (_I, [_P, _P]),
     "bitsmoe_free": (None, [_P]),
     "bitsmoe_strerror": (ctypes.c_char_p, [_I]),
@@ -316,6 +322,26 @@ def bitsmoe_quantize_units(p_ptr: int, bits_ptr: int, U: int, I: int, group: int
                                          status_ptr, stream), "bitsmoe_quantize_units")
 
 
+def bitsmoe_allocate_workspace_bytes(U: int) -> int:
+    return int(_lib().bitsmoe_allocate_workspace_bytes(U))
+
+
+def bitsmoe_allocate_bits(p_ptr: int, alpha_ptr: int, beta_ptr: int, gamma: float, U: int, d: int, kappa,
+                          budget: int, bits_ptr: int, ws_ptr: int, ws_bytes: int, stream: int = 0,
+                          profile: bool = False):
+    """Bit-width per unit (device, U bytes) for one projection type; with profile=True the call
+    synchronises and returns the phase durations (ms: costs and hull, cut, fill)."""
+    k = (ctypes.c_float * 3)(*[float(v) for v in kappa])
+    if profile:
+        ms = (ctypes.c_float * 3)()
+        _check(_lib().bitsmoe_profile_allocate_bits(p_ptr, alpha_ptr, beta_ptr, gamma, U, d, k, budget, bits_ptr,
+                                                    ws_ptr, ws_bytes, stream, ms), "bitsmoe_profile_allocate_bits")
+        return [float(v) for v in ms]
+    _check(_lib().bitsmoe_allocate_bits(p_ptr, alpha_ptr, beta_ptr, gamma, U, d, k, budget, bits_ptr, ws_ptr,
+                                        ws_bytes, stream), "bitsmoe_allocate_bits")
+    return None
+
+
 def bitsmoe_last_device_status(ws_ptr: int, stream: int = 0) -> int:
     return int(_lib().bitsmoe_last_device_status(ws_ptr, stream))
 
@@ -371,4 +397,20 @@ def quantize_units(p, bits, group: int, grid: int = 256, stream=None):
     bitsmoe_quantize_units(p.data_ptr(), bits.data_ptr(), U, I, group, grid, codes.data_ptr(), scale.data_ptr(),
                            zero.data_ptr(), status.data_ptr(), st.cuda_stream)
     return codes, scale, zero, status
+
+
+def allocate_bits(p, alpha, beta, gamma: float, kappa, budget: int, stream=None):
+    """Bit-widths (torch uint8, U) of the units in the rows of `p` (torch fp32 U x d on the
+    device) with spectral energies `alpha` and importances `beta` (fp32, U) under `budget`."""
+    import torch
+    U, d = int(p.shape[0]), int(p.shape[1])
+    dev = p.device
+    bits = torch.empty(U, dtype=torch.uint8, device=dev)
+    nb = bitsmoe_allocate_workspace_bytes(U)
+    ws = torch.empty(nb + 256, dtype=torch.uint8, device=dev)
+    st = stream if stream is not None else torch.cuda.current_stream(dev)
+    bitsmoe_allocate_bits(p.data_ptr(), alpha.data_ptr(), beta.data_ptr(), gamma, U, d, kappa, budget,
+                          bits.data_ptr(), (ws.data_ptr() + 255) // 256 * 256, nb, st.cuda_stream)
+    ws.record_stream(st)   # the workspace is freed here but used by the kernels still queued on st
+    return bits
 

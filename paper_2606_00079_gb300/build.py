@@ -1,10 +1,11 @@
 """Build libbitsmoe.so in-tree with nvcc for sm_103a (GB300).
 
-Six translation units, compiled in parallel: the host packer (pack.cpp,
+Seven translation units, compiled in parallel: the host packer (pack.cpp,
 plain C++), the CUDA kernel chain + C ABI (forward.cu), the fused
 single-token decode kernel (fused.cu), the tensor-core projections
-(gemm.cu), the tensor-core expert factors (expert_tc.cu) and the per-unit
-quantiser from float spectral vectors (quantize.cu).  The CUDA runtime is linked
+(gemm.cu), the tensor-core expert factors (expert_tc.cu), the per-unit
+quantiser from float spectral vectors (quantize.cu) and the per-projection
+bit allocation (allocate.cu).  The CUDA runtime is linked
 statically, so the library loads on a machine without a GPU (the host-only
 entry points then work; the device ones return BITSMOE_ERR_CUDA).
 """
@@ -39,7 +40,8 @@ def _run(cmd):
 
 
 def sources():
-    return [os.path.join(CSRC, f) for f in ("pack.cpp", "forward.cu", "fused.cu", "gemm.cu", "expert_tc.cu", "quantize.cu")]
+    return [os.path.join(CSRC, f) for f in ("pack.cpp", "forward.cu", "fused.cu", "gemm.cu", "expert_tc.cu", "quantize.cu",
+                                              "allocate.cu")]
 
 
 def up_to_date() -> bool:

@@ -1,0 +1,432 @@
+// Per-projection bit allocation: which bit-width every spectral unit gets.
+//
+// BitsMoE chooses b_u in {0,1,2,3,4,6,8,16} for the units of one projection
+// type by the ILP of Eq. ilp_piecewise_eps: minimise sum_u C_u(b_u) subject to
+// sum_u b_u <= B_h, with C_u(b) = alpha_u^2 beta_u^gamma E_u(b) (Eq.
+// app_component_loss_final) and the piecewise distortion of Eq.
+// piecewise_expected_eps (eta 2^(-2b) for b >= 6 with eta = d rho^2 / 3,
+// kappa_b for 2..4, sin^2 theta = 1 - ||p||_1^2 / d for 1 bit, 1 for 0 bits).
+// The paper hands the ILP to a commercial solver; here it is solved by the
+// Lagrangian relaxation of the multiple-choice knapsack plus a greedy fill:
+//
+//   k_alloc_cost   one warp per 32 units: rho = max |p| and ||p||_1 (an exact
+//                  fixed-point sum, so the order of the lanes does not matter)
+//                  per unit, then each lane builds its unit's costs and the
+//                  lower convex hull of (b, C(b)) from b = 0 (ties to the
+//                  smaller b, efficiencies capped so they never increase); an
+//                  increment's key is (bits of its efficiency) << 32 | ~u
+//   radix select   four passes over the 16-bit digits of the keys: a histogram
+//                  of the increments' bit counts by digit (k_alloc_hist), then
+//                  one block finds the digit where the bits taken so far would
+//                  pass B_h (k_alloc_scan); after the last pass the cut K* is
+//                  the key of the first increment group that does not fit
+//   k_alloc_final  every unit takes its increments with key > K* (the
+//                  Lagrangian solution) and exposes its next one
+//   fill rounds    while a next increment fits the bits left, the one with
+//                  the largest key is taken (grid-wide max, then one thread)
+//
+// Everything is fp32 with each operation rounded once, in the same steps as
+// the allocation oracle, so the bit-widths are a deterministic function of
+// the inputs.  The cost kernel streams the units once (HBM-bound); the rest
+// works on 64 bytes per unit of workspace.
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <algorithm>
+
+#include "device.cuh"
+#include "internal.h"
+
+namespace {
+
+constexpr int kAW = 8;                 // warps per block of the cost kernel
+constexpr int kNB = 8;                 // bit-width options
+constexpr int kNS = 7;                 // at most 7 hull increments
+constexpr int kFillRounds = 16;        // the fill takes at most 15 increments (bits left < 16)
+constexpr int kDigits = 65536;
+__constant__ int c_bits[kNB] = {0, 1, 2, 3, 4, 6, 8, 16};
+
+struct AllocState {
+  unsigned long long prefix;   // key bits decided by the radix passes
+  unsigned long long above;    // bits of the increments above the current bucket (all taken)
+  unsigned long long kstar;    // the cut: increments with key > kstar are taken (0: all)
+  unsigned long long used;     // bits after the cut
+  unsigned long long best;     // fill round: largest fitting next key
+  long long left;              // fill: bits left
+  int all_fit;                 // every increment fits: nothing to select
+  int fill_done;
+};
+
+struct AllocWs {
+  AllocState* st;
+  unsigned long long* hist;    // [kDigits]
+  unsigned long long* keys;    // [U][kNS], 0 = none
+  uint8_t* reach;              // [U][kNS] option index reached by each increment
+  uint8_t* taken;              // [U]
+  unsigned long long* nkey;    // [U] next increment's key (0 = none)
+  uint8_t* ndb;                // [U] its bits
+};
+
+size_t ws_layout(int64_t U, size_t* off) {
+  size_t o = 0;
+  auto put = [&](int i, size_t bytes) {
+    off[i] = o;
+    o = (o + bytes + 255) / 256 * 256;
+  };
+  put(0, sizeof(AllocState));
+  put(1, (size_t)kDigits * 8);
+  put(2, (size_t)U * kNS * 8);
+  put(3, (size_t)U * kNS);
+  put(4, (size_t)U);
+  put(5, (size_t)U * 8);
+  put(6, (size_t)U);
+  return o;
+}
+
+__device__ __forceinline__ float weight(float a, float b, float gamma) {
+  float bg;
+  if (gamma == 0.f) bg = 1.f;
+  else if (gamma == 0.5f) bg = __fsqrt_rn(b);
+  else if (gamma == 1.f) bg = b;
+  else bg = powf(b, gamma);
+  return __fmul_rn(__fmul_rn(a, a), bg);
+}
+
+// Costs and hull of one unit (one lane), written to its rows of the workspace.
+__device__ void unit_hull(float rho, long long l1fix, int d, float w, float k2, float k3, float k4, uint32_t u,
+                          unsigned long long* keys, uint8_t* reach) {
+  const float l1 = __fmul_rn(__ll2float_rn(l1fix), 9.094947017729282e-13f);   // 2^-40
+  const float sin2 = __fsub_rn(1.f, __fdiv_rn(__fmul_rn(l1, l1), (float)d));
+  const float eta = __fdiv_rn(__fmul_rn(__fmul_rn(rho, rho), (float)d), 3.f);
+  float C[kNB];
+  C[0] = w;                                  // w * 1
+  C[1] = __fmul_rn(w, sin2);
+  C[2] = __fmul_rn(w, k2);
+  C[3] = __fmul_rn(w, k3);
+  C[4] = __fmul_rn(w, k4);
+  C[5] = __fmul_rn(w, __fmul_rn(eta, 2.44140625e-4f));       // 2^-12
+  C[6] = __fmul_rn(w, __fmul_rn(eta, 1.52587890625e-5f));    // 2^-16
+  C[7] = __fmul_rn(w, __fmul_rn(eta, 2.3283064365386963e-10f));   // 2^-32
+  int cur = 0;
+  float curc = C[0], prev = __int_as_float(0x7F800000);
+  const unsigned long long low = 0xFFFFFFFFull - u;
+#pragma unroll 1
+  for (int s = 0; s < kNS; ++s) {
+    float be = 0.f;
+    int bj = -1;
+#pragma unroll
+    for (int j = 1; j < kNB; ++j) {
+      if (j > cur) {
+        const float e = __fdiv_rn(__fsub_rn(curc, C[j]), (float)(c_bits[j] - c_bits[cur]));
+        if (e > 0.f && e > be) {
+          be = e;
+          bj = j;
+        }
+      }
+    }
+    if (bj < 0) {
+      for (int r = s; r < kNS; ++r) {
+        keys[r] = 0ull;
+        reach[r] = 0xFF;
+      }
+      return;
+    }
+    const float e = fminf(be, prev);
+    keys[s] = ((unsigned long long)__float_as_uint(e) << 32) | low;
+    reach[s] = (uint8_t)bj;
+    curc = C[bj];
+    cur = bj;
+    prev = e;
+  }
+}
+
+struct CostArgs {
+  const float* p;
+  const float* alpha;
+  const float* beta;
+  float gamma, k2, k3, k4;
+  int64_t U;
+  int d;
+  AllocWs w;
+};
+
+// One warp per 32 consecutive units; lane l keeps unit (base + l)'s rho and ||p||_1.
+__global__ void __launch_bounds__(kAW * 32) k_alloc_cost(CostArgs a) {
+  const int lane = threadIdx.x & 31;
+  const int64_t nwarps = (int64_t)gridDim.x * kAW;
+  const bool v4 = (a.d & 3) == 0;
+  for (int64_t base = ((int64_t)blockIdx.x * kAW + (threadIdx.x >> 5)) * 32; base < a.U; base += nwarps * 32) {
+    const int nu = a.U - base < 32 ? (int)(a.U - base) : 32;
+    float my_rho = 0.f;
+    long long my_l1 = 0;
+    for (int k = 0; k < nu; ++k) {
+      const float* row = a.p + (size_t)(base + k) * a.d;
+      float mx = 0.f;
+      long long s = 0;
+      if (v4) {
+        for (int i = lane; i < a.d / 4; i += 32) {
+          const float4 x = __ldcs(reinterpret_cast<const float4*>(row) + i);
+          const float ax = fabsf(x.x), ay = fabsf(x.y), az = fabsf(x.z), aw = fabsf(x.w);
+          mx = fmaxf(mx, fmaxf(fmaxf(ax, ay), fmaxf(az, aw)));
+          s += __float2ll_rd(__fmul_rn(ax, 1099511627776.f)) + __float2ll_rd(__fmul_rn(ay, 1099511627776.f)) +
+               __float2ll_rd(__fmul_rn(az, 1099511627776.f)) + __float2ll_rd(__fmul_rn(aw, 1099511627776.f));
+        }
+      } else {
+        for (int i = lane; i < a.d; i += 32) {
+          const float ax = fabsf(__ldcs(row + i));
+          mx = fmaxf(mx, ax);
+          s += __float2ll_rd(__fmul_rn(ax, 1099511627776.f));   // 2^40
+        }
+      }
+      mx = warp_max(mx);
+#pragma unroll
+      for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
+      if (lane == k) {
+        my_rho = mx;
+        my_l1 = s;
+      }
+    }
+    if (lane < nu) {
+      const int64_t u = base + lane;
+      const float w = weight(__ldg(a.alpha + u), __ldg(a.beta + u), a.gamma);
+      unit_hull(my_rho, my_l1, a.d, w, a.k2, a.k3, a.k4, (uint32_t)u, a.w.keys + (size_t)u * kNS,
+                a.w.reach + (size_t)u * kNS);
+    }
+  }
+}
+
+__device__ __forceinline__ int step_bits(const uint8_t* r, int s) {
+  return c_bits[r[s]] - (s ? c_bits[r[s - 1]] : 0);
+}
+
+// Radix pass: bits of the increments in the current bucket, by the digit at `shift`.
+__global__ void k_alloc_hist(AllocWs w, int64_t U, int shift) {
+  const AllocState& st = *w.st;
+  if (st.all_fit) return;
+  const int hs = shift + 16;
+  const unsigned long long pre = st.prefix;
+  for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < U; u += (int64_t)gridDim.x * blockDim.x) {
+    const unsigned long long* k = w.keys + (size_t)u * kNS;
+    const uint8_t* r = w.reach + (size_t)u * kNS;
+#pragma unroll 1
+    for (int s = 0; s < kNS; ++s) {
+      const unsigned long long key = k[s];
+      if (!key) break;
+      if (hs < 64 && (key >> hs) != (pre >> hs)) continue;
+      atomicAdd(w.hist + ((key >> shift) & 0xFFFFull), (unsigned long long)step_bits(r, s));
+    }
+  }
+}
+
+// One block: find the largest digit d with above + sum_{d' >= d} hist[d'] > budget.
+__global__ void __launch_bounds__(1024) k_alloc_scan(AllocWs w, long long budget, int shift, int last) {
+  __shared__ unsigned long long part[1024];
+  __shared__ int found;
+  AllocState& st = *w.st;
+  const int t = threadIdx.x;
+  constexpr int per = kDigits / 1024;
+  const bool skip = st.all_fit != 0;
+  // thread t owns digits [t * per, t * per + per); suffix sums run from the top digit down
+  unsigned long long mine = 0;
+  for (int i = 0; i < per; ++i) mine += w.hist[t * per + i];
+  part[t] = mine;
+  if (t == 0) found = 0;
+  __syncthreads();
+  // inclusive suffix scan over threads (Hillis-Steele, from high t to low t)
+  for (int o = 1; o < 1024; o <<= 1) {
+    const unsigned long long v = t + o < 1024 ? part[t + o] : 0ull;
+    __syncthreads();
+    part[t] += v;
+    __syncthreads();
+  }
+  const unsigned long long above = st.above;
+  const unsigned long long bud = (unsigned long long)budget;
+  if (!skip) {
+    unsigned long long run = (t + 1 < 1024 ? part[t + 1] : 0ull);   // digits above this thread's range
+    if (above + run + mine > bud && above + run <= bud) {
+      for (int i = per - 1; i >= 0; --i) {
+        const unsigned long long h = w.hist[t * per + i];
+        if (above + run + h > bud) {
+          const int dgt = t * per + i;
+          st.prefix |= (unsigned long long)dgt << shift;
+          st.above = above + run;
+          found = 1;
+          break;
+        }
+        run += h;
+      }
+    }
+  }
+  __syncthreads();
+  if (t == 0 && !skip) {
+    if (!found) {   // only possible in the first pass: every increment fits
+      st.all_fit = 1;
+      st.kstar = 0ull;
+    } else if (last) {
+      st.kstar = st.prefix;
+    }
+  }
+  for (int i = 0; i < per; ++i) w.hist[t * per + i] = 0ull;   // ready for the next pass
+}
+
+// Step 3 for every unit, and its next increment for the fill.
+__global__ void k_alloc_final(AllocWs w, int64_t U, uint8_t* bits) {
+  const unsigned long long ks = w.st->kstar;
+  unsigned long long used = 0;
+  for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < U; u += (int64_t)gridDim.x * blockDim.x) {
+    const unsigned long long* k = w.keys + (size_t)u * kNS;
+    const uint8_t* r = w.reach + (size_t)u * kNS;
+    int t = 0;
+    while (t < kNS && k[t] > ks) ++t;
+    const int b = t ? c_bits[r[t - 1]] : 0;
+    bits[u] = (uint8_t)b;
+    used += (unsigned long long)b;
+    w.taken[u] = (uint8_t)t;
+    const bool more = t < kNS && k[t] != 0ull;
+    w.nkey[u] = more ? k[t] : 0ull;
+    w.ndb[u] = more ? (uint8_t)step_bits(r, t) : (uint8_t)0;
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) used += __shfl_xor_sync(0xFFFFFFFFu, used, o);
+  if ((threadIdx.x & 31) == 0 && used) atomicAdd(&w.st->used, used);
+}
+
+__global__ void k_fill_init(AllocWs w, long long budget) {
+  AllocState& st = *w.st;
+  st.left = budget - (long long)st.used;
+  st.best = 0ull;
+  st.fill_done = 0;
+}
+
+__global__ void k_fill_max(AllocWs w, int64_t U) {
+  const AllocState& st = *w.st;
+  if (st.fill_done) return;
+  const long long left = st.left;
+  unsigned long long best = 0ull;
+  for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < U; u += (int64_t)gridDim.x * blockDim.x) {
+    const unsigned long long k = w.nkey[u];
+    if (k > best && (long long)w.ndb[u] <= left) best = k;
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) {
+    const unsigned long long v = __shfl_xor_sync(0xFFFFFFFFu, best, o);
+    best = v > best ? v : best;
+  }
+  if ((threadIdx.x & 31) == 0 && best) atomicMax(&w.st->best, best);
+}
+
+__global__ void k_fill_take(AllocWs w, int64_t U, uint8_t* bits) {
+  AllocState& st = *w.st;
+  if (st.fill_done) return;
+  const unsigned long long k = st.best;
+  if (!k) {
+    st.fill_done = 1;
+    return;
+  }
+  const int64_t u = (int64_t)(0xFFFFFFFFull - (k & 0xFFFFFFFFull));
+  if (u < 0 || u >= U) {   // cannot happen: keys carry their unit
+    st.fill_done = 1;
+    return;
+  }
+  const uint8_t* r = w.reach + (size_t)u * kNS;
+  const unsigned long long* ks = w.keys + (size_t)u * kNS;
+  const int t = w.taken[u];
+  st.left -= (long long)w.ndb[u];
+  bits[u] = (uint8_t)c_bits[r[t]];
+  w.taken[u] = (uint8_t)(t + 1);
+  const bool more = t + 1 < kNS && ks[t + 1] != 0ull;
+  w.nkey[u] = more ? ks[t + 1] : 0ull;
+  w.ndb[u] = more ? (uint8_t)step_bits(r, t + 1) : (uint8_t)0;
+  st.best = 0ull;
+}
+
+int sms_of_current(int* sms) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(sms, cudaDevAttrMultiProcessorCount, dev);
+  return e == cudaSuccess ? BITSMOE_OK : bmoe::record_cuda_error((int)e);
+}
+
+int allocate_impl(const float* p, const float* alpha, const float* beta, float gamma, int64_t U, int d,
+                  const float* kappa, int64_t budget, uint8_t* bits, void* ws, size_t ws_bytes, cudaStream_t st,
+                  float* phase_ms) {
+  if (U < 0 || d < 1 || budget < 0 || !(gamma >= 0.f && gamma <= 1.f)) return BITSMOE_ERR_INVALID_ARG;
+  if (U > 0xFFFFFFFEll || (int64_t)d > (1ll << 24)) return BITSMOE_ERR_SHAPE;
+  if (U == 0) return BITSMOE_OK;
+  if (!p || !alpha || !beta || !kappa || !bits || !ws) return BITSMOE_ERR_INVALID_ARG;
+  if ((uintptr_t)p % 16 || (uintptr_t)alpha % 4 || (uintptr_t)beta % 4 || (uintptr_t)ws % 256)
+    return BITSMOE_ERR_ALIGNMENT;
+  size_t off[7];
+  if (ws_bytes < ws_layout(U, off)) return BITSMOE_ERR_WORKSPACE_TOO_SMALL;
+  int sms = 0;
+  int rc = sms_of_current(&sms);
+  if (rc) return rc;
+  uint8_t* wb = static_cast<uint8_t*>(ws);
+  AllocWs w{reinterpret_cast<AllocState*>(wb + off[0]), reinterpret_cast<unsigned long long*>(wb + off[1]),
+            reinterpret_cast<unsigned long long*>(wb + off[2]), wb + off[3], wb + off[4],
+            reinterpret_cast<unsigned long long*>(wb + off[5]), wb + off[6]};
+  cudaEvent_t ev[4] = {};
+  if (phase_ms) {
+    for (auto& e : ev)
+      if (cudaEventCreate(&e) != cudaSuccess) return bmoe::record_cuda_error((int)cudaGetLastError());
+  }
+  auto fail = [&](cudaError_t e) {
+    if (phase_ms)
+      for (auto& x : ev) cudaEventDestroy(x);
+    return bmoe::record_cuda_error((int)e);
+  };
+  cudaError_t e = cudaMemsetAsync(wb + off[0], 0, off[2], st);   // state and histogram
+  if (e != cudaSuccess) return fail(e);
+  if (phase_ms) cudaEventRecord(ev[0], st);
+  CostArgs ca{p, alpha, beta, gamma, kappa[0], kappa[1], kappa[2], U, d, w};
+  const int64_t groups = (U + 31) / 32;
+  const int64_t cost_blocks = std::min<int64_t>((groups + kAW - 1) / kAW, (int64_t)sms * 8);
+  k_alloc_cost<<<(unsigned)cost_blocks, kAW * 32, 0, st>>>(ca);
+  if (phase_ms) cudaEventRecord(ev[1], st);
+  const unsigned ub = (unsigned)std::min<int64_t>((U + 255) / 256, (int64_t)sms * 8);
+  for (int pass = 0; pass < 4; ++pass) {
+    const int shift = 48 - 16 * pass;
+    k_alloc_hist<<<ub, 256, 0, st>>>(w, U, shift);
+    k_alloc_scan<<<1, 1024, 0, st>>>(w, (long long)budget, shift, pass == 3);
+  }
+  k_alloc_final<<<ub, 256, 0, st>>>(w, U, bits);
+  if (phase_ms) cudaEventRecord(ev[2], st);
+  k_fill_init<<<1, 1, 0, st>>>(w, (long long)budget);
+  for (int r = 0; r < kFillRounds; ++r) {
+    k_fill_max<<<ub, 256, 0, st>>>(w, U);
+    k_fill_take<<<1, 1, 0, st>>>(w, U, bits);
+  }
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return fail(e);
+  if (phase_ms) {
+    cudaEventRecord(ev[3], st);
+    e = cudaEventSynchronize(ev[3]);
+    if (e != cudaSuccess) return fail(e);
+    for (int i = 0; i < 3; ++i) cudaEventElapsedTime(&phase_ms[i], ev[i], ev[i + 1]);
+    for (auto& x : ev) cudaEventDestroy(x);
+  }
+  return BITSMOE_OK;
+}
+
+}  // namespace
+
+extern "C" size_t bitsmoe_allocate_workspace_bytes(int64_t U) {
+  if (U < 0 || U > 0xFFFFFFFEll) return 0;
+  size_t off[7];
+  return ws_layout(U, off);
+}
+
+extern "C" int bitsmoe_allocate_bits(const float* p, const float* alpha, const float* beta, float gamma, int64_t U,
+                                     int d, const float* kappa, int64_t budget, uint8_t* bits, void* ws,
+                                     size_t ws_bytes, void* stream) {
+  return allocate_impl(p, alpha, beta, gamma, U, d, kappa, budget, bits, ws, ws_bytes,
+                       static_cast<cudaStream_t>(stream), nullptr);
+}
+
+extern "C" int bitsmoe_profile_allocate_bits(const float* p, const float* alpha, const float* beta, float gamma,
+                                             int64_t U, int d, const float* kappa, int64_t budget, uint8_t* bits,
+                                             void* ws, size_t ws_bytes, void* stream, float phase_ms[3]) {
+  if (!phase_ms) return BITSMOE_ERR_INVALID_ARG;
+  return allocate_impl(p, alpha, beta, gamma, U, d, kappa, budget, bits, ws, ws_bytes,
+                       static_cast<cudaStream_t>(stream), phase_ms);
+}

@@ -181,3 +181,27 @@ def test_quantize_units_host_checks(bm):
     assert q(4, 128, 64, 256, p=A + 4) == bm.ERR_CODE["ALIGNMENT"]
     assert q(4, 128, 64, 256, codes=A + 8) == bm.ERR_CODE["ALIGNMENT"]
     assert q(4, 128, 64, 256, scale=A + 1) == bm.ERR_CODE["ALIGNMENT"]
+
+
+def test_allocate_bits_host_checks(bm):
+    """bitsmoe_allocate_bits rejects bad arguments on the host, before any device work."""
+    import ctypes
+    lib = bm._lib()
+    A = 4096
+    k = (ctypes.c_float * 3)(0.149492, 0.0406789, 0.01184786)
+    nb = bm.bitsmoe_allocate_workspace_bytes(100)
+    assert nb > 100 * 64 and bm.bitsmoe_allocate_workspace_bytes(-1) == 0
+    call = lambda U=100, d=64, gamma=0.5, budget=50, p=A, ws=A, wsb=nb, kap=k: lib.bitsmoe_allocate_bits(
+        p, A, A, gamma, U, d, kap, budget, A, ws, wsb, 0)
+    assert call(U=0) == 0                                            # no-op
+    assert call(U=-1) == bm.ERR_CODE["INVALID_ARG"]
+    assert call(d=0) == bm.ERR_CODE["INVALID_ARG"]
+    assert call(budget=-1) == bm.ERR_CODE["INVALID_ARG"]
+    assert call(gamma=1.5) == bm.ERR_CODE["INVALID_ARG"]
+    assert call(gamma=float("nan")) == bm.ERR_CODE["INVALID_ARG"]
+    assert call(U=1 << 32) == bm.ERR_CODE["SHAPE"]
+    assert call(p=0) == bm.ERR_CODE["INVALID_ARG"]
+    assert call(kap=None) == bm.ERR_CODE["INVALID_ARG"]
+    assert call(p=A + 4) == bm.ERR_CODE["ALIGNMENT"]
+    assert call(ws=A + 16) == bm.ERR_CODE["ALIGNMENT"]
+    assert call(wsb=nb - 1) == bm.ERR_CODE["WORKSPACE_TOO_SMALL"]
