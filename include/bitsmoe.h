@@ -317,12 +317,12 @@ int bitsmoe_quantize_units(const float* p, const uint8_t* bits, int64_t U, int I
  * Arithmetic is fp32, each operation rounded once (||p||_1 as an exact
  * fixed-point sum of floor(|p_i| 2^40)); the result is deterministic.
  *   p       device, U x d fp32 (row u = unit u, the normalised spectral
- *           vector), 16-byte aligned, |p_i| < 2^20
+ *           vector), 16-byte aligned, |p_i| < 32
  *   alpha   device, U fp32 spectral energies; beta device, U fp32 importances
  *           (beta_u = phi_u^T H phi_u, Eq. app_beta_vector_def), beta >= 0
  *   gamma   smoothing exponent in [0, 1]; 0, 1/2 and 1 are exact (1, sqrt,
  *           identity), other values use powf
- *   U       units, 0 .. 2^32 - 2 (U == 0 is a successful no-op); d >= 1
+ *   U       units, 0 .. 2^32 - 2 (U == 0 is a successful no-op); 1 <= d <= 16384
  *   kappa   host, 3 floats: the distortion of 2, 3 and 4 bits
  *   budget  >= 0, in bits per unit element (sum of b_u)
  *   bits    device, U bytes (written)

@@ -9,8 +9,9 @@
 // The paper hands the ILP to a commercial solver; here it is solved by the
 // Lagrangian relaxation of the multiple-choice knapsack plus a greedy fill:
 //
-//   k_alloc_cost   one warp per 32 units: rho = max |p| and ||p||_1 (an exact
-//                  fixed-point sum, so the order of the lanes does not matter)
+//   k_alloc_cost   one warp per 32 units, eight rows streamed side by side:
+//                  rho = max |p| and ||p||_1 (an exact fixed-point sum, so the
+//                  order of the lanes does not matter)
 //                  per unit, then each lane builds its unit's costs and the
 //                  lower convex hull of (b, C(b)) from b = 0 (ties to the
 //                  smaller b, efficiencies capped so they never increase); an
@@ -150,7 +151,23 @@ struct CostArgs {
   AllocWs w;
 };
 
+// floor(|x| 2^40) for |x| < 32 as A 2^22 + B with A = floor(y), B = floor(frac(y) 2^22),
+// y = |x| 2^18 < 2^23: each is read off the bits of a round-toward-zero add of 2^23
+// (2^23 + floor(v) for 0 <= v < 2^23).  The raw bit patterns are summed; the caller
+// subtracts count * bits(2^23) (mod 2^32).  Also the running max |x|.
+__device__ __forceinline__ void fix_add(float ax, float& mx, uint32_t& sa, uint32_t& sb) {
+  mx = fmaxf(mx, ax);
+  const float y = __fmul_rn(ax, 262144.f);                                          // 2^18
+  const float ty = __fadd_rz(y, 8388608.f);                                         // 2^23 + floor(y)
+  const float z = __fmul_rn(__fsub_rn(y, __fsub_rn(ty, 8388608.f)), 4194304.f);   // frac(y) 2^22
+  sa += __float_as_uint(ty);
+  sb += __float_as_uint(__fadd_rz(z, 8388608.f));
+}
+
 // One warp per 32 consecutive units; lane l keeps unit (base + l)'s rho and ||p||_1.
+// The warp streams kUK units' rows side by side, so kUK 16-byte loads per lane are in
+// flight at once.
+constexpr int kUK = 8;
 __global__ void __launch_bounds__(kAW * 32) k_alloc_cost(CostArgs a) {
   const int lane = threadIdx.x & 31;
   const int64_t nwarps = (int64_t)gridDim.x * kAW;
@@ -159,31 +176,53 @@ __global__ void __launch_bounds__(kAW * 32) k_alloc_cost(CostArgs a) {
     const int nu = a.U - base < 32 ? (int)(a.U - base) : 32;
     float my_rho = 0.f;
     long long my_l1 = 0;
-    for (int k = 0; k < nu; ++k) {
-      const float* row = a.p + (size_t)(base + k) * a.d;
-      float mx = 0.f;
-      long long s = 0;
+    for (int k0 = 0; k0 < nu; k0 += kUK) {
+      float mx[kUK];
+      uint32_t sa[kUK], sb[kUK];
+#pragma unroll
+      for (int q = 0; q < kUK; ++q) {
+        mx[q] = 0.f;
+        sa[q] = sb[q] = 0u;
+      }
+      const float* rows[kUK];
+#pragma unroll
+      for (int q = 0; q < kUK; ++q) rows[q] = a.p + (size_t)(base + (k0 + q < nu ? k0 + q : 0)) * a.d;
+      uint32_t cnt = 0;
       if (v4) {
         for (int i = lane; i < a.d / 4; i += 32) {
-          const float4 x = __ldcs(reinterpret_cast<const float4*>(row) + i);
-          const float ax = fabsf(x.x), ay = fabsf(x.y), az = fabsf(x.z), aw = fabsf(x.w);
-          mx = fmaxf(mx, fmaxf(fmaxf(ax, ay), fmaxf(az, aw)));
-          s += __float2ll_rd(__fmul_rn(ax, 1099511627776.f)) + __float2ll_rd(__fmul_rn(ay, 1099511627776.f)) +
-               __float2ll_rd(__fmul_rn(az, 1099511627776.f)) + __float2ll_rd(__fmul_rn(aw, 1099511627776.f));
+          float4 x[kUK];
+#pragma unroll
+          for (int q = 0; q < kUK; ++q) x[q] = __ldcs(reinterpret_cast<const float4*>(rows[q]) + i);
+#pragma unroll
+          for (int q = 0; q < kUK; ++q) {
+            fix_add(fabsf(x[q].x), mx[q], sa[q], sb[q]);
+            fix_add(fabsf(x[q].y), mx[q], sa[q], sb[q]);
+            fix_add(fabsf(x[q].z), mx[q], sa[q], sb[q]);
+            fix_add(fabsf(x[q].w), mx[q], sa[q], sb[q]);
+          }
+          cnt += 4;
         }
       } else {
         for (int i = lane; i < a.d; i += 32) {
-          const float ax = fabsf(__ldcs(row + i));
-          mx = fmaxf(mx, ax);
-          s += __float2ll_rd(__fmul_rn(ax, 1099511627776.f));   // 2^40
+          float x[kUK];
+#pragma unroll
+          for (int q = 0; q < kUK; ++q) x[q] = __ldcs(rows[q] + i);
+#pragma unroll
+          for (int q = 0; q < kUK; ++q) fix_add(fabsf(x[q]), mx[q], sa[q], sb[q]);
+          cnt += 1;
         }
       }
-      mx = warp_max(mx);
 #pragma unroll
-      for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, o);
-      if (lane == k) {
-        my_rho = mx;
-        my_l1 = s;
+      for (int q = 0; q < kUK; ++q) {
+        const uint32_t A = sa[q] - cnt * 0x4B000000u, B = sb[q] - cnt * 0x4B000000u;
+        long long sum = ((long long)A << 22) + (long long)B;
+        const float m = warp_max(mx[q]);
+#pragma unroll
+        for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
+        if (lane == k0 + q) {
+          my_rho = m;
+          my_l1 = sum;
+        }
       }
     }
     if (lane < nu) {
@@ -351,7 +390,7 @@ int allocate_impl(const float* p, const float* alpha, const float* beta, float g
                   const float* kappa, int64_t budget, uint8_t* bits, void* ws, size_t ws_bytes, cudaStream_t st,
                   float* phase_ms) {
   if (U < 0 || d < 1 || budget < 0 || !(gamma >= 0.f && gamma <= 1.f)) return BITSMOE_ERR_INVALID_ARG;
-  if (U > 0xFFFFFFFEll || (int64_t)d > (1ll << 24)) return BITSMOE_ERR_SHAPE;
+  if (U > 0xFFFFFFFEll || d > 16384) return BITSMOE_ERR_SHAPE;
   if (U == 0) return BITSMOE_OK;
   if (!p || !alpha || !beta || !kappa || !bits || !ws) return BITSMOE_ERR_INVALID_ARG;
   if ((uintptr_t)p % 16 || (uintptr_t)alpha % 4 || (uintptr_t)beta % 4 || (uintptr_t)ws % 256)
@@ -379,8 +418,11 @@ int allocate_impl(const float* p, const float* alpha, const float* beta, float g
   if (e != cudaSuccess) return fail(e);
   if (phase_ms) cudaEventRecord(ev[0], st);
   CostArgs ca{p, alpha, beta, gamma, kappa[0], kappa[1], kappa[2], U, d, w};
+  int per_sm = 0;
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_alloc_cost, kAW * 32, 0);
+  if (e != cudaSuccess) return fail(e);
   const int64_t groups = (U + 31) / 32;
-  const int64_t cost_blocks = std::min<int64_t>((groups + kAW - 1) / kAW, (int64_t)sms * 8);
+  const int64_t cost_blocks = std::min<int64_t>((groups + kAW - 1) / kAW, (int64_t)sms * std::max(per_sm, 1));
   k_alloc_cost<<<(unsigned)cost_blocks, kAW * 32, 0, st>>>(ca);
   if (phase_ms) cudaEventRecord(ev[1], st);
   const unsigned ub = (unsigned)std::min<int64_t>((U + 255) / 256, (int64_t)sms * 8);

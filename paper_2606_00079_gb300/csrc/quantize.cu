@@ -26,7 +26,8 @@
 // staged in shared memory; for the scale search each lane owns grid / 32
 // candidates in registers and scores them all on every element it reads (a
 // broadcast read), so the inner loop is eight fp32 instructions per
-// (element, candidate) and no shuffles; one lexicographic (error, index)
+// (element, candidate) — six for the upper quarter of the candidates, which
+// provably never clip — and no shuffles; one lexicographic (error, index)
 // warp reduction picks the scale.  The search is ALU-bound: the fp32 input is
 // read once and the codes written once.
 #include <cuda_fp16.h>
@@ -71,6 +72,33 @@ __device__ __forceinline__ float candidate(float top, int c, int grid) {
   return f16_round(__fdiv_rn(__fmul_rn(top, (float)c), (float)grid));
 }
 
+// Scores of the NC candidates of a lane over the group.  With FREE, the candidates
+// m >= kFree(NC) skip the clamp: their index c > 3 grid / 4, so with a normal fp16 scale
+// |v| / s <= 2^(b-2) (grid / c) (1 + 2^-10) < 1.34 * 2^(b-2) < 2^(b-1) - 1/2 for b <= 4,
+// and round(v / s) is already a level: the clamp would change nothing.
+template <int NC>
+__host__ __device__ constexpr int kFree() { return (3 * NC + 3) / 4; }
+template <int NC, bool FREE>
+__device__ __forceinline__ void score(const float* v, int g, const float (&sc)[NC], const float (&rc)[NC],
+                                      float (&e)[NC], float qmin, float qmax) {
+#pragma unroll 2
+  for (int i = 0; i < g; i += 4) {
+    const float4 x4 = *reinterpret_cast<const float4*>(v + i);
+    const float xs[4] = {x4.x, x4.y, x4.z, x4.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+#pragma unroll
+      for (int m = 0; m < NC; ++m) {
+        const float q = (FREE && m >= kFree<NC>())
+                            ? __fsub_rn(__fadd_rn(__fmul_rn(xs[k], rc[m]), kRne), kRne)
+                            : level(xs[k], rc[m], qmin, qmax);
+        const float d = fmaf(-sc[m], q, xs[k]);   // sc * q is exact (11 x 4 significant bits)
+        e[m] = __fadd_rn(e[m], __fmul_rn(d, d));
+      }
+    }
+  }
+}
+
 // Scale search of one group for b in {2, 3, 4}: NC candidates per lane.
 template <int NC>
 __device__ float search_scale(const float* v, int g, float rho, int b, int grid, int lane) {
@@ -86,20 +114,12 @@ __device__ float search_scale(const float* v, int g, float rho, int b, int grid,
     rc[m] = __frcp_rn(sc[m]);
     e[m] = ok ? 0.f : kInf;
   }
-#pragma unroll 2
-  for (int i = 0; i < g; i += 4) {
-    const float4 x4 = *reinterpret_cast<const float4*>(v + i);
-    const float xs[4] = {x4.x, x4.y, x4.z, x4.w};
+  // the clamp-free path needs every lane's upper candidates to be normal fp16 scales (or skipped)
+  bool normal = true;
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
-#pragma unroll
-      for (int m = 0; m < NC; ++m) {
-        const float q = level(xs[k], rc[m], qmin, qmax);
-        const float d = fmaf(-sc[m], q, xs[k]);   // sc * q is exact (11 x 4 significant bits)
-        e[m] = __fadd_rn(e[m], __fmul_rn(d, d));
-      }
-    }
-  }
+  for (int m = kFree<NC>(); m < NC; ++m) normal &= (sc[m] >= 6.103515625e-05f) || e[m] == kInf;
+  if (__all_sync(0xFFFFFFFFu, normal)) score<NC, true>(v, g, sc, rc, e, qmin, qmax);
+  else score<NC, false>(v, g, sc, rc, e, qmin, qmax);
   float be = e[0];
   int bc = lane + 1;
 #pragma unroll
