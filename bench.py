@@ -554,7 +554,13 @@ def run_allocate(args, spec, rank, world, local):
     ms = max_over_ranks(ms_own, world, dev)
     clocks = clk.stop()
     value = job_throughput(world, args.steps, 3 * U, ms)
-    # roofline of the cost kernel (the one that streams the units), timed alone by the profiling call
+    # roofline of the dominant phase (the profiling call times the three phases alone, with CUDA
+    # events on the launching stream): algorithmic bytes of each phase
+    #   costs_and_hull   k_alloc_cost: the unit rows, alpha, beta                       U (4 I + 8)
+    #   cut_and_result   4 radix passes over the increments (key 8 B + reach 1 B, 7 a unit),
+    #                    their 64 Ki-bin histograms read and cleared, the cut applied and
+    #                    the bit-widths written                                         5 U 63 + U + 4 MB
+    #   fill             16 rounds over every unit's next key and bit count             16 U 9
     nprof = 6
     ph = np.zeros(3)
     for i in range(nprof):
@@ -562,14 +568,20 @@ def run_allocate(args, spec, rank, world, local):
     ph /= nprof
     peaks, peak_src = measured_peaks()
     peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
-    cost_bytes = U * (4.0 * I + 8.0)
-    achieved = cost_bytes / (ph[0] / 1e3) / 1e9
-    roofline = {"bound": "hbm", "kernel": "k_alloc_cost (distortions, costs and hull of every unit)",
-                "achieved": achieved, "peak": peak, "peak_source": peak_src, "unit": "GB/s",
-                "frac": achieved / peak, "traffic": None, "bytes_per_launch": cost_bytes,
-                "duration_us": ph[0] * 1e3, "duration_source": "CUDA events around the kernel (profiling call)",
-                "phase_ms": {"costs_and_hull": ph[0], "cut_and_result": ph[1], "fill": ph[2]},
-                "frac_of_8tbs": achieved / NOMINAL_HBM_GBS}
+    names = ["costs_and_hull", "cut_and_result", "fill"]
+    kernels = ["k_alloc_cost (distortions, costs and hull of every unit)",
+               "radix select: k_alloc_hist + k_alloc_scan (4 passes), k_alloc_final",
+               "fill: 16 rounds of k_fill_max + k_fill_take"]
+    pbytes = [U * (4.0 * I + 8.0), 5.0 * U * 63 + U + 4 * 2 * 65536 * 8.0, 16.0 * U * 9]
+    dom = int(np.argmax(ph))
+    gbs = [pbytes[i] / (ph[i] / 1e3) / 1e9 for i in range(3)]
+    roofline = {"bound": "hbm", "kernel": kernels[dom], "achieved": gbs[dom], "peak": peak,
+                "peak_source": peak_src, "unit": "GB/s", "frac": gbs[dom] / peak, "traffic": None,
+                "bytes_per_launch": pbytes[dom], "duration_us": ph[dom] * 1e3,
+                "duration_source": "CUDA events around the phase (profiling call)",
+                "phase_ms": {names[i]: ph[i] for i in range(3)},
+                "phase_frac_of_measured": {names[i]: gbs[i] / peak for i in range(3)},
+                "frac_of_8tbs": gbs[dom] / NOMINAL_HBM_GBS}
     # e2e: pinned host units in, bit-widths out, every step
     ne = 3
     Ph = P.cpu().pin_memory()
