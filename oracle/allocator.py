@@ -54,7 +54,9 @@ FIX_SHIFT = 40
 
 
 def projection_budget(E: int, n: int, m: int, b_eq) -> int:
-    """B_h = floor(E n b_eq - 16 n^2 / m) (Eq. app_projection_normalized_budget), exactly."""
+    """B_h = floor(E n b_eq - 16 n^2 / m) (Eq. app_projection_normalized_budget), exactly.
+    Negative when the fp16 bases alone exceed the layer's budget (tiny layers): no
+    allocation meets it."""
     return int(np.floor(Fraction(E * n) * Fraction(str(b_eq)) - Fraction(16 * n * n, m)))
 
 
