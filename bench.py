@@ -18,6 +18,12 @@ basis) on one synthetic token.
           measured HBM copy bandwidth.
   cpu_baseline  the fp64 oracle on the host cores, on a bounded sample.
 
+`--task quantize` measures the per-unit quantiser instead (bitsmoe_quantize_units on a
+Qwen3-shaped layer's 786,432 float units; roofline against the fp32 lanes, since the
+MSE-optimal scale search is ALU-bound) and `--task allocate` the per-projection bit
+allocation (bitsmoe_allocate_bits on the same layer's three projections under the paper's
+budget; roofline of the dominant phase against HBM).  Both print the same kind of JSON line.
+
 `--impl reference` times the oracle (the only reference for this path) on the
 host cores instead and prints the same JSON line with "impl": "reference".
 Multi-GPU: the forward does not shard, so `--gpus N` under torchrun runs N
