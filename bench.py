@@ -519,8 +519,11 @@ def run_allocate(args, spec, rank, world, local):
     alpha = j.pow(-0.5).contiguous()
     beta = torch.exp(torch.randn(3 * U, generator=g, device=dev, dtype=torch.float32)).contiguous()
     gamma = 0.5
-    from fractions import Fraction
-    budget = int((Fraction(U) * Fraction(str(spec.mean_bits)) * I - 16 * spec.n * spec.n) // I)
+    if U % spec.n == 0:   # the paper's budget for U / n experts (library helper, exact integers)
+        budget = bm.bitsmoe_projection_budget(U // spec.n, spec.n, I, spec.mean_bits)
+    else:
+        from fractions import Fraction
+        budget = int((Fraction(U) * Fraction(str(spec.mean_bits)) * I - 16 * spec.n * spec.n) // I)
     bits = torch.empty(3 * U, dtype=torch.uint8, device=dev)
     nb = bm.bitsmoe_allocate_workspace_bytes(U)
     wsb = torch.empty(nb + 256, dtype=torch.uint8, device=dev)

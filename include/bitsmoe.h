@@ -332,6 +332,15 @@ int bitsmoe_quantize_units(const float* p, const uint8_t* bits, int64_t U, int I
  * WORKSPACE_TOO_SMALL); never allocates, never synchronises.  43 kernel
  * launches and one memset on `stream`. */
 size_t bitsmoe_allocate_workspace_bytes(int64_t U);
+/* The budget of one projection type, B_h = floor(E n b_eq - 16 n^2 / m) (Eq.
+ * app_projection_normalized_budget): E experts, shared rank n, unit length m,
+ * target equivalent bits b_eq = beq_num / beq_den (the fp16 bases are
+ * charged against it).  Exact integer arithmetic on the host; *out may be
+ * negative for layers whose bases alone exceed the target (no allocation can
+ * meet it).  Errors: INVALID_ARG (null out, non-positive sizes or
+ * denominator, negative numerator), SHAPE (E, n > 2^20, m > 2^24, numerator
+ * or denominator > 2^16). */
+int bitsmoe_projection_budget(int64_t E, int64_t n, int64_t m, int64_t beq_num, int64_t beq_den, int64_t* out);
 int bitsmoe_allocate_bits(const float* p, const float* alpha, const float* beta, float gamma, int64_t U, int d,
                           const float* kappa, int64_t budget, uint8_t* bits, void* ws, size_t ws_bytes,
                           void* stream);

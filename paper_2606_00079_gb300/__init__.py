@@ -65,6 +65,7 @@ SIGNATURES = {
     "bitsmoe_moe_block_forward": (_I, [_P, _P, ctypes.c_float, _I, _I, _P, _P, _SZ, _P]),
     "bitsmoe_quantize_units": (_I, [_P, _P, ctypes.c_int64, _I, _I, _I, _P, _P, _P, _P, _P]),
     "bitsmoe_allocate_workspace_bytes": (_SZ, [ctypes.c_int64]),
+    "bitsmoe_projection_budget": (_I, [ctypes.c_int64] * 5 + [ctypes.POINTER(ctypes.c_int64)]),
     "bitsmoe_allocate_bits": (_I, [_P, _P, _P, ctypes.c_float, ctypes.c_int64, _I, ctypes.POINTER(ctypes.c_float),
                                    ctypes.c_int64, _P, _P, _SZ, _P]),
     "bitsmoe_profile_allocate_bits": (_I, [_P, _P, _P, ctypes.c_float, ctypes.c_int64, _I,
@@ -320,6 +321,16 @@ def bitsmoe_quantize_units(p_ptr: int, bits_ptr: int, U: int, I: int, group: int
     """Quantise U float units (device U x I fp32) into codes / fp16 scale / fp16 zero (device)."""
     _check(_lib().bitsmoe_quantize_units(p_ptr, bits_ptr, U, I, group, grid, codes_ptr, scale_ptr, zero_ptr,
                                          status_ptr, stream), "bitsmoe_quantize_units")
+
+
+def bitsmoe_projection_budget(E: int, n: int, m: int, b_eq) -> int:
+    """B_h = floor(E n b_eq - 16 n^2 / m) for b_eq given as a float, an int or a (num, den) pair."""
+    from fractions import Fraction
+    fr = Fraction(*b_eq) if isinstance(b_eq, tuple) else Fraction(str(b_eq))
+    out = ctypes.c_int64()
+    _check(_lib().bitsmoe_projection_budget(E, n, m, fr.numerator, fr.denominator, ctypes.byref(out)),
+           "bitsmoe_projection_budget")
+    return int(out.value)
 
 
 def bitsmoe_allocate_workspace_bytes(U: int) -> int:

@@ -452,6 +452,20 @@ int allocate_impl(const float* p, const float* alpha, const float* beta, float g
 
 }  // namespace
 
+extern "C" int bitsmoe_projection_budget(int64_t E, int64_t n, int64_t m, int64_t beq_num, int64_t beq_den,
+                                         int64_t* out) {
+  // floor(E n b_eq - 16 n^2 / m) = floor((E n num m - 16 n^2 den) / (m den)), b_eq = num / den
+  if (!out || E < 1 || n < 1 || m < 1 || beq_den < 1 || beq_num < 0) return BITSMOE_ERR_INVALID_ARG;
+  if (E > (1 << 20) || n > (1 << 20) || m > (1 << 24) || beq_num > (1 << 16) || beq_den > (1 << 16))
+    return BITSMOE_ERR_SHAPE;
+  const __int128 num = (__int128)E * n * beq_num * m - (__int128)16 * n * n * beq_den;
+  const __int128 den = (__int128)m * beq_den;
+  __int128 q = num / den;
+  if ((num % den) != 0 && num < 0) q -= 1;   // floor for negative budgets
+  *out = (int64_t)q;
+  return BITSMOE_OK;
+}
+
 extern "C" size_t bitsmoe_allocate_workspace_bytes(int64_t U) {
   if (U < 0 || U > 0xFFFFFFFEll) return 0;
   size_t off[7];

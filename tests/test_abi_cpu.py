@@ -205,3 +205,27 @@ def test_allocate_bits_host_checks(bm):
     assert call(p=A + 4) == bm.ERR_CODE["ALIGNMENT"]
     assert call(ws=A + 16) == bm.ERR_CODE["ALIGNMENT"]
     assert call(wsb=nb - 1) == bm.ERR_CODE["WORKSPACE_TOO_SMALL"]
+
+
+def test_projection_budget_matches_the_formula(bm):
+    """bitsmoe_projection_budget (host only) against hand values and the oracle's exact
+    rational evaluation of Eq. app_projection_normalized_budget."""
+    from oracle import allocator as A
+    assert bm.bitsmoe_projection_budget(128, 2048, 768, 2.0) == 436906
+    assert bm.bitsmoe_projection_budget(8, 4096, 14336, 2.0) == 46811
+    assert bm.bitsmoe_projection_budget(4, 64, 128, 1.5) == -128           # bases exceed the target
+    assert bm.bitsmoe_projection_budget(3, 7, 5, (7, 3)) == -108           # floor(49 - 784/5) = floor(-107.8)
+    rng = np.random.default_rng(0)
+    for _ in range(300):
+        E, n, m = int(rng.integers(1, 300)), int(rng.integers(1, 5000)), int(rng.integers(1, 20000))
+        beq = round(float(rng.uniform(0, 8)), 3)
+        assert bm.bitsmoe_projection_budget(E, n, m, beq) == A.projection_budget(E, n, m, beq), (E, n, m, beq)
+    lib = bm._lib()
+    import ctypes
+    out = ctypes.c_int64()
+    assert lib.bitsmoe_projection_budget(0, 1, 1, 1, 1, ctypes.byref(out)) == bm.ERR_CODE["INVALID_ARG"]
+    assert lib.bitsmoe_projection_budget(1, 1, 1, 1, 0, ctypes.byref(out)) == bm.ERR_CODE["INVALID_ARG"]
+    assert lib.bitsmoe_projection_budget(1, 1, 1, -1, 1, ctypes.byref(out)) == bm.ERR_CODE["INVALID_ARG"]
+    assert lib.bitsmoe_projection_budget(1, 1, 1, 1, 1, None) == bm.ERR_CODE["INVALID_ARG"]
+    assert lib.bitsmoe_projection_budget(1 << 21, 1, 1, 1, 1, ctypes.byref(out)) == bm.ERR_CODE["SHAPE"]
+
