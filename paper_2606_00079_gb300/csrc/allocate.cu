@@ -454,15 +454,16 @@ int allocate_impl(const float* p, const float* alpha, const float* beta, float g
 
 extern "C" int bitsmoe_projection_budget(int64_t E, int64_t n, int64_t m, int64_t beq_num, int64_t beq_den,
                                          int64_t* out) {
-  // floor(E n b_eq - 16 n^2 / m) = floor((E n num m - 16 n^2 den) / (m den)), b_eq = num / den
+  // floor(E n b_eq - 16 n^2 / m), b_eq = num / den, in exact int64 arithmetic
   if (!out || E < 1 || n < 1 || m < 1 || beq_den < 1 || beq_num < 0) return BITSMOE_ERR_INVALID_ARG;
   if (E > (1 << 20) || n > (1 << 20) || m > (1 << 24) || beq_num > (1 << 16) || beq_den > (1 << 16))
     return BITSMOE_ERR_SHAPE;
-  const __int128 num = (__int128)E * n * beq_num * m - (__int128)16 * n * n * beq_den;
-  const __int128 den = (__int128)m * beq_den;
-  __int128 q = num / den;
-  if ((num % den) != 0 && num < 0) q -= 1;   // floor for negative budgets
-  *out = (int64_t)q;
+  // a / den - b / m with a = E n num (< 2^56), b = 16 n^2 (< 2^45): whole parts q1 - q2, and
+  // the fractional parts r1 / den - r2 / m in (-1, 1) take one more off when negative
+  // (r1 m and r2 den stay below 2^40)
+  const int64_t a = E * n * beq_num, b = 16 * n * n;
+  const int64_t q1 = a / beq_den, r1 = a % beq_den, q2 = b / m, r2 = b % m;
+  *out = q1 - q2 - (r1 * m < r2 * beq_den ? 1 : 0);
   return BITSMOE_OK;
 }
 
