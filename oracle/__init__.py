@@ -6,5 +6,5 @@ Python binding.
 """
 from .bitsmoe_oracle import *  # noqa: F401,F403
 from . import bitsmoe_oracle as core  # noqa: F401
-from . import quantizer, allocator  # noqa: F401,E402
+from . import quantizer, allocator, calibration  # noqa: F401,E402
 from .quantizer import quantize_units  # noqa: F401,E402
