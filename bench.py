@@ -390,6 +390,77 @@ def quant_inputs(torch, U, I, dist, seed, dev):
     return P, bits.contiguous()
 
 
+def quant_config(spec, U, I, group, grid):
+    return {"workload": f"quantiser: {spec.name} layer's spectral units (3 x {spec.E} x {spec.n} units "
+                        f"of {I}, group {group}, mean {spec.mean_bits} bits, {grid} scale candidates)",
+            "units": U, "unit_length": I, "group": group, "grid": grid,
+            "l2": f"input {U * I * 4 / 1e9:.2f} GB per step (129 MB L2)"}
+
+
+def alloc_config(spec, U, I, budget, gamma):
+    return {"workload": f"bit allocation: {spec.name} layer, 3 projections x {U} units of {I}, budget "
+                        f"B_h = {budget} (b_eq {spec.mean_bits}), gamma {gamma}",
+            "units": 3 * U, "unit_length": I, "budget_per_projection": budget,
+            "l2": f"input {3 * U * I * 4 / 1e9:.2f} GB per step (129 MB L2)"}
+
+
+def run_reference_task(args, spec):
+    """Reference arm of --task quantize / allocate: the oracle of that step on the host cores,
+    each step a bounded sample of the same workload (the units/s of the sample)."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    I = spec.I
+    budget_s = float(os.environ.get("BITSMOE_REF_BUDGET_S", "90")) / max(1, args.steps)
+    if args.task == "quantize":
+        from oracle import quantizer as Q
+        U = args.units or 3 * spec.E * spec.n
+        config = quant_config(spec, U, I, spec.group, args.grid)
+        chunk = 2048
+        P, bits = synth.make_float_units(chunk, I, seed=0, bits_dist=dict(spec.bits_dist))
+        run = lambda: Q.quantize_units(P, bits, spec.group, args.grid)
+        metric, what = QUANT_METRIC, f"fp32 numpy quantiser on chunks of {chunk} units"
+    else:
+        from oracle import allocator as Aor
+        U = args.units or spec.E * spec.n
+        budget = Aor.projection_budget(U // spec.n, spec.n, I, spec.mean_bits) if U % spec.n == 0 else None
+        if budget is None:
+            from fractions import Fraction
+            budget = int((Fraction(U) * Fraction(str(spec.mean_bits)) * I - 16 * spec.n * spec.n) // I)
+        config = alloc_config(spec, U, I, budget, 0.5)
+        chunk = 16384
+        P, _ = synth.make_float_units(chunk, I, seed=0)
+        an = (((np.arange(chunk) % spec.n) + 1.0) ** -0.5).astype(np.float32)
+        bn = np.random.default_rng([0, 5]).lognormal(0.0, 1.0, chunk).astype(np.float32)
+        kap = {2: KAPPA_TABLE[0], 3: KAPPA_TABLE[1], 4: KAPPA_TABLE[2]}
+        run = lambda: Aor.allocate(Aor.costs(P, an, bn, 0.5, kap), int(budget * chunk / U))
+        metric, what = ALLOC_METRIC, f"numpy allocation of chunks of {chunk} units (budget scaled)"
+    for _ in range(max(1, min(args.warmup, 3))):
+        run()
+    done, secs = 0, 0.0
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        reps = 0
+        while True:   # one step: at least one chunk, up to the per-step budget
+            run()
+            reps += 1
+            if time.perf_counter() - t0 > min(budget_s, 10.0) or reps >= 64:
+                break
+        secs += time.perf_counter() - t0
+        done += reps * chunk
+    v = done / secs
+    line = {
+        "impl": "reference", "metric": metric, "value": v, "unit": "units/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * secs / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": config,
+        "cpu_baseline": {"value": v, "unit": "units/s", "cores": cpu_cores(), "kind": "oracle",
+                         "sample": f"{done} units in {args.steps} steps ({secs:.1f} s), {what}"},
+        "e2e": {"value": v, "unit": "units/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
 def run_quantize(args, spec, rank, world, local):
     """Quantiser of one Qwen3-shaped layer's spectral units (U = 3 E n units of length I, group
     128, bits from the workload's distribution, 256 scale candidates): one
@@ -488,10 +559,7 @@ def run_quantize(args, spec, rank, world, local):
             "metric": QUANT_METRIC, "value": value, "unit": "units/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": {"workload": f"quantiser: {spec.name} layer's spectral units (3 x {spec.E} x {spec.n} units "
-                                   f"of {I}, group {group}, mean {spec.mean_bits} bits, {grid} scale candidates)",
-                       "units": U, "unit_length": I, "group": group, "grid": grid,
-                       "l2": f"input {U * I * 4 / 1e9:.2f} GB per step (129 MB L2)"},
+            "config": quant_config(spec, U, I, group, grid),
             "roofline": roofline, "cpu_baseline": cpu,
             "e2e": {"value": world * ne * U / e2e_s, "unit": "units/s", "steps": ne,
                     "h2d_bytes_per_step": U * I * 4, "d2h_bytes_per_step": U * I * 2 + 2 * U * ng * 2},
@@ -625,10 +693,7 @@ def run_allocate(args, spec, rank, world, local):
             "metric": ALLOC_METRIC, "value": value, "unit": "units/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": {"workload": f"bit allocation: {spec.name} layer, 3 projections x {U} units of {I}, budget "
-                                   f"B_h = {budget} (b_eq {spec.mean_bits}), gamma {gamma}",
-                       "units": 3 * U, "unit_length": I, "budget_per_projection": budget,
-                       "bits_used": used, "l2": f"input {3 * U * I * 4 / 1e9:.2f} GB per step (129 MB L2)"},
+            "config": alloc_config(spec, U, I, budget, gamma), "bits_used": used,
             "roofline": roofline, "cpu_baseline": cpu,
             "e2e": {"value": world * ne * 3 * U / e2e_s, "unit": "units/s", "steps": ne,
                     "h2d_bytes_per_step": 3 * U * I * 4, "d2h_bytes_per_step": 3 * U},
@@ -663,7 +728,10 @@ def main():
     if args.steps is None:
         args.steps = 20 if args.task != "forward" else (20000 if spec.layers == 1 else 400)
     if args.impl == "reference":
-        run_reference(args, spec, T)
+        if args.task == "forward":
+            run_reference(args, spec, T)
+        else:
+            run_reference_task(args, spec)
         return
 
     import torch
