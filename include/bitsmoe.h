@@ -191,8 +191,10 @@ int bitsmoe_moe_forward(const void* x, const float* logits, int T, int top_k,
  * back to host memory and synchronises `stream`.  Pinned host memory gives
  * asynchronous copies; pageable memory works but is slower.  A single token
  * on the fused kernel with all three buffers pinned (device-mapped, 16-byte
- * aligned) skips the copies: the kernel reads x and the logits from, and
- * writes y to, the host buffers directly. */
+ * aligned, each with its whole extent -- D x 2, E x 4 and D x 4 bytes -- inside
+ * one mapped allocation) skips the copies: the kernel reads x and the logits
+ * from, and writes y to, the host buffers directly.  Buffers that do not meet
+ * this take the copies. */
 int bitsmoe_moe_forward_host(const void* x_host, const float* logits_host, int T, int top_k,
                              const bitsmoe_layer* layer, float* y_host,
                              void* ws, size_t ws_bytes, void* stream);
@@ -249,7 +251,8 @@ int bitsmoe_profile_forward(const void* x, const float* logits, int T, int top_k
  * until the process exits.  This call allocates nothing: no cudaMalloc, no
  * cudaFree, no allocating library routine.  The first call on a device looks
  * up that device's address of the array (once per device, with the device
- * current); make the first call before any stream capture.
+ * current); make the first call before any stream capture (a first call on
+ * a device while `stream` is capturing returns BITSMOE_ERR_INVALID_ARG).
  *   x, logits, y, T, top_k, layer, stream: as for bitsmoe_moe_forward.
  * Errors: as bitsmoe_moe_forward, and BITSMOE_ERR_WORKSPACE_TOO_SMALL when
  * bitsmoe_workspace_bytes(layer, T, top_k) > BITSMOE_NOALLOC_SCRATCH_BYTES.
@@ -259,6 +262,14 @@ int bitsmoe_profile_forward(const void* x, const float* logits, int T, int top_k
  * threads) race and give wrong results: serialise them. */
 int bitsmoe_moe_forward_noalloc(const void* x, const float* logits, int T, int top_k,
                                 const bitsmoe_layer* layer, float* y, void* stream);
+
+/* Device status word of the no-allocation scratch on the current device: what
+ * bitsmoe_last_device_status reports for a caller's workspace, for the calls
+ * of bitsmoe_moe_forward_noalloc (whose workspace the caller cannot name).
+ * Synchronises `stream`, returns BITSMOE_OK or the first device-side error a
+ * no-allocation call recorded (BITSMOE_ERR_TIMEOUT, BITSMOE_ERR_WORKSPACE_STATE,
+ * BITSMOE_ERR_DEVICE_BOUNDS) and clears it.  Not during a stream capture. */
+int bitsmoe_noalloc_last_status(void* stream);
 
 /* Quantise spectral units into the stored unit format above (the offline
  * step that produces `codes`, `scale` and `zero` of bitsmoe_layer_host), on

@@ -23,7 +23,7 @@ The paper solves the ILP with a commercial solver.  This build solves it with
 the Lagrangian relaxation of the multiple-choice knapsack plus a greedy fill,
 the same steps on both sides (``allocate``), and checks the result against the
 exact optimum (``ilp_optimum``: dynamic programming over the budget, tiny
-inputs) and the LP bound.  Steps (readings, listed in the design doc):
+inputs) and the LP bound.  Steps (readings where the paper leaves the arithmetic open):
 
 1. costs in fp32, each operation rounded once: ||p||_1 as the exact integer sum
    of floor(|p_i| 2^40) scaled by 2^-40 (order-free), sin^2 = 1 - (l1 l1) / d,

@@ -27,7 +27,7 @@ Passages followed (BitsMoE paper):
   the quantised spectral factors compute the routed experts; SwiGLU
   gate/up/down projections (Sec. Shared-basis Spectral Decomposition).
 
-Readings where the paper is silent (each is listed in the design doc):
+Readings where the paper is silent (the same readings on the CUDA side):
 * stored format of a unit of b bits, 0 < b < 16: unsigned codes q in
   [0, 2^b) with one fp16 scale s and fp16 zero z per group of `group`
   consecutive elements along the unit vector, p_hat[i] = s[g(i)] * (q[i] - z[g(i)]).

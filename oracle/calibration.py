@@ -13,7 +13,7 @@ loss lemma; appendix Eqs. app_beta_def, app_down_beta_approx, app_unified_beta_d
   beta_k = p_k^T H p_k for the down projection (the expert-specific vector, H over the
   expert's intermediate activations).
 
-Reading (listed in the design doc): a token's routing affinity to expert e is its gate weight
+Reading (the paper does not fix it): a token's routing affinity to expert e is its gate weight
 (the softmax over its k selected experts) when e is selected and 0 otherwise, the same
 weights the forward applies.
 """
@@ -48,29 +48,54 @@ def affinities(logits: np.ndarray, top_k: int, E: int) -> np.ndarray:
     return g
 
 
-def intermediate(layer, x_bits: np.ndarray, e: int) -> np.ndarray:
-    """The expert's SwiGLU output h = SiLU(W_gate x) * (W_up x) for every token (I x T):
-    the activations entering its down projection."""
-    X = bf16_bits_to_f64(x_bits).T                                   # D x T
-    zg = basis(layer, GATE).T @ X
-    zu = basis(layer, UP).T @ X
-    a_g = alpha(layer, GATE, e)[:, None]
-    a_u = alpha(layer, UP, e)[:, None]
-    gate = dequantize_factor(layer, GATE, e) @ (a_g * zg)
-    up = dequantize_factor(layer, UP, e) @ (a_u * zu)
+def swiglu_intermediate(Phi_g: np.ndarray, Phi_u: np.ndarray, Pa_g: np.ndarray, Pa_u: np.ndarray,
+                        X: np.ndarray) -> np.ndarray:
+    """h = SiLU(P_g A_g Phi_g^T X) * (P_u A_u Phi_u^T X) (I x T) for activations X (D x T),
+    given the factors with their energies folded in (Pa = P diag(alpha), I x n)."""
+    gate = Pa_g @ (np.asarray(Phi_g, np.float64).T @ X)
+    up = Pa_u @ (np.asarray(Phi_u, np.float64).T @ X)
     return silu(gate) * up
 
 
-def layer_importance(layer, x_bits: np.ndarray, logits: np.ndarray, top_k: int) -> Tuple[np.ndarray, ...]:
-    """beta[h][e, k] of every projection and expert on calibration tokens (x, logits)."""
-    E, n = int(layer["E"]), int(layer["n"])
+def intermediate(layer, x_bits: np.ndarray, e: int) -> np.ndarray:
+    """The expert's SwiGLU output h = SiLU(W_gate x) * (W_up x) for every token (I x T) with
+    the stored (quantised) factors: the activations entering its down projection."""
+    X = bf16_bits_to_f64(x_bits).T                                   # D x T
+    Pa_g = dequantize_factor(layer, GATE, e) * alpha(layer, GATE, e)[None, :]
+    Pa_u = dequantize_factor(layer, UP, e) * alpha(layer, UP, e)[None, :]
+    return swiglu_intermediate(basis(layer, GATE), basis(layer, UP), Pa_g, Pa_u, X)
+
+
+def factor_importance(Phi, alpha_, P, x_bits: np.ndarray, logits: np.ndarray, top_k: int) -> np.ndarray:
+    """beta[h][e, k] from the decomposition's float factors, before any quantisation.
+
+    Phi[h]: D x n bases (h = gate, up, down); alpha_[h]: E x n energies; P[h][e]: I x n
+    normalised spectral factors.  This is the allocation's input: the importance weights the
+    loss of quantising each unit (appendix Eq. app_unified_beta_def), so it is taken on the
+    unquantised factors, and the down projection's activations are the expert's SwiGLU
+    outputs of the float layer (appendix Eq. app_down_beta_approx).
+    """
+    E, n = np.asarray(alpha_[0]).shape
     g = affinities(logits, top_k, E)
     X = bf16_bits_to_f64(x_bits).T
     out = np.zeros((3, E, n))
     for e in range(E):
         H_in = activation_metric(X, g[:, e])
-        out[GATE, e] = importance(basis(layer, GATE), H_in)
-        out[UP, e] = importance(basis(layer, UP), H_in)
-        H_dn = activation_metric(intermediate(layer, x_bits, e), g[:, e])
-        out[DOWN, e] = importance(dequantize_factor(layer, DOWN, e), H_dn)
+        out[GATE, e] = importance(Phi[GATE], H_in)
+        out[UP, e] = importance(Phi[UP], H_in)
+        Pa_g = np.asarray(P[GATE][e], np.float64) * np.asarray(alpha_[GATE][e], np.float64)[None, :]
+        Pa_u = np.asarray(P[UP][e], np.float64) * np.asarray(alpha_[UP][e], np.float64)[None, :]
+        H_dn = activation_metric(swiglu_intermediate(Phi[GATE], Phi[UP], Pa_g, Pa_u, X), g[:, e])
+        out[DOWN, e] = importance(np.asarray(P[DOWN][e], np.float64), H_dn)
     return out
+
+
+def layer_importance(layer, x_bits: np.ndarray, logits: np.ndarray, top_k: int) -> Tuple[np.ndarray, ...]:
+    """beta[h][e, k] of a stored (quantised) layer on calibration tokens (x, logits): the same
+    definition as factor_importance with the dequantised factors in place of the float ones.
+    Used by the eviction-loss pin, whose loss is measured on the stored layer."""
+    E = int(layer["E"])
+    Phi = [basis(layer, h) for h in (GATE, UP, DOWN)]
+    al = [np.stack([alpha(layer, h, e) for e in range(E)]) for h in (GATE, UP, DOWN)]
+    P = [[dequantize_factor(layer, h, e) for e in range(E)] for h in (GATE, UP, DOWN)]
+    return factor_importance(Phi, al, P, x_bits, logits, top_k)

@@ -25,7 +25,7 @@ per group, p_hat = scale * (code - zero).  Symmetric levels q are stored as
 code = q + 2^(b-1) with zero = 2^(b-1); the sign quantiser as code = [p >= 0],
 zero = 1/2, scale = 2 s_1.
 
-Readings where the paper leaves the arithmetic open (listed in the design doc):
+Readings where the paper leaves the arithmetic open:
 * precision: fp32, every operation rounded once to nearest-even (no fused
   multiply-add in the error sums); the quotient p / s is taken as p times the
   fp32 reciprocal of s (within one ulp of the quotient: a code exactly at a

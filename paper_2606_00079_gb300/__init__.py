@@ -61,6 +61,7 @@ SIGNATURES = {
     "bitsmoe_moe_forward": (_I, [_P, _P, _I, _I, _P, _P, _P, _SZ, _P]),
     "bitsmoe_moe_forward_host": (_I, [_P, _P, _I, _I, _P, _P, _P, _SZ, _P]),
     "bitsmoe_moe_forward_noalloc": (_I, [_P, _P, _I, _I, _P, _P, _P]),
+    "bitsmoe_noalloc_last_status": (_I, [_P]),
     "bitsmoe_rmsnorm_router": (_I, [_P, _P, ctypes.c_float, _I, _I, _I, _P, _P, _P]),
     "bitsmoe_moe_block_forward": (_I, [_P, _P, ctypes.c_float, _I, _I, _P, _P, _SZ, _P]),
     "bitsmoe_quantize_units": (_I, [_P, _P, ctypes.c_int64, _I, _I, _I, _P, _P, _P, _P, _P]),
@@ -355,6 +356,11 @@ def bitsmoe_allocate_bits(p_ptr: int, alpha_ptr: int, beta_ptr: int, gamma: floa
 
 def bitsmoe_last_device_status(ws_ptr: int, stream: int = 0) -> int:
     return int(_lib().bitsmoe_last_device_status(ws_ptr, stream))
+
+
+def bitsmoe_noalloc_last_status(stream: int = 0) -> int:
+    """Device status of the no-allocation scratch on the current device (read and cleared)."""
+    return int(_lib().bitsmoe_noalloc_last_status(stream))
 
 
 def bitsmoe_strerror(code: int) -> str:

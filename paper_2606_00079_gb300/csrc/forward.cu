@@ -1351,15 +1351,20 @@ int launch_k2k3_dec(const Fwd& p, int A_max, int sms, cudaStream_t st, bool pdl,
 
 bool aligned(const void* ptr, size_t a) { return ((uintptr_t)ptr % a) == 0; }
 
-// The device address of pinned, device-mapped host memory (null for anything else or when
-// not aligned to `a` bytes).
-const void* mapped_host(const void* p, size_t a) {
-  cudaPointerAttributes at;
-  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+// The device address of `bytes` of pinned, device-mapped host memory at p (null for
+// anything else, when not aligned to `a` bytes, or when the last byte is not mapped at
+// the same offset, i.e. [p, p + bytes) does not lie inside one mapping).
+const void* mapped_host(const void* p, size_t bytes, size_t a) {
+  cudaPointerAttributes at, end;
+  if (bytes == 0 || cudaPointerGetAttributes(&at, p) != cudaSuccess ||
+      cudaPointerGetAttributes(&end, static_cast<const uint8_t*>(p) + bytes - 1) != cudaSuccess) {
     cudaGetLastError();
     return nullptr;
   }
   if (at.type != cudaMemoryTypeHost || !at.devicePointer || !aligned(at.devicePointer, a)) return nullptr;
+  if (end.type != cudaMemoryTypeHost || !end.devicePointer ||
+      static_cast<const uint8_t*>(end.devicePointer) != static_cast<const uint8_t*>(at.devicePointer) + bytes - 1)
+    return nullptr;
   return at.devicePointer;
 }
 
@@ -1707,11 +1712,18 @@ static __device__ __align__(256) uint8_t g_noalloc_scratch[kNoAllocBytes];
 std::mutex g_noalloc_mu;
 void* g_noalloc_addr[kNoAllocMaxDevices] = {};
 
-// Device address of the scratch on `device` (which must be current).
-int noalloc_scratch(int device, void** out) {
+// Device address of the scratch on `device` (which must be current).  The first
+// lookup on a device is refused while `st` is capturing a graph: the symbol lookup
+// is not a stream operation and may initialise the module, so it must happen
+// before any capture.
+int noalloc_scratch(int device, cudaStream_t st, void** out) {
   if (device < 0 || device >= kNoAllocMaxDevices) return BITSMOE_ERR_INVALID_ARG;
   std::lock_guard<std::mutex> lock(g_noalloc_mu);
   if (!g_noalloc_addr[device]) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    const cudaError_t ce = cudaStreamIsCapturing(st, &cs);
+    if (ce != cudaSuccess) return cuda_fail(ce);
+    if (cs != cudaStreamCaptureStatusNone) return BITSMOE_ERR_INVALID_ARG;
     void* p = nullptr;
     const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
     if (e != cudaSuccess || !p) return cuda_fail(e != cudaSuccess ? e : cudaErrorInvalidSymbol);
@@ -1742,8 +1754,17 @@ int bitsmoe_moe_forward_noalloc(const void* x, const float* logits, int T, int t
   int rc = check_device(L);
   if (rc) return rc;
   void* ws = nullptr;
-  if ((rc = noalloc_scratch(L->device, &ws))) return rc;
+  if ((rc = noalloc_scratch(L->device, static_cast<cudaStream_t>(stream), &ws))) return rc;
   return forward_impl(x, logits, T, top_k, L, y, ws, kNoAllocBytes, static_cast<cudaStream_t>(stream));
+}
+
+int bitsmoe_noalloc_last_status(void* stream) {
+  int dev = -1;
+  BM_CK(cudaGetDevice(&dev));
+  void* ws = nullptr;
+  const int rc = noalloc_scratch(dev, static_cast<cudaStream_t>(stream), &ws);
+  if (rc) return rc;
+  return bitsmoe_last_device_status(ws, stream);
 }
 
 int bitsmoe_pack(const bitsmoe_layer_host* src, int device, bitsmoe_layer** out) {
@@ -1871,9 +1892,9 @@ int bitsmoe_moe_forward_host(const void* x_host, const float* logits_host, int T
     // One token on the fused kernel with pinned (device-mapped) host buffers: the kernel reads x
     // and the logits and writes y through the unified address space (the bytes cross the
     // host link inside the kernel), which saves the copy round trips of a few KB.
-    const void* xd = mapped_host(x_host, 16);
-    const void* ld = mapped_host(logits_host, 16);
-    void* yd = const_cast<void*>(mapped_host(y_host, 16));
+    const void* xd = mapped_host(x_host, (size_t)hd.D * 2, 16);
+    const void* ld = mapped_host(logits_host, (size_t)hd.E * 4, 16);
+    void* yd = const_cast<void*>(mapped_host(y_host, (size_t)hd.D * 4, 16));
     if (xd && ld && yd) {
       rc = forward_impl(xd, static_cast<const float*>(ld), T, top_k, L, static_cast<float*>(yd), ws, ws_bytes, st);
       if (rc) return rc;

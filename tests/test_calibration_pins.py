@@ -96,3 +96,33 @@ def test_intermediate_activations_rebuild_the_forward():
         y += g[:, e][:, None] * (Wdn @ C.intermediate(layer, x, e)).T
     ref = oracle.moe_forward_dense(layer, x, logits, spec.top_k)
     np.testing.assert_allclose(y, ref, rtol=1e-9, atol=1e-12 * np.max(np.abs(ref)))
+
+
+def test_float_factor_importance_against_dense_weights():
+    """beta from the decomposition's float factors (before quantisation): for gate/up it is
+    sum_t g_t (phi_k^T x_t)^2, and for down, removing unit k of the float down factor changes
+    the g-weighted output energy by alpha_k^2 beta_k, with the expert's SwiGLU activations
+    taken from the dense float weights themselves (not through the factors)."""
+    rng = np.random.default_rng(12)
+    D, I, E, T, k = 6, 5, 3, 20, 2
+    Wg = [rng.standard_normal((I, D)) for _ in range(E)]
+    Wu = [rng.standard_normal((I, D)) for _ in range(E)]
+    Wd = [rng.standard_normal((D, I)) for _ in range(E)]
+    dec = [oracle.shared_basis_decompose(W, side) for W, side in ((Wg, "in"), (Wu, "in"), (Wd, "out"))]
+    Phi = [d[0] for d in dec]
+    al = [d[1] for d in dec]
+    P = [d[2] for d in dec]
+    x = synth.f32_to_bf16_bits(rng.standard_normal((T, D)).astype(np.float32))
+    logits = rng.standard_normal((T, E)).astype(np.float32)
+    beta = C.factor_importance(Phi, al, P, x, logits, k)
+    g = C.affinities(logits, k, E)
+    X = oracle.bf16_bits_to_f64(x).T
+    for e in range(E):
+        for h in (oracle.GATE, oracle.UP):
+            want = np.sum(g[:, e][None, :] * (Phi[h].T @ X) ** 2, axis=1)
+            np.testing.assert_allclose(beta[h, e], want, rtol=1e-10, atol=1e-12)
+        Hact = oracle.silu(Wg[e] @ X) * (Wu[e] @ X)                       # I x T, dense definition
+        for j in range(Phi[2].shape[1]):
+            dW = al[2][e, j] * np.outer(Phi[2][:, j], P[2][e][:, j])
+            loss = float(np.sum(g[:, e] * np.sum((dW @ Hact) ** 2, axis=0)))
+            assert loss == pytest.approx(al[2][e, j] ** 2 * beta[2, e, j], rel=1e-9, abs=1e-12)

@@ -371,3 +371,31 @@ def test_rms_norm_closed_forms():
     r = oracle.rms_norm(h, 1e-2)
     np.testing.assert_allclose(np.mean(r * r, axis=1), m / (m + 1e-2), rtol=1e-12)
     np.testing.assert_allclose(oracle.rms_norm(7.0 * h, 0.0), oracle.rms_norm(h, 0.0), rtol=1e-12)
+
+
+# --------------------------------------------------------------------------
+# router logits of a stacked block: W_r x with W_r E x D, hand-evaluated
+# --------------------------------------------------------------------------
+def _bf16(vals):
+    """bf16 bit patterns of values that bf16 holds exactly (the top half of their fp32 bits)."""
+    return (np.asarray(vals, dtype=np.float32).view(np.uint32) >> 16).astype(np.uint16)
+
+
+def test_router_logits_hand_values():
+    # one-hot router rows pick coordinates of x: logit e = x[c_e]
+    x = _bf16([[1.0, -2.0, 0.5, 3.0, 0.25], [4.0, 0.0, -0.75, 1.5, 8.0]])
+    pick = [3, 0, 4]
+    W = np.zeros((3, 5), dtype=np.float32)
+    W[np.arange(3), pick] = 1.0
+    got = oracle.router_logits(_bf16(W), x)
+    np.testing.assert_array_equal(got, [[3.0, 1.0, 0.25], [1.5, 4.0, 8.0]])
+    # non-square (E = 2 < D = 4), sums written out by hand
+    W2 = _bf16([[1.0, 2.0, 0.0, 0.0], [0.0, 0.0, -1.0, 0.5]])
+    x2 = _bf16([[1.0, 1.0, 1.0, 1.0], [2.0, 1.0, 4.0, 10.0]])
+    np.testing.assert_array_equal(oracle.router_logits(W2, x2), [[3.0, -0.5], [4.0, 1.0]])
+    # square and not symmetric: a transposed operand gives [1, 3] instead of [3, 1]
+    W3 = _bf16([[1.0, 2.0], [0.0, 1.0]])
+    np.testing.assert_array_equal(oracle.router_logits(W3, _bf16([[1.0, 1.0]])), [[3.0, 1.0]])
+    # the router weights are read as bf16 (0x3F81 = 1 + 2^-7), not rounded or truncated further
+    W4 = np.array([[0x3F81, 0x4040]], dtype=np.uint16)            # 1.0078125, 3.0
+    np.testing.assert_array_equal(oracle.router_logits(W4, _bf16([[2.0, -1.0]])), [[2.015625 - 3.0]])

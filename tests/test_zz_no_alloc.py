@@ -70,3 +70,55 @@ def test_noalloc_rejects_batches_beyond_its_scratch(env):
     with pytest.raises(bm.BitsMoEError) as ei:
         bm.bitsmoe_moe_forward_noalloc(x.data_ptr(), lg.data_ptr(), T, spec.top_k, L, y.data_ptr(), 0)
     assert ei.value.code == bm.ERR_CODE["WORKSPACE_TOO_SMALL"]
+
+
+def test_noalloc_status_word_is_readable(env):
+    """The caller cannot name the scratch, so its device status comes through its own accessor:
+    zero after calls that completed (and it stays cleared on a second read)."""
+    torch, bm = env
+    spec = synth.WORKLOADS["tiny"]
+    layer = synth.make_layer(spec, seed=5)
+    L = bm.bitsmoe_pack(layer, device=0)
+    x, logits = synth.make_inputs(spec, 1, seed=5)
+    xd = torch.from_numpy(x.view(np.int16)).cuda()
+    ld = torch.from_numpy(logits).cuda()
+    y = torch.zeros((1, spec.D), dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream().cuda_stream
+    bm.bitsmoe_moe_forward_noalloc(xd.data_ptr(), ld.data_ptr(), 1, spec.top_k, L, y.data_ptr(), stream)
+    assert bm.bitsmoe_noalloc_last_status(stream) == 0
+    assert bm.bitsmoe_noalloc_last_status(stream) == 0
+
+
+_CAPTURE_FIRST = r"""
+import ctypes, sys
+import numpy as np, torch
+sys.path.insert(0, sys.argv[1])
+import synth, paper_2606_00079_gb300 as bm
+spec = synth.WORKLOADS["tiny"]
+L = bm.bitsmoe_pack(synth.make_layer(spec, seed=6), device=0)
+x = torch.zeros((1, spec.D), dtype=torch.int16, device="cuda")
+lg = torch.zeros((1, spec.E), dtype=torch.float32, device="cuda")
+y = torch.zeros((1, spec.D), dtype=torch.float32, device="cuda")
+s = torch.cuda.Stream()
+torch.cuda.synchronize()
+rc = None
+g = torch.cuda.CUDAGraph()
+try:
+    with torch.cuda.graph(g, stream=s):
+        rc = bm._lib().bitsmoe_moe_forward_noalloc(x.data_ptr(), lg.data_ptr(), 1, spec.top_k, L.handle,
+                                                   y.data_ptr(), ctypes.c_void_p(s.cuda_stream))
+except Exception:
+    pass
+print("RC", rc)
+"""
+
+
+def test_noalloc_first_call_inside_capture_is_refused(env):
+    """A fresh process whose first no-allocation call on the device comes inside a stream
+    capture gets BITSMOE_ERR_INVALID_ARG (the scratch address must be looked up before)."""
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    r = subprocess.run([sys.executable, "-c", _CAPTURE_FIRST, root], capture_output=True, text=True, timeout=300)
+    assert "RC -1" in r.stdout, (r.stdout, r.stderr[-2000:])
