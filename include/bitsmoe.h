@@ -157,8 +157,32 @@ int bitsmoe_forward_launches(const bitsmoe_layer* layer, int T, int top_k);
  *   8  tensor-core gate/up factors (layers without 16-bit gate/up units whose
  *      group is a multiple of 128 rows; otherwise the dp2a kernel)
  *  16  tensor-core down factor (the same condition on the down units)
+ *  32  with 1: the fused kernel is the clustered one, in which a thread-block
+ *      cluster owns one (routing slot, 128-row block) pair of the token and
+ *      its blocks exchange partial gate/up rows through distributed shared
+ *      memory (when the device holds a cluster per pair at once, the layer's
+ *      parts fit in shared memory and the pairs' blocks span at least 90% of
+ *      the SMs; see bitsmoe_debug_single_token_kernel)
  * Returns a negative error code for invalid arguments; 0 for T == 0. */
 int bitsmoe_forward_plan(const bitsmoe_layer* layer, int T, int top_k);
+
+/* Testing hook (no counterpart in the paper): bound every wait of the fused
+ * single-token kernels to `spin_clocks` SM clocks (<= 0: the default, about one
+ * second), and when skip_arrival is 1 let block 0 skip its arrival at the
+ * first grid barrier, so that every other block's bounded wait runs out.  The
+ * calls after it report BITSMOE_ERR_TIMEOUT through the device status word and
+ * return; the workspace is left zeroed for the next call.  Applies to calls
+ * issued after it on any host thread; skip_arrival = 0 with spin_clocks = 0
+ * restores the normal behaviour.  Returns BITSMOE_OK. */
+int bitsmoe_debug_wait_limit(int skip_arrival, long long spin_clocks);
+
+/* Testing hook (no counterpart in the paper): which = 1 keeps single-token
+ * forwards on the fused kernel without clusters, which = 2 takes the clustered
+ * one wherever the device and the layer fit it (bitsmoe_forward_plan reports
+ * which), so that tests cover both fused kernels on the same cases; which = 0
+ * restores the automatic choice.  Applies to calls issued after it.  Returns
+ * BITSMOE_OK, or BITSMOE_ERR_INVALID_ARG for another value. */
+int bitsmoe_debug_single_token_kernel(int which);
 
 /* Kernels one bitsmoe_moe_block_forward call launches: 1 a token when the
  * fused single-token kernel runs (it computes the pre-norm and router too),

@@ -76,6 +76,8 @@ SIGNATURES = {
     "bitsmoe_free": (None, [_P]),
     "bitsmoe_strerror": (ctypes.c_char_p, [_I]),
     "bitsmoe_last_cuda_error": (_I, []),
+    "bitsmoe_debug_wait_limit": (_I, [_I, ctypes.c_longlong]),
+    "bitsmoe_debug_single_token_kernel": (_I, [_I]),
 }
 
 
@@ -248,11 +250,12 @@ def bitsmoe_forward_launches(layer: Layer, T: int, top_k: int) -> int:
 
 
 PLAN_FUSED, PLAN_DECODE_CHAIN, PLAN_TC_PROJECTIONS, PLAN_TC_GATE_UP, PLAN_TC_DOWN = 1, 2, 4, 8, 16
+PLAN_CLUSTERED = 32
 
 
 def bitsmoe_forward_plan(layer: Layer, T: int, top_k: int) -> int:
     """Bit set of how a T-token forward runs: PLAN_FUSED, PLAN_DECODE_CHAIN, PLAN_TC_PROJECTIONS,
-    PLAN_TC_GATE_UP, PLAN_TC_DOWN."""
+    PLAN_TC_GATE_UP, PLAN_TC_DOWN, PLAN_CLUSTERED (with PLAN_FUSED: the clustered single-token kernel)."""
     n = int(_lib().bitsmoe_forward_plan(layer.handle, T, top_k))
     if n < 0:
         raise BitsMoEError(n, "bitsmoe_forward_plan")
@@ -431,3 +434,14 @@ def allocate_bits(p, alpha, beta, gamma: float, kappa, budget: int, stream=None)
     ws.record_stream(st)   # the workspace is freed here but used by the kernels still queued on st
     return bits
 
+
+def bitsmoe_debug_single_token_kernel(which: int) -> None:
+    """Testing hook: 1 keeps single-token forwards on the fused kernel without clusters, 2 takes the
+    clustered one wherever it fits, 0 restores the automatic choice."""
+    _check(_lib().bitsmoe_debug_single_token_kernel(which), "bitsmoe_debug_single_token_kernel")
+
+
+def bitsmoe_debug_wait_limit(skip_arrival: int, spin_clocks: int) -> None:
+    """Testing hook: bound the fused kernels' waits to spin_clocks SM clocks (0: default) and let
+    block 0 skip its first grid-barrier arrival (skip_arrival = 1)."""
+    _check(_lib().bitsmoe_debug_wait_limit(skip_arrival, spin_clocks), "bitsmoe_debug_wait_limit")

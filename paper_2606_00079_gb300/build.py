@@ -1,8 +1,9 @@
 """Build libbitsmoe.so in-tree with nvcc for sm_103a (GB300).
 
-Seven translation units, compiled in parallel: the host packer (pack.cpp,
-plain C++), the CUDA kernel chain + C ABI (forward.cu), the fused
-single-token decode kernel (fused.cu), the tensor-core projections
+Eight translation units, compiled in parallel: the host packer (pack.cpp,
+plain C++), the CUDA kernel chain + C ABI (forward.cu), the two fused
+single-token decode kernels (fused.cu, and the clustered one in fused2.cu),
+the tensor-core projections
 (gemm.cu), the tensor-core expert factors (expert_tc.cu), the per-unit
 quantiser from float spectral vectors (quantize.cu) and the per-projection
 bit allocation (allocate.cu).  The CUDA runtime is linked
@@ -40,8 +41,8 @@ def _run(cmd):
 
 
 def sources():
-    return [os.path.join(CSRC, f) for f in ("pack.cpp", "forward.cu", "fused.cu", "gemm.cu", "expert_tc.cu", "quantize.cu",
-                                              "allocate.cu")]
+    return [os.path.join(CSRC, f) for f in ("pack.cpp", "forward.cu", "fused.cu", "fused2.cu", "gemm.cu", "expert_tc.cu",
+                                              "quantize.cu", "allocate.cu")]
 
 
 def up_to_date() -> bool:

@@ -94,6 +94,92 @@ struct FusedArgs {
   int nslot_c, slot_c, nslot_d, slot_d; // gate/up and down staging slots (count, bytes)
   int off_route, off_xs, off_r1, off_d, off_rc, off_cq, off_rec, off_part, smem;
   int smax, s16, seg_al, ul_max_tiles, d_code_bytes, d_h_bytes;
+  int dbg;             // bit 0: block 0 skips its arrival at grid barrier 1 (tests of the bounded waits)
+  long long spin;      // bound of the grid-barrier waits, in SM clocks
+};
+
+// Records of the clustered single-token kernel (fused2.cu), derived at upload for
+// each cluster size CL: the tiles of every (projection, expert) are cut into CL
+// contiguous parts of about equal code bytes, and cluster rank r works on part r.
+struct F2Gu {              // gate/up part r of (h, e): a run of row-lane tiles
+  uint64_t code0;          // image offset of the part's codes in row block 0
+  uint64_t unit0, alpha0;  // image offsets of its first slot's unit index and alpha
+  uint64_t sz0;            // image offset of its first slot's scale/zero in group row 0
+  uint32_t rb_stride;      // bytes between row blocks of the code stream
+  uint32_t sz_row;         // bytes between group rows of the scale/zero matrix
+  uint32_t bytes;          // code bytes per row block (0: empty part)
+  uint32_t nslot;          // slots (a multiple of 4)
+  uint8_t nr;              // buckets the part touches
+  uint8_t bits[kNumBk];    // their bit-widths (ascending; 16 last)
+  uint16_t ntl[kNumBk];    // tiles per touched bucket
+  uint8_t pad_[10];
+};
+static_assert(sizeof(F2Gu) == 80, "F2Gu layout");
+
+struct F2Dn {              // down part r of e: a run of unit-lane tiles
+  uint64_t code[kNumBk];   // per touched bucket: image offset of its first part tile in row block 0
+  uint64_t unit0, alpha0;  // image offsets of the part's first slot's unit index and alpha
+  uint64_t sz0;            // image offset of its first slot's scale/zero in group row 0
+  uint32_t sz_row;         // bytes between group rows
+  uint32_t nslot;          // slots (32 per tile; 0: empty part)
+  uint8_t nr;
+  uint8_t bits[kNumBk];
+  uint16_t ntl[kNumBk];
+  uint8_t pad_[2];
+};
+static_assert(sizeof(F2Dn) == 112, "F2Dn layout");
+
+// Warps of the clustered kernel per gate/up projection in the factor phase.
+constexpr int kF2GuWarps = 8;
+
+// Tile index at which warp w of nw starts on a run of row-lane tiles (buckets
+// bits[0..nr), ntl tiles each): the first tile whose code-byte prefix reaches
+// w/nw of the run's bytes.  The host sizes the activation tables with it.
+__host__ __device__ inline int rl_split_at(const uint8_t* bits, const uint16_t* ntl, int nr, int w, int nw) {
+  // in 512-byte chunks (a part stays far below 2^32 bytes), 32-bit arithmetic only
+  uint32_t tot = 0;
+  int nt = 0;
+  for (int k = 0; k < nr; ++k) {
+    tot += (uint32_t)ntl[k] * (uint32_t)rl_chunks(bits[k]);
+    nt += ntl[k];
+  }
+  if (w <= 0) return 0;
+  if (w >= nw) return nt;
+  const uint32_t target = (tot * (uint32_t)w + (uint32_t)nw - 1) / (uint32_t)nw;   // ceil: first chunk at or past w/nw
+  uint32_t pre = 0;
+  int t = 0;
+  for (int k = 0; k < nr; ++k) {
+    const uint32_t cb = (uint32_t)rl_chunks(bits[k]);
+    const uint32_t end = pre + (uint32_t)ntl[k] * cb;
+    if (end >= target) return t + (int)(target > pre ? (target - pre + cb - 1) / cb : 0);
+    pre = end;
+    t += ntl[k];
+  }
+  return nt;
+}
+
+// Launch plan of the clustered kernel (fused2.cu).
+struct F2Args {
+  uint32_t* cnt;           // grid-barrier counters (workspace)
+  const uint8_t* tab;      // records of this cluster size: per rank [gate E][up E][down E]
+  uint32_t rank_bytes;     // bytes of one rank's records
+  int CL, npairs;          // cluster size; (routing slot, row block) pairs, one per cluster
+  int b_per, e_per;         // input- and output-basis rows of a pair block
+  int b_free, e_free;       // the same for the other blocks (they stream no expert part)
+  int b_stage, b_nst;       // input-basis rows per stage, stages
+  int s16;                 // int16 activation table row (elements) per warp and group
+  int off_rec, off_route, off_xs, off_cq, off_pw, off_xch, off_h, off_r1, off_d, off_r2, off_ss, smem;
+  int dbg;                 // bit 0: block 0 skips its arrival at grid barrier 1 (tests of the bounded waits)
+  int prefetch_io;         // x and the logits are device memory: prefetch them into L2 before the wait
+  int rec_smem;            // this rank's record table fits the gate/up staging area (copied there first)
+  long long spin;          // bound of every wait, in SM clocks
+};
+
+// Sizes of a layer's clustered-kernel parts for one cluster size (host side).
+struct F2Sizes {
+  int gu_stage;            // most shared-memory bytes of one block's staged gate + up part
+  int dn_stage;            // most bytes of one block's staged down part
+  int s16;                 // most quantised slots of one warp's share of a gate/up part
 };
 
 // Shared-memory plan of the fused kernel for this layer, or false when the
@@ -119,6 +205,17 @@ cudaError_t launch_dn_tc(const Fwd& p, int ul_max_tiles, cudaStream_t st, bool p
 cudaError_t launch_h_pack(const Fwd& p, cudaStream_t st, bool pdl);
 // Staging records of a packed image (host side, at upload).
 void build_stage_tables(const uint8_t* img, std::vector<CStage>& cst, std::vector<DStage>& dst);
+// Records of the clustered kernel for cluster size CL (host side, at upload):
+// per rank r, [F2Gu gate E][F2Gu up E][F2Dn E]; and the largest staged sizes.
+// False when a record would reach outside the image (the kernel is then not used).
+bool build_f2_tables(const uint8_t* img, int CL, std::vector<uint8_t>& out, F2Sizes* sizes);
+// Most clusters of CL blocks of the clustered kernel that can be resident at once
+// (1 block per SM), or 0.
+int f2_max_clusters(int G, int CL);
+// Shared-memory plan of the clustered kernel, or false when the layer does not fit it.
+bool f2_plan(const ImageHeader& hd, int top_k, int CL, int nclusters, const F2Sizes& sz, F2Args* f);
+// The clustered kernel on `st` (grid = nclusters x CL blocks).
+cudaError_t launch_f2(const Fwd& p, const F2Args& f, int nclusters, cudaStream_t st, bool pdl);
 
 }  // namespace bmoe
 

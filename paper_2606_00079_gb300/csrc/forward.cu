@@ -59,6 +59,17 @@ struct bitsmoe_layer {
   std::vector<uint8_t> meta;   // host copy of header + descriptors + segment table
   int seg_bytes = 0;           // largest gate/up item: code bytes inside one row block
   int ul_max_chunks = 1;       // largest 16-byte chunks per row block of any down unit
+  // clustered single-token kernel: records per cluster size (kF2Sizes), the most
+  // clusters of that size that fit the device at once, the staged sizes
+  uint8_t* d_f2 = nullptr;
+  uint64_t f2_off[5] = {};
+  int f2_nc[5] = {};
+  F2Sizes f2_sz[5] = {};
+  // the clustered kernel's plan per top_k (1..32), computed on first use
+  mutable std::mutex f2_mu;
+  mutable signed char f2_ci[33];
+  mutable F2Args f2_args[33];
+  bitsmoe_layer() { std::memset(f2_ci, 0x7F, sizeof(f2_ci)); }
   const ImageHeader& hd() const { return *reinterpret_cast<const ImageHeader*>(meta.data()); }
   const ExpertDesc* desc() const {
     return reinterpret_cast<const ExpertDesc*>(meta.data() + hd().off_desc);
@@ -66,6 +77,18 @@ struct bitsmoe_layer {
 };
 
 namespace {
+
+// Cluster sizes of the clustered single-token kernel, largest first (index into
+// bitsmoe_layer's f2_* arrays).
+constexpr int kF2Sizes[5] = {8, 4, 3, 2, 1};
+
+// Testing hook (bitsmoe_debug_wait_limit): bound of the single-token kernels' waits
+// and whether block 0 skips its arrival at their first grid barrier.
+std::atomic<long long> g_dbg_spin{0};
+std::atomic<int> g_dbg_skip{0};
+// Testing hook (bitsmoe_debug_single_token_kernel): 1 keeps single-token forwards on the
+// kernel without clusters, 2 takes the clustered one wherever it fits.
+std::atomic<int> g_dbg_kernel{0};
 
 thread_local int g_last_cuda = 0;
 int cuda_fail(cudaError_t e) {
@@ -1429,9 +1452,34 @@ bool fused_fits(const bitsmoe_layer* L, int top_k) {
   return decode_mode(hd, 1) && fused_plan(hd, 1, top_k, L->seg_bytes, L->ul_max_chunks, s16, L->num_sms, &fa);
 }
 
+// The clustered single-token plan for this layer and top_k: the index of its cluster
+// size in kF2Sizes (the largest whose co-resident clusters hold one (routing slot, row
+// block) pair each and whose shared-memory plan fits), or -1.
+// Taken automatically only where its expert phase spans at least 90% of the SMs: with
+// fewer, the blocks that hold pairs carry the whole factor work and the kernel without
+// clusters (which deals that work over every block) is faster (Qwen3-shaped layer on 152
+// SMs: 48 pairs fit clusters of 2 but not of 3, so 96 blocks: 24.8 against 23.1 us).
+int f2_choose(const bitsmoe_layer* L, int top_k, F2Args* fa) {
+  const int dbg = g_dbg_kernel.load();
+  if (top_k < 1 || top_k > 32 || dbg == 1) return -1;
+  std::lock_guard<std::mutex> lock(L->f2_mu);
+  if (L->f2_ci[top_k] == 0x7F) {
+    const ImageHeader& hd = L->hd();
+    int ci = -1;
+    for (int i = 0; i < 5 && ci < 0; ++i)
+      if (L->f2_nc[i] > 0 && f2_plan(hd, top_k, kF2Sizes[i], L->f2_nc[i], L->f2_sz[i], &L->f2_args[top_k])) ci = i;
+    L->f2_ci[top_k] = (signed char)ci;
+  }
+  const int ci = L->f2_ci[top_k];
+  if (ci < 0) return -1;
+  *fa = L->f2_args[top_k];
+  if (dbg != 2 && 10 * fa->npairs * fa->CL < 9 * L->num_sms) return -1;
+  return ci;
+}
+
 int forward_impl(const void* x, const float* logits, int T, int top_k, const bitsmoe_layer* L, float* y,
                  void* ws, size_t ws_bytes, cudaStream_t st, cudaEvent_t* ev = nullptr, bool accum = false,
-                 const NormArgs* norm = nullptr) {
+                 const NormArgs* norm = nullptr, bool host_io = false) {
   const ImageHeader& hd = L->hd();
   if (T > 1 && T <= kFusedMaxTokens && fused_fits(L, top_k)) {
     // a few tokens: one fused forward each, on the same workspace (profiled as one phase)
@@ -1505,10 +1553,30 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
     return BITSMOE_OK;
   };
   const int G = std::max(1, kRows / hd.group);
+  if (T == 1 && !norm) {   // one token: the clustered kernel when the layer fits it
+    F2Args f2;
+    const int ci = f2_choose(L, top_k, &f2);
+    if (ci >= 0) {
+      f2.cnt = reinterpret_cast<uint32_t*>(wb + w.sync);
+      f2.tab = L->d_f2 + L->f2_off[ci];
+      f2.dbg = g_dbg_skip.load();
+      f2.prefetch_io = host_io ? 0 : 1;   // no L2 prefetch of host memory mapped into the address space
+      const long long sp = g_dbg_spin.load();
+      if (sp > 0) f2.spin = sp;
+      if ((rc = mark(0))) return rc;
+      const cudaError_t e = launch_f2(p, f2, L->f2_nc[ci], st, pdl);
+      if (e != cudaSuccess) return cuda_fail(e);
+      for (int i = 1; i <= 5; ++i)
+        if ((rc = mark(i))) return rc;
+      return BITSMOE_OK;
+    }
+  }
   FusedArgs fa;
   if (p.decode && fused_plan(hd, T, top_k, L->seg_bytes, L->ul_max_chunks, p.s16, sms, &fa)) {
     // one token: the whole layer in one persistent kernel
     fa.cnt = reinterpret_cast<uint32_t*>(wb + w.sync);
+    fa.dbg = g_dbg_skip.load();
+    if (g_dbg_spin.load() > 0) fa.spin = g_dbg_spin.load();
     fa.cst = L->d_cst;
     fa.dst = L->d_dst;
     fa.tab_bytes = L->stage_bytes;
@@ -1632,24 +1700,51 @@ int upload(std::vector<uint8_t>&& img, int device, bitsmoe_layer** out) {
   std::vector<DStage> dst;
   build_stage_tables(img.data(), cst, dst);
   const size_t cst_bytes = cst.size() * sizeof(CStage), dst_bytes = dst.size() * sizeof(DStage);
+  // records of the clustered single-token kernel for every cluster size, one buffer
+  std::vector<uint8_t> f2all;
+  uint64_t f2_off[5] = {};
+  int f2_nc[5] = {};
+  F2Sizes f2_sz[5] = {};
+  {
+    const int G = std::max(1, kRows / header_of(img.data())->group);
+    for (int i = 0; i < 5; ++i) {
+      std::vector<uint8_t> t;
+      const bool ok = build_f2_tables(img.data(), kF2Sizes[i], t, &f2_sz[i]);
+      f2_off[i] = f2all.size();
+      f2all.insert(f2all.end(), t.begin(), t.end());
+      f2all.resize(align_up(f2all.size(), 256), 0);
+      if (e == cudaSuccess && ok) f2_nc[i] = f2_max_clusters(G, kF2Sizes[i]);
+    }
+  }
   uint8_t* d = nullptr;
   uint8_t* ds = nullptr;
+  uint8_t* df2 = nullptr;
   if (e == cudaSuccess) e = cudaMalloc(&d, img.size());
   if (e == cudaSuccess) e = cudaMemcpy(d, img.data(), img.size(), cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMalloc(&ds, cst_bytes + dst_bytes + 16);
   if (e == cudaSuccess && cst_bytes) e = cudaMemcpy(ds, cst.data(), cst_bytes, cudaMemcpyHostToDevice);
   if (e == cudaSuccess && dst_bytes) e = cudaMemcpy(ds + cst_bytes, dst.data(), dst_bytes, cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMalloc(&df2, f2all.size() + 16);
+  if (e == cudaSuccess && !f2all.empty()) e = cudaMemcpy(df2, f2all.data(), f2all.size(), cudaMemcpyHostToDevice);
   cudaSetDevice(prev);
   if (e != cudaSuccess) {
     if (d) cudaFree(d);
     if (ds) cudaFree(ds);
+    if (df2) cudaFree(df2);
     return e == cudaErrorMemoryAllocation ? BITSMOE_ERR_OOM : cuda_fail(e);
   }
   bitsmoe_layer* L = new (std::nothrow) bitsmoe_layer;
   if (!L) {
     cudaFree(d);
     cudaFree(ds);
+    cudaFree(df2);
     return BITSMOE_ERR_OOM;
+  }
+  L->d_f2 = df2;
+  for (int i = 0; i < 5; ++i) {
+    L->f2_off[i] = f2_off[i];
+    L->f2_nc[i] = f2_nc[i];
+    L->f2_sz[i] = f2_sz[i];
   }
   L->d_stage = ds;
   L->d_cst = reinterpret_cast<const CStage*>(ds);
@@ -1824,11 +1919,18 @@ int bitsmoe_expert_moved_bytes(const bitsmoe_layer* L, int e, uint64_t out[3]) {
   return BITSMOE_OK;
 }
 
-int bitsmoe_forward_launches(const bitsmoe_layer* L, int T, int top_k) {
+}  // extern "C"
+
+namespace {
+// Kernels one forward launches; allow_f2: the plain forward (the pre-norm block
+// forward does not take the clustered kernel).
+int forward_launches(const bitsmoe_layer* L, int T, int top_k, bool allow_f2) {
   if (!L || T < 0) return BITSMOE_ERR_INVALID_ARG;
   const ImageHeader& hd = L->hd();
   if (top_k < 1 || top_k > std::min(hd.E, 32)) return BITSMOE_ERR_INVALID_ARG;
   if (T == 0) return 0;
+  F2Args f2;
+  if (allow_f2 && T == 1 && f2_choose(L, top_k, &f2) >= 0) return 1;
   const bool decode = decode_mode(hd, T);
   FusedArgs fa;
   const int s16 = (int)align_up(std::max(hd.seg_max_slots, 8), 64) + 8;
@@ -1837,10 +1939,17 @@ int bitsmoe_forward_launches(const bitsmoe_layer* L, int T, int top_k) {
   if (decode || !L->maps) return 5;
   return 3 + (L->tcx ? 2 : 1) + (L->tcd ? 3 : 1);   // router, projection, gate/up, [h pack,] down, output basis
 }
+}  // namespace
+
+extern "C" {
+
+int bitsmoe_forward_launches(const bitsmoe_layer* L, int T, int top_k) { return forward_launches(L, T, top_k, true); }
 
 int bitsmoe_forward_plan(const bitsmoe_layer* L, int T, int top_k) {
   const int n = bitsmoe_forward_launches(L, T, top_k);
   if (n <= 0) return n;
+  F2Args f2;
+  if (T <= kFusedMaxTokens && (T == 1 || fused_fits(L, top_k)) && f2_choose(L, top_k, &f2) >= 0) return 1 | 32;
   if (T <= kFusedMaxTokens && fused_fits(L, top_k)) return 1;
   const ImageHeader& hd = L->hd();
   if (decode_mode(hd, T)) return 2 | (L->maps && T >= 4 ? 4 : 0);
@@ -1848,7 +1957,7 @@ int bitsmoe_forward_plan(const bitsmoe_layer* L, int T, int top_k) {
 }
 
 int bitsmoe_block_forward_launches(const bitsmoe_layer* L, int T, int top_k) {
-  const int n = bitsmoe_forward_launches(L, T, top_k);
+  const int n = forward_launches(L, T, top_k, false);
   if (n > 0 && T <= kFusedMaxTokens && fused_fits(L, top_k)) return n;   // the fused kernels norm in place
   return n > 1 ? n + 1 : n;
 }
@@ -1896,7 +2005,8 @@ int bitsmoe_moe_forward_host(const void* x_host, const float* logits_host, int T
     const void* ld = mapped_host(logits_host, (size_t)hd.E * 4, 16);
     void* yd = const_cast<void*>(mapped_host(y_host, (size_t)hd.D * 4, 16));
     if (xd && ld && yd) {
-      rc = forward_impl(xd, static_cast<const float*>(ld), T, top_k, L, static_cast<float*>(yd), ws, ws_bytes, st);
+      rc = forward_impl(xd, static_cast<const float*>(ld), T, top_k, L, static_cast<float*>(yd), ws, ws_bytes, st,
+                        nullptr, false, nullptr, true);
       if (rc) return rc;
       BM_CK(cudaStreamSynchronize(st));
       return BITSMOE_OK;
@@ -1999,11 +2109,24 @@ void bitsmoe_free(bitsmoe_layer* L) {
     cudaSetDevice(L->device);
     cudaFree(L->d_img);
     cudaFree(L->d_stage);
+    cudaFree(L->d_f2);
     cudaSetDevice(prev);
   }
   delete L;
 }
 
 int bitsmoe_last_cuda_error(void) { return g_last_cuda; }
+
+int bitsmoe_debug_single_token_kernel(int which) {
+  if (which < 0 || which > 2) return BITSMOE_ERR_INVALID_ARG;
+  g_dbg_kernel.store(which);
+  return BITSMOE_OK;
+}
+
+int bitsmoe_debug_wait_limit(int skip_arrival, long long spin_clocks) {
+  g_dbg_skip.store(skip_arrival ? 1 : 0);
+  g_dbg_spin.store(spin_clocks > 0 ? spin_clocks : 0);
+  return BITSMOE_OK;
+}
 
 }  // extern "C"

@@ -19,8 +19,10 @@ TOL = 2e-3
 ALL_BITS = {0: 0.1, 1: 0.15, 2: 0.2, 3: 0.15, 4: 0.1, 6: 0.1, 8: 0.1, 16: 0.1}
 
 
-@pytest.fixture(scope="module")
-def env():
+@pytest.fixture(scope="module", params=["clustered", "plain"])
+def env(request):
+    """Every case runs on both single-token kernels, each forced through the testing hook: the
+    clustered one and the one without clusters."""
     torch = pytest.importorskip("torch")
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
@@ -28,7 +30,9 @@ def env():
     __graft_entry__.build()
     import paper_2606_00079_gb300 as bm
     torch.cuda.set_device(0)
-    return torch, bm
+    bm.bitsmoe_debug_single_token_kernel(1 if request.param == "plain" else 2)
+    yield torch, bm, request.param
+    bm.bitsmoe_debug_single_token_kernel(0)
 
 
 def rel_err(y, ref):
@@ -42,8 +46,10 @@ def small(**kw):
 
 
 def run(env, L, x, logits, k, ws=None):
-    torch, bm = env
+    torch, bm, kern = env
     assert bm.bitsmoe_forward_launches(L, x.shape[0], k) == 1, "fused path not taken"
+    plan = bm.bitsmoe_forward_plan(L, x.shape[0], k)
+    assert plan == bm.PLAN_FUSED | (bm.PLAN_CLUSTERED if kern == "clustered" else 0), plan
     xd = torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).cuda()
     ld = torch.from_numpy(np.ascontiguousarray(logits)).cuda()
     if ws is None:
@@ -54,8 +60,18 @@ def run(env, L, x, logits, k, ws=None):
     return y.cpu().numpy().astype(np.float64)
 
 
+def plain_forward(bm, L, x, lg, k, ws, kern):
+    """The forward on the fused kernel without clusters (the one pre-norm blocks use), so that
+    a block's update can be compared with it up to the order of float atomics."""
+    bm.bitsmoe_debug_single_token_kernel(1)
+    try:
+        return bm.moe_forward(L, x, lg, k, ws=ws)
+    finally:
+        bm.bitsmoe_debug_single_token_kernel(1 if kern == "plain" else 2)
+
+
 def check(env, layer, x, logits, k, L=None, ws=None):
-    torch, bm = env
+    torch, bm, _ = env
     L = L or bm.bitsmoe_pack(layer, device=0)
     y = run(env, L, x, logits, k, ws)
     ref = oracle.moe_forward_factored(layer, x, logits, k)
@@ -97,7 +113,7 @@ def test_fused_top1_and_all_experts(env):
     layer = synth.make_layer(spec, seed=9, bits_dist=ALL_BITS, alpha_scale=3.0)
     x, _ = synth.make_inputs(spec, 1, seed=9)
     logits = np.array([[1.0, 2.0, 2.0, -1.0, 2.0, 0.0]], np.float32)   # ties
-    torch, bm = env
+    torch, bm, kern = env
     L = bm.bitsmoe_pack(layer, device=0)
     for k in (1, 2, spec.E):
         check(env, layer, x, logits, k, L=L)
@@ -113,14 +129,14 @@ def test_fused_routing_ties_many_experts(env, E):
     rng = np.random.default_rng(E)
     logits = rng.integers(-2, 3, size=(1, E)).astype(np.float32)
     logits[0, rng.integers(0, E, size=4)] = -0.0
-    torch, bm = env
+    torch, bm, kern = env
     L = bm.bitsmoe_pack(layer, device=0)
     for k in (1, 8, 32):
         check(env, layer, x, logits, k, L=L)
 
 
 def test_fused_consecutive_calls_layers_and_workspace_state(env):
-    torch, bm = env
+    torch, bm, kern = env
     spec = synth.scaled_spec(synth.WORKLOADS["qw3"], D=512, E=32, I=384, n=512, top_k=4)
     layers = [synth.make_layer(spec, seed=s) for s in (21, 22)]
     Ls = [bm.bitsmoe_pack(l, device=0) for l in layers]
@@ -153,7 +169,7 @@ def test_fused_consecutive_calls_layers_and_workspace_state(env):
 
 
 def test_fused_graph_replay(env):
-    torch, bm = env
+    torch, bm, kern = env
     spec = synth.scaled_spec(synth.WORKLOADS["qw3"], D=512, E=32, I=384, n=512, top_k=4)
     layer = synth.make_layer(spec, seed=31)
     L = bm.bitsmoe_pack(layer, device=0)
@@ -182,7 +198,7 @@ def test_fused_graph_replay(env):
 
 
 def test_fused_plan_taken_for_qw3_dims_not_for_d4096(env):
-    torch, bm = env
+    torch, bm, kern = env
     qw3 = synth.scaled_spec(synth.WORKLOADS["qw3"], E=8, top_k=8)   # full qw3 dims, fewer experts
     L = bm.bitsmoe_pack(synth.make_layer(qw3, seed=1), device=0)
     assert bm.bitsmoe_forward_launches(L, 1, 8) == 1
@@ -201,7 +217,7 @@ def test_block_forward_fused_norm(env, E, top_k):
     rows on some blocks).  Its update must match the two-step path
     (norm/router kernel, then the forward) up to the order of the float
     atomics, and the oracle's MoE on the same x and logits."""
-    torch, bm = env
+    torch, bm, kern = env
     spec = small(E=E, top_k=top_k, n=72)
     layer = synth.make_layer(spec, seed=5)
     L = bm.bitsmoe_pack(layer, device=0)
@@ -215,7 +231,7 @@ def test_block_forward_fused_norm(env, E, top_k):
     x = torch.empty((1, spec.D), dtype=torch.int16, device="cuda")
     lg = torch.empty((1, spec.E), dtype=torch.float32, device="cuda")
     bm.bitsmoe_rmsnorm_router(h0.data_ptr(), wr.data_ptr(), eps, 1, spec.D, spec.E, x.data_ptr(), lg.data_ptr(), st)
-    y2 = bm.moe_forward(L, x, lg, top_k, ws=ws)
+    y2 = plain_forward(bm, L, x, lg, top_k, ws, kern)   # the block runs on the kernel without clusters too
     torch.cuda.synchronize()
     for rep in range(3):   # the same workspace, repeatedly
         h = h0.clone()
@@ -235,12 +251,13 @@ def test_block_forward_fused_norm(env, E, top_k):
 def test_few_tokens_as_fused_forwards(env, T):
     """Two to four tokens run as one fused forward per token on one workspace: plain and
     as a pre-norm block (norm mode), against the oracle and the two-step path."""
-    torch, bm = env
+    torch, bm, kern = env
     spec = small(E=8, top_k=3, n=72)
     layer = synth.make_layer(spec, seed=30 + T, alpha_scale=3.0)
     L = bm.bitsmoe_pack(layer, device=0)
     assert bm.bitsmoe_forward_launches(L, T, spec.top_k) == T
-    assert bm.bitsmoe_forward_plan(L, T, spec.top_k) == bm.PLAN_FUSED
+    assert bm.bitsmoe_forward_plan(L, T, spec.top_k) == bm.PLAN_FUSED | (
+        bm.PLAN_CLUSTERED if kern == "clustered" else 0)
     x, logits = synth.make_inputs(spec, T, seed=30 + T)
     ws = bm.Workspace(L, T, spec.top_k)
     y = bm.moe_forward(L, torch.from_numpy(x.view(np.int16)).cuda(), torch.from_numpy(logits).cuda(), spec.top_k,
@@ -256,7 +273,7 @@ def test_few_tokens_as_fused_forwards(env, T):
     xb = torch.empty((T, spec.D), dtype=torch.int16, device="cuda")
     lg = torch.empty((T, spec.E), dtype=torch.float32, device="cuda")
     bm.bitsmoe_rmsnorm_router(h0.data_ptr(), wr.data_ptr(), 1e-6, T, spec.D, spec.E, xb.data_ptr(), lg.data_ptr(), st)
-    y2 = bm.moe_forward(L, xb, lg, spec.top_k, ws=ws)
+    y2 = plain_forward(bm, L, xb, lg, spec.top_k, ws, kern)
     h = h0.clone()
     bm.bitsmoe_moe_block_forward(h.data_ptr(), wr.data_ptr(), 1e-6, T, spec.top_k, L, ws.ptr, ws.nbytes, st)
     torch.cuda.synchronize()
@@ -264,3 +281,41 @@ def test_few_tokens_as_fused_forwards(env, T):
     two_step = (h0 + y2).cpu().numpy().astype(np.float64)
     ymax, hmax = float(y2.abs().max()), float(h0.abs().max())
     assert np.max(np.abs(h.cpu().numpy() - two_step)) <= 1e-5 * ymax + 2.4e-7 * hmax
+
+
+def test_bounded_wait_runs_out_and_is_reported(env):
+    """Block 0 skips its arrival at the first grid barrier (testing hook) and every wait is
+    bounded to about a millisecond: the kernel returns, the status word reports TIMEOUT (no
+    trap, the context stays usable), and the next call on the same workspace is correct."""
+    torch, bm, kern = env
+    spec = small(E=8, top_k=2, n=72)
+    layer = synth.make_layer(spec, seed=40)
+    L = bm.bitsmoe_pack(layer, device=0)
+    ws = bm.Workspace(L, 1, spec.top_k)
+    x, logits = synth.make_inputs(spec, 1, seed=40)
+    xd = torch.from_numpy(x.view(np.int16)).cuda()
+    ld = torch.from_numpy(logits).cuda()
+    bm.bitsmoe_debug_wait_limit(1, 2_000_000)
+    try:
+        bm.moe_forward(L, xd, ld, spec.top_k, ws=ws)
+        torch.cuda.synchronize()
+    finally:
+        bm.bitsmoe_debug_wait_limit(0, 0)
+    assert bm.bitsmoe_last_device_status(ws.ptr) == bm.ERR_CODE["TIMEOUT"]
+    assert bm.bitsmoe_last_device_status(ws.ptr) == 0          # read and cleared
+    check(env, layer, x, logits, spec.top_k, L=L, ws=ws)       # the counters were left at zero
+
+
+def test_clustered_plan_for_qw3_dims(env):
+    """The Qwen3-shaped layer (full dims, top-8) runs on the clustered kernel at one token when
+    it is forced (the device holds a cluster per (routing slot, row block) pair) and on the
+    other one; both match the oracle."""
+    torch, bm, kern = env
+    spec = synth.scaled_spec(synth.WORKLOADS["qw3"], E=16, top_k=8)
+    layer = synth.make_layer(spec, seed=41)
+    L = bm.bitsmoe_pack(layer, device=0)
+    plan = bm.bitsmoe_forward_plan(L, 1, 8)
+    assert plan == bm.PLAN_FUSED | (bm.PLAN_CLUSTERED if kern == "clustered" else 0), plan
+    for step in range(2):
+        x, logits = synth.make_inputs(spec, 1, seed=41, step=step)
+        check(env, layer, x, logits, 8, L=L)

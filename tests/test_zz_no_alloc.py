@@ -122,3 +122,33 @@ def test_noalloc_first_call_inside_capture_is_refused(env):
     root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
     r = subprocess.run([sys.executable, "-c", _CAPTURE_FIRST, root], capture_output=True, text=True, timeout=300)
     assert "RC -1" in r.stdout, (r.stdout, r.stderr[-2000:])
+
+
+def test_noalloc_status_reports_a_timeout(env):
+    """A no-allocation call whose bounded wait runs out (testing hook: block 0 skips its first
+    grid-barrier arrival) reports TIMEOUT through the no-allocation status accessor, and the
+    next call on the shared scratch is correct again."""
+    torch, bm = env
+    lib = bm._lib()
+    spec = synth.WORKLOADS["tiny"]
+    layer = synth.make_layer(spec, seed=7)
+    L = bm.bitsmoe_pack(layer, device=0)
+    x, logits = synth.make_inputs(spec, 1, seed=7)
+    xd = torch.from_numpy(x.view(np.int16)).cuda()
+    ld = torch.from_numpy(logits).cuda()
+    y = torch.zeros((1, spec.D), dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream().cuda_stream
+    bm.bitsmoe_debug_wait_limit(1, 2_000_000)
+    try:
+        bm.bitsmoe_moe_forward_noalloc(xd.data_ptr(), ld.data_ptr(), 1, spec.top_k, L, y.data_ptr(), stream)
+        torch.cuda.synchronize()
+    finally:
+        bm.bitsmoe_debug_wait_limit(0, 0)
+    assert bm.bitsmoe_noalloc_last_status(stream) == bm.ERR_CODE["TIMEOUT"]
+    y_ref = bm.moe_forward(L, xd, ld, spec.top_k)
+    rc = lib.bitsmoe_moe_forward_noalloc(xd.data_ptr(), ld.data_ptr(), 1, spec.top_k, L.handle, y.data_ptr(),
+                                         ctypes.c_void_p(stream))
+    assert rc == 0
+    torch.cuda.synchronize()
+    assert bm.bitsmoe_noalloc_last_status(stream) == 0
+    assert _rel(y.cpu().numpy().astype(np.float64), y_ref.cpu().numpy().astype(np.float64)) <= TOL
