@@ -201,6 +201,39 @@ def oracle_tokens_per_s(spec, layer, T, budget_s=12.0, max_steps=None, seed=0):
     return toks / sum(times), steps, sum(times)
 
 
+def oracle_one_core(spec, T, budget_s=12.0):
+    """The oracle's factored forward on one host core (BLAS threads limited to 1 in a child
+    process), on a bounded sample: a layer of the workload's dims whose experts number the
+    ones a T-token step routes to (at most T * top_k), so that a step's work is the same."""
+    E = min(spec.E, T * spec.top_k)
+    code = (
+        "import sys, time, json\n"
+        f"sys.path.insert(0, {ROOT!r})\n"
+        "import synth, oracle\n"
+        f"spec = synth.scaled_spec(synth.WORKLOADS[{spec.name!r}], E={E})\n"
+        "layer = synth.make_layer(spec, seed=0)\n"
+        "n, secs = 0, 0.0\n"
+        f"while secs < {budget_s} and n < 64:\n"
+        f"    x, lg = synth.make_inputs(spec, {T}, seed=0, step=1000 + n)\n"
+        "    t0 = time.perf_counter()\n"
+        "    oracle.moe_forward_factored(layer, x, lg, spec.top_k)\n"
+        "    secs += time.perf_counter() - t0\n"
+        "    n += 1\n"
+        "print(json.dumps({'steps': n, 'secs': secs}))\n")
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    try:
+        r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, timeout=600)
+        d = json.loads(r.stdout.strip().splitlines()[-1])
+    except Exception as e:   # reported, not fatal: the GPU line stands without it
+        return {"value": None, "unit": "tokens/s", "cores": 1, "kind": "oracle", "sample": f"failed: {e}"}
+    layers = spec.layers
+    v = d["steps"] * T / d["secs"] / layers
+    return {"value": v, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+            "sample": f"{d['steps']} fp64 numpy factored forwards of {T} token(s) on a layer with the workload's "
+                      f"dims and {E} experts (BLAS threads 1, {d['secs']:.1f} s)"
+                      + (f", extrapolated to {layers} layers" if layers > 1 else "")}
+
+
 def cpu_cores():
     try:
         from threadpoolctl import threadpool_info
@@ -359,13 +392,41 @@ def run_stack(args, spec, T, torch, bm, dev, rank, world, local):
         "config": dict(config_of(spec, T, args), layers=spec.layers, l2="48 distinct layers per step (>> L2)"),
         "hbm_gbs": gbs, "hbm_frac_of_8tbs": gbs / NOMINAL_HBM_GBS, "hbm_frac_of_measured": gbs / peak,
         "bytes_per_step": step_bytes,
+        # the step is 48 block forwards back to back: its roofline is the step's, algorithmic bytes over
+        # the timed region
+        "roofline": {"bound": "hbm", "kernel": f"{spec.layers} pre-norm MoE blocks (the whole step)",
+                     "achieved": gbs, "peak": peak, "peak_source": peak_src, "unit": "GB/s", "frac": gbs / peak,
+                     "traffic": None, "bytes_per_launch": step_bytes / spec.layers,
+                     "duration_us": ms / args.steps * 1e3 / spec.layers,
+                     "duration_source": "CUDA events over the timed region / (steps x layers)",
+                     "frac_of_8tbs": gbs / NOMINAL_HBM_GBS},
         "e2e": {"value": world * ne * T / e2e_s, "unit": "tokens/s", "steps": ne,
                 "h2d_bytes_per_step": T * spec.D * 4, "d2h_bytes_per_step": T * spec.D * 4},
         "clocks": clocks,
         "gpu_launches": args.steps * spec.layers * bm.bitsmoe_block_forward_launches(layers[0], T, k),
     }
-    if rank == 0:
-        print(json.dumps(line), flush=True)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        # the oracle on one layer of the stack (RMSNorm, router, factored MoE forward), T tokens,
+        # extrapolated to the 48 layers of a step
+        import oracle
+        host = synth.make_layer(spec, seed=0, layer_index=0)
+        wr = synth.make_router_weight(spec, seed=0, layer_index=0)
+        hs = synth.make_hidden(spec, T, seed=0, step=0).astype(np.float64)
+        reps, secs = 0, 0.0
+        while secs < 12.0 and reps < 8:
+            t0 = time.perf_counter()
+            xb = synth.f32_to_bf16_bits(oracle.rms_norm(hs, eps).astype(np.float32))
+            lg = oracle.router_logits(wr, xb)
+            oracle.moe_forward_factored(host, xb, lg, k)
+            secs += time.perf_counter() - t0
+            reps += 1
+        per_layer = secs / reps
+        line["cpu_baseline"] = {"value": T / (per_layer * spec.layers), "unit": "tokens/s", "cores": cpu_cores(),
+                                "kind": "oracle",
+                                "sample": f"{reps} forwards of one stacked layer ({T} token(s), fp64 numpy, "
+                                          f"{per_layer * 1e3:.0f} ms each), extrapolated to {spec.layers} layers"}
+        line["cpu_baseline_1core"] = oracle_one_core(spec, T)
+    return line
 
 
 QUANT_METRIC = "spectral units quantised/s (per-unit Q_b into the stored format, MSE-optimal group scales)"
@@ -412,6 +473,18 @@ def run_reference_task(args, spec):
         return
     I = spec.I
     budget_s = float(os.environ.get("BITSMOE_REF_BUDGET_S", "90")) / max(1, args.steps)
+    if args.task == "importance":
+        cpu = imp_oracle_rate(spec, budget_s=min(60.0, float(os.environ.get("BITSMOE_REF_BUDGET_S", "90"))))
+        line = {
+            "impl": "reference", "metric": IMP_METRIC, "value": cpu["value"], "unit": "tokens/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1000.0 * args.calib_tokens / cpu["value"], "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": imp_config(spec, args.calib_tokens),
+            "cpu_baseline": cpu,
+            "e2e": {"value": cpu["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        }
+        print(json.dumps(line), flush=True)
+        return
     if args.task == "quantize":
         from oracle import quantizer as Q
         U = args.units or 3 * spec.E * spec.n
@@ -568,6 +641,132 @@ def run_quantize(args, spec, rank, world, local):
         print(json.dumps(line), flush=True)
 
 
+IMP_METRIC = "calibration tokens/s (importance beta of every unit of an MoE layer from calibration activations)"
+FP32_FLOPS_PER_SM_CLK = 256   # 128 fp32 lanes x 2 flops per fused multiply-add
+
+
+def imp_flops(spec, T):
+    """FLOPs of one importance step: Z = Phi^T X for gate and up, the token contraction of z^2,
+    the experts' gate/up factors on their tokens, the down factor's transposed product."""
+    D, n, E, I, k = spec.D, spec.n, spec.E, spec.I, spec.top_k
+    return 2.0 * 2 * n * D * T + 2.0 * 2 * n * T * E + 2.0 * 2 * I * n * T * k + 2.0 * n * I * T * k
+
+
+def imp_config(spec, T):
+    return {"workload": f"importance: {spec.name} layer's float factors (hidden {spec.D}, {spec.E} experts, top-"
+                        f"{spec.top_k}, intermediate {spec.I}, rank {spec.n}), {T} calibration tokens",
+            "tokens": T, "l2": f"float factors {3 * spec.E * spec.I * spec.n * 4 / 1e9:.2f} GB per step (129 MB L2)"}
+
+
+def run_importance(args, spec, rank, world, local):
+    """Importance beta of one Qwen3-shaped layer from T calibration tokens: one bitsmoe_importance
+    call per step on float factors drawn on the device (orthonormal-scale bases, j^-1/2 energies,
+    unit-norm spectral vectors), bf16 N(0, 1) activations, N(0, 1) router logits."""
+    import torch
+    import paper_2606_00079_gb300 as bm
+    dev = torch.device("cuda", local)
+    T, D, n, E, I, k = args.calib_tokens, spec.D, spec.n, spec.E, spec.I, spec.top_k
+    g = torch.Generator(device=dev)
+    g.manual_seed(4000 + rank)
+    basis = [torch.randn((D, n), generator=g, device=dev) / float(np.sqrt(D)) for _ in range(2)]
+    j = torch.arange(1, n + 1, device=dev, dtype=torch.float32)
+    alpha = [j.pow(-0.5).repeat(E, 1).contiguous() for _ in range(2)]
+    factor = []
+    for _ in range(3):
+        f = torch.randn((E, I, n), generator=g, device=dev)
+        factor.append((f / f.norm(dim=1, keepdim=True)).contiguous())
+    x = (torch.randn((T, D), generator=g, device=dev).to(torch.bfloat16)).view(torch.int16).contiguous()
+    logits = torch.randn((T, E), generator=g, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def step():
+        return bm.importance(x, logits, k, basis, alpha, factor, stream=stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(max(3, min(args.warmup, 5))):
+            step()
+    stream.synchronize()
+    clk = ClockSampler(local)
+    clk.start()
+    rank_barrier(world)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clk.mark("t0")
+    e0.record(stream)
+    with torch.cuda.stream(stream):
+        for _ in range(args.steps):
+            step()
+    e1.record(stream)
+    e1.synchronize()
+    clk.mark("t1")
+    torch.cuda.synchronize()
+    rank_barrier(world)
+    ms_own = e0.elapsed_time(e1)
+    ms = max_over_ranks(ms_own, world, dev)
+    clocks = clk.stop()
+    value = job_throughput(world, args.steps, T, ms)
+    flops = imp_flops(spec, T)
+    sec = ms_own / args.steps / 1e3
+    peaks, _ = measured_peaks()
+    sm_mhz = clocks.get("sm_mhz") or float(peaks.get("sm_max_mhz", 2070.0))
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    peak = sms * FP32_FLOPS_PER_SM_CLK * sm_mhz * 1e6 / 1e12
+    roofline = {"bound": "alu", "kernel": "bitsmoe_importance (fp32 contractions on the CUDA cores)",
+                "achieved": flops / sec / 1e12, "peak": peak, "unit": "TFLOP/s", "frac": flops / sec / 1e12 / peak,
+                "peak_source": f"{sms} SMs x 128 fp32 lanes x 2 flops x {sm_mhz:.0f} MHz (median SM clock under load)",
+                "traffic": None, "flops_per_launch": flops, "duration_us": sec * 1e6}
+    # e2e: pinned host activations and logits in, beta out, every step (the factors stay resident)
+    ne = 3
+    xh = x.cpu().pin_memory()
+    lh = logits.cpu().pin_memory()
+    bh = torch.empty((3, E, n), dtype=torch.float32).pin_memory()
+    t0 = time.perf_counter()
+    for _ in range(ne):
+        with torch.cuda.stream(stream):
+            x.copy_(xh, non_blocking=True)
+            logits.copy_(lh, non_blocking=True)
+            bh.copy_(step(), non_blocking=True)
+        stream.synchronize()
+    e2e_s = time.perf_counter() - t0
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = imp_oracle_rate(spec, budget_s=12.0)
+    if rank == 0:
+        line = {
+            "metric": IMP_METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": imp_config(spec, T),
+            "roofline": roofline, "cpu_baseline": cpu,
+            "e2e": {"value": world * ne * T / e2e_s, "unit": "tokens/s", "steps": ne,
+                    "h2d_bytes_per_step": T * D * 2 + T * E * 4, "d2h_bytes_per_step": 3 * E * n * 4},
+            "clocks": clocks, "gpu_launches": args.steps * 7,
+        }
+        print(json.dumps(line), flush=True)
+
+
+def imp_oracle_rate(spec, budget_s=12.0):
+    """The calibration oracle (fp64 numpy) on the host cores, on a bounded sample: a layer with
+    the workload's D, n and I and top_k + 1 experts, 32 tokens per call (calibration tokens/s)."""
+    from oracle import calibration as Co
+    rng = np.random.default_rng(5)
+    E = spec.top_k + 1
+    D, n, I, T = spec.D, spec.n, spec.I, 32
+    Phi = [np.linalg.qr(rng.standard_normal((D, n)))[0] for _ in range(3)]
+    al = [np.tile(np.arange(1, n + 1) ** -0.5, (E, 1)) for _ in range(3)]
+    P = [[rng.standard_normal((I, n)) / np.sqrt(I) for _ in range(E)] for _ in range(3)]
+    x = synth.f32_to_bf16_bits(rng.standard_normal((T, D)).astype(np.float32))
+    lg = rng.standard_normal((T, E)).astype(np.float32)
+    n_done, secs = 0, 0.0
+    while secs < budget_s and n_done < 64 * T:
+        t0 = time.perf_counter()
+        Co.factor_importance(Phi, al, P, x, lg, spec.top_k)
+        secs += time.perf_counter() - t0
+        n_done += T
+    return {"value": n_done / secs * (E / spec.E), "unit": "tokens/s", "cores": cpu_cores(), "kind": "oracle",
+            "sample": f"{n_done} tokens through factor_importance on a layer with {E} experts of the workload's dims "
+                      f"({secs:.1f} s), scaled to {spec.E} experts by the per-expert work"}
+
+
 ALLOC_METRIC = "spectral units allocated/s (per-projection bit allocation: costs, Lagrangian cut, greedy fill)"
 KAPPA_TABLE = (0.14949200, 0.04067890, 0.01184786)   # kappa_2, kappa_3, kappa_4 (Table kappa_values)
 
@@ -702,62 +901,9 @@ def run_allocate(args, spec, rank, world, local):
         print(json.dumps(line), flush=True)
 
 
-def main():
-    ap = argparse.ArgumentParser()
-    ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=None,
-                    help="default 20000 (one layer), 400 (layer stack), 20 (--task quantize)")
-    ap.add_argument("--warmup", type=int, default=200)
-    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="qw3")
-    ap.add_argument("--tokens", type=int, default=None)
-    ap.add_argument("--copies", type=int, default=8)
-    ap.add_argument("--inputs", type=int, default=64)
-    ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--graph", type=int, default=256, help="forwards per captured CUDA graph")
-    ap.add_argument("--task", default="forward", choices=["forward", "quantize", "allocate"],
-                    help="forward: the MoE-layer forward (default); quantize: the per-unit quantiser; "
-                         "allocate: the per-projection bit allocation")
-    ap.add_argument("--grid", type=int, default=256, help="scale candidates of the quantiser (--task quantize)")
-    ap.add_argument("--units", type=int, default=None,
-                    help="units per quantiser step (default the whole layer, 3 E n) or per allocated "
-                         "projection (default E n)")
-    args = ap.parse_args()
-    spec = synth.WORKLOADS[args.workload]
-    T = args.tokens or spec.tokens[0]
-    if args.steps is None:
-        args.steps = 20 if args.task != "forward" else (20000 if spec.layers == 1 else 400)
-    if args.impl == "reference":
-        if args.task == "forward":
-            run_reference(args, spec, T)
-        else:
-            run_reference_task(args, spec)
-        return
-
-    import torch
-    import paper_2606_00079_gb300 as bm
-    from paper_2606_00079_gb300 import build as bmbuild
-    bmbuild.build()
-    rank, world, local = dist_env()
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-
-    if args.task != "forward":
-        (run_quantize if args.task == "quantize" else run_allocate)(args, spec, rank, world, local)
-        if world > 1:
-            torch.distributed.barrier()
-            torch.distributed.destroy_process_group()
-        return
-    if spec.layers > 1:
-        run_stack(args, spec, T, torch, bm, dev, rank, world, local)
-        if world > 1:
-            torch.distributed.barrier()
-            torch.distributed.destroy_process_group()
-        return
-
+def run_layer(args, spec, T, torch, bm, dev, rank, world, local):
+    """One MoE layer: K forwards of T tokens from CUDA graphs over rotating packed copies; returns
+    rank 0's JSON line (None on the other ranks)."""
     # ---- workload: one generated layer, packed once, uploaded as rotating copies
     layer = synth.make_layer(spec, seed=0)
     blob = bm.bitsmoe_pack_to_host(layer)
@@ -850,7 +996,7 @@ def main():
         # one fused kernel does the whole step: its average duration is at most the timed region per
         # step (which also holds the gap between launches), so this is a lower bound
         achieved = (total_bytes / args.steps) / (ms / args.steps / 1e3) / 1e9
-        traffic = measured_traffic("ncu_full_k_fused_qw3_T1.txt", ("fused.cu", "device.cuh", "format.h"))
+        traffic = measured_traffic("ncu_full_k_fused_qw3_T1.txt", ("fused.cu", "fused_common.cuh", "device.cuh", "format.h"))
         roofline = {"bound": "hbm", "kernel": "k_fused (whole single-token forward)", "achieved": achieved,
                     "peak": peak, "peak_source": peak_src, "unit": "GB/s", "frac": achieved / peak,
                     "traffic": traffic,
@@ -902,12 +1048,14 @@ def main():
            "h2d_bytes_per_step": T * spec.D * 2 + T * spec.E * 4, "d2h_bytes_per_step": T * spec.D * 4}
 
     # ---- CPU baseline (rank 0, N = 1 only)
-    cpu = None
+    cpu = cpu1 = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         v, steps, secs = oracle_tokens_per_s(spec, layer, T, budget_s=12.0)
         cpu = {"value": v, "unit": "tokens/s", "cores": cpu_cores(), "kind": "oracle",
                "sample": f"{steps} decode steps of {T} token(s), fp64 numpy factored forward ({secs:.1f} s)"}
+        cpu1 = oracle_one_core(spec, T)
 
+    line = None
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
@@ -917,10 +1065,103 @@ def main():
             "data": "synthetic", "config": config_of(spec, T, args),
             "hbm_gbs": fwd_gbs, "hbm_frac_of_8tbs": fwd_gbs / NOMINAL_HBM_GBS, "hbm_frac_of_measured": fwd_gbs / peak,
             "bytes_per_step": total_bytes / args.steps,
-            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks,
+            "roofline": roofline, "cpu_baseline": cpu, "cpu_baseline_1core": cpu1, "e2e": e2e, "clocks": clocks,
             "gpu_launches": args.steps * launches,
         }
-        print(json.dumps(line), flush=True)
+    return line
+
+
+ALL_CONFIGS = [("qw3", 1), ("qw3_skew", 1), ("qw3_skew", 8), ("qw3_skew", 32), ("qw3_skew", 128),
+               ("mixtral", 1), ("mixtral", 16), ("qw3_stack", 1), ("qw3_stack", 32)]
+
+
+def run_all(args, torch, bm, dev, rank, world, local):
+    """Every workload configuration in turn, one JSON line each; the step count adapts so that
+    each timed region is a fraction of a second to a few seconds."""
+    import copy
+    import gc
+    for wl, T in ALL_CONFIGS:
+        spec = synth.WORKLOADS[wl]
+        a = copy.copy(args)
+        a.workload, a.tokens = wl, T
+        if spec.layers > 1:
+            a.steps = args.steps or (200 if T == 1 else 20)
+            line = run_stack(a, spec, T, torch, bm, dev, rank, world, local)
+        else:
+            a.steps = args.steps or (4000 if T <= 4 else 1000 if T <= 32 else 400)
+            line = run_layer(a, spec, T, torch, bm, dev, rank, world, local)
+        if rank == 0:
+            print(json.dumps(line), flush=True)
+        gc.collect()
+        torch.cuda.empty_cache()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=None,
+                    help="default 20000 (one layer), 400 (layer stack), 20 (--task quantize)")
+    ap.add_argument("--warmup", type=int, default=200)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="qw3")
+    ap.add_argument("--tokens", type=int, default=None)
+    ap.add_argument("--copies", type=int, default=8)
+    ap.add_argument("--inputs", type=int, default=64)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--graph", type=int, default=256, help="forwards per captured CUDA graph")
+    ap.add_argument("--task", default="forward", choices=["forward", "quantize", "allocate", "importance"],
+                    help="forward: the MoE-layer forward (default); quantize: the per-unit quantiser; "
+                         "allocate: the per-projection bit allocation; importance: the importance beta of "
+                         "every unit from calibration tokens")
+    ap.add_argument("--calib-tokens", type=int, default=4096,
+                    help="calibration tokens per step of --task importance")
+    ap.add_argument("--grid", type=int, default=256, help="scale candidates of the quantiser (--task quantize)")
+    ap.add_argument("--all", action="store_true",
+                    help="one JSON line per workload configuration and token count (the single layers at "
+                         "T = 1; qw3_skew at 1, 8, 32, 128; mixtral at 1, 16; the 48-layer stack at 1, 32)")
+    ap.add_argument("--units", type=int, default=None,
+                    help="units per quantiser step (default the whole layer, 3 E n) or per allocated "
+                         "projection (default E n)")
+    args = ap.parse_args()
+    spec = synth.WORKLOADS[args.workload]
+    T = args.tokens or spec.tokens[0]
+    if args.steps is None and not args.all:
+        args.steps = 20 if args.task != "forward" else (20000 if spec.layers == 1 else 400)
+    if args.impl == "reference":
+        if args.task == "forward":
+            run_reference(args, spec, T)
+        else:
+            run_reference_task(args, spec)
+        return
+
+    import torch
+    import paper_2606_00079_gb300 as bm
+    from paper_2606_00079_gb300 import build as bmbuild
+    bmbuild.build()
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    if args.task != "forward":
+        {"quantize": run_quantize, "allocate": run_allocate,
+         "importance": run_importance}[args.task](args, spec, rank, world, local)
+        if world > 1:
+            torch.distributed.barrier()
+            torch.distributed.destroy_process_group()
+        return
+    if args.all:
+        run_all(args, torch, bm, dev, rank, world, local)
+    elif spec.layers > 1:
+        line = run_stack(args, spec, T, torch, bm, dev, rank, world, local)
+        if rank == 0:
+            print(json.dumps(line), flush=True)
+    else:
+        line = run_layer(args, spec, T, torch, bm, dev, rank, world, local)
+        if rank == 0:
+            print(json.dumps(line), flush=True)
     if world > 1:
         torch.distributed.barrier()
         torch.distributed.destroy_process_group()

@@ -386,6 +386,48 @@ int bitsmoe_profile_allocate_bits(const float* p, const float* alpha, const floa
                                   int d, const float* kappa, int64_t budget, uint8_t* bits, void* ws,
                                   size_t ws_bytes, void* stream, float phase_ms[3]);
 
+/* Importance beta of every spectral unit from calibration tokens, on the GPU:
+ * the allocation's input (bitsmoe_allocate_bits' beta), computed on the float
+ * factors of the shared-basis decomposition before anything is quantised.
+ * BitsMoE weighs each unit's quantisation loss by the activation metric of its
+ * expert, H_e = X Diag(g_e) X^T over the calibration activations X with the
+ * tokens' routing affinities g_e (appendix Eq. app_affinity_gram):
+ *   beta[h][e][k] = phi_{h,k}^T H_e phi_{h,k}
+ *                 = sum_t g_{t,e} (phi_{h,k}^T x_t)^2                 h = gate, up
+ *   beta[2][e][k] = p_{dn,e,k}^T H'_e p_{dn,e,k}
+ *                 = sum_t g_{t,e} (p_{dn,e,k}^T h_{t,e})^2             down
+ * with h_{t,e} = SiLU(P_g,e diag(alpha_g,e) Phi_g^T x_t) * (P_u,e diag(alpha_u,e)
+ * Phi_u^T x_t) the expert's SwiGLU output (appendix Eqs. app_beta_def,
+ * app_down_beta_approx, app_unified_beta_def).  A token's affinity to expert e
+ * is its gate weight (softmax over its top_k logits, ties to the lower index)
+ * when e is selected and 0 otherwise.
+ *   x        device, T x D bf16 calibration activations (row-major)
+ *   logits   device, T x E fp32 router logits of those tokens
+ *   basis    host array of 2 device pointers: Phi_gate, Phi_up, each D x n fp32
+ *            (row d, column k = phi_k)
+ *   alpha    host array of 2 device pointers: alpha_gate, alpha_up, E x n fp32
+ *   factor   host array of 3 device pointers: P_gate, P_up, P_down, each
+ *            E x I x n fp32 (expert e's I x n factor, column k = p_{e,k})
+ *   beta     device, 3 x E x n fp32 (written)
+ *   ws       device workspace of >= bitsmoe_importance_workspace_bytes(T, E,
+ *            I, n, top_k) bytes, 256-byte aligned, caller-owned
+ * fp32 arithmetic throughout (the contractions on the CUDA cores).  T == 0
+ * writes beta = 0.  Host-side checks only (INVALID_ARG, SHAPE,
+ * WORKSPACE_TOO_SMALL); asynchronous on `stream`, never allocates. */
+size_t bitsmoe_importance_workspace_bytes(int64_t T, int E, int I, int n, int top_k);
+int bitsmoe_importance(const void* x, const float* logits, int64_t T, int D, int E, int I, int n, int top_k,
+                       const float* const basis[2], const float* const alpha[2], const float* const factor[3],
+                       float* beta, void* ws, size_t ws_bytes, void* stream);
+
+/* Where bitsmoe_moe_block_forward(T, top_k) leaves the block's normalised
+ * activations x (T x D bf16) and router logits (T x E fp32) in its workspace:
+ * byte offsets from the workspace start, valid after the call completes (the
+ * fused single-token kernel, which normalises and routes inside, writes them
+ * there too).  For inspection and tests; no counterpart in the paper.
+ * Errors: INVALID_ARG. */
+int bitsmoe_block_norm_outputs(const bitsmoe_layer* layer, int T, int top_k, size_t* x_offset,
+                               size_t* logits_offset);
+
 /* Synchronise `stream`, then read and clear the device status word kept in
  * `ws`: BITSMOE_OK, or the first device-side error recorded by the last
  * forward that used this workspace (each forward resets it when it starts). */

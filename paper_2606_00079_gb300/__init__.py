@@ -72,6 +72,10 @@ SIGNATURES = {
     "bitsmoe_profile_allocate_bits": (_I, [_P, _P, _P, ctypes.c_float, ctypes.c_int64, _I,
                                            ctypes.POINTER(ctypes.c_float), ctypes.c_int64, _P, _P, _SZ, _P,
                                            ctypes.POINTER(ctypes.c_float)]),
+    "bitsmoe_importance_workspace_bytes": (_SZ, [ctypes.c_int64, _I, _I, _I, _I]),
+    "bitsmoe_importance": (_I, [_P, _P, ctypes.c_int64, _I, _I, _I, _I, _I, ctypes.POINTER(_P), ctypes.POINTER(_P),
+                                ctypes.POINTER(_P), _P, _P, _SZ, _P]),
+    "bitsmoe_block_norm_outputs": (_I, [_P, _I, _I, ctypes.POINTER(_SZ), ctypes.POINTER(_SZ)]),
     "bitsmoe_last_device_status": (_I, [_P, _P]),
     "bitsmoe_free": (None, [_P]),
     "bitsmoe_strerror": (ctypes.c_char_p, [_I]),
@@ -361,6 +365,14 @@ def bitsmoe_last_device_status(ws_ptr: int, stream: int = 0) -> int:
     return int(_lib().bitsmoe_last_device_status(ws_ptr, stream))
 
 
+def bitsmoe_block_norm_outputs(layer: Layer, T: int, top_k: int):
+    """Byte offsets of a block forward's normalised x and router logits in its workspace."""
+    xo, lo = _SZ(0), _SZ(0)
+    _check(_lib().bitsmoe_block_norm_outputs(layer.handle, T, top_k, ctypes.byref(xo), ctypes.byref(lo)),
+           "bitsmoe_block_norm_outputs")
+    return int(xo.value), int(lo.value)
+
+
 def bitsmoe_noalloc_last_status(stream: int = 0) -> int:
     """Device status of the no-allocation scratch on the current device (read and cleared)."""
     return int(_lib().bitsmoe_noalloc_last_status(stream))
@@ -433,6 +445,30 @@ def allocate_bits(p, alpha, beta, gamma: float, kappa, budget: int, stream=None)
                           bits.data_ptr(), (ws.data_ptr() + 255) // 256 * 256, nb, st.cuda_stream)
     ws.record_stream(st)   # the workspace is freed here but used by the kernels still queued on st
     return bits
+
+
+def importance(x, logits, top_k: int, basis, alpha, factor, stream=None):
+    """Importance beta (torch fp32, 3 x E x n) of every unit from calibration tokens: x (torch
+    int16 bf16 bit patterns, T x D), logits (fp32, T x E), basis = (Phi_gate, Phi_up) fp32 D x n,
+    alpha = (alpha_gate, alpha_up) fp32 E x n, factor = (P_gate, P_up, P_down) fp32 E x I x n,
+    all on the device."""
+    import torch
+    T, D = int(x.shape[0]), int(x.shape[1])
+    E = int(logits.shape[1])
+    _, I, n = (int(v) for v in factor[0].shape)
+    dev = x.device
+    beta = torch.empty((3, E, n), dtype=torch.float32, device=dev)
+    nb = int(_lib().bitsmoe_importance_workspace_bytes(T, E, I, n, top_k))
+    ws = torch.empty(nb + 256, dtype=torch.uint8, device=dev)
+    st = stream if stream is not None else torch.cuda.current_stream(dev)
+    bp = (_P * 2)(*[b.data_ptr() for b in basis])
+    ap = (_P * 2)(*[a.data_ptr() for a in alpha])
+    fp = (_P * 3)(*[f.data_ptr() for f in factor])
+    _check(_lib().bitsmoe_importance(x.data_ptr(), logits.data_ptr(), T, D, E, I, n, top_k, bp, ap, fp,
+                                     beta.data_ptr(), (ws.data_ptr() + 255) // 256 * 256, nb, st.cuda_stream),
+           "bitsmoe_importance")
+    ws.record_stream(st)
+    return beta
 
 
 def bitsmoe_debug_single_token_kernel(which: int) -> None:

@@ -239,61 +239,107 @@ __device__ __forceinline__ int step_bits(const uint8_t* r, int s) {
 }
 
 // Radix pass: bits of the increments in the current bucket, by the digit at `shift`.
+// Many increments share a digit (the leading digits hold the efficiency's exponent), so
+// the lanes of a warp that hit the same digit add their bits first and one of them
+// updates the histogram.
 __global__ void k_alloc_hist(AllocWs w, int64_t U, int shift) {
   const AllocState& st = *w.st;
   if (st.all_fit) return;
   const int hs = shift + 16;
   const unsigned long long pre = st.prefix;
-  for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < U; u += (int64_t)gridDim.x * blockDim.x) {
-    const unsigned long long* k = w.keys + (size_t)u * kNS;
-    const uint8_t* r = w.reach + (size_t)u * kNS;
+  const int lane = threadIdx.x & 31;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  // whole warps walk the units together, so that every lane reaches the shuffles
+  for (int64_t u0 = (int64_t)blockIdx.x * blockDim.x + (threadIdx.x & ~31); u0 < U; u0 += stride) {
+    const int64_t u = u0 + lane;
+    const bool live = u < U;
+    const unsigned long long* k = w.keys + (size_t)(live ? u : 0) * kNS;
+    const uint8_t* r = w.reach + (size_t)(live ? u : 0) * kNS;
+    bool more = live;
 #pragma unroll 1
     for (int s = 0; s < kNS; ++s) {
-      const unsigned long long key = k[s];
-      if (!key) break;
-      if (hs < 64 && (key >> hs) != (pre >> hs)) continue;
-      atomicAdd(w.hist + ((key >> shift) & 0xFFFFull), (unsigned long long)step_bits(r, s));
+      const unsigned long long key = more ? k[s] : 0ull;
+      more = more && key != 0ull;
+      const bool take = more && (hs >= 64 || (key >> hs) == (pre >> hs));
+      const unsigned act = __ballot_sync(0xFFFFFFFFu, take);
+      if (!__any_sync(0xFFFFFFFFu, more)) break;
+      if (take) {
+        const unsigned dgt = (unsigned)((key >> shift) & 0xFFFFull);
+        const unsigned grp = __match_any_sync(act, dgt);
+        const unsigned tot = __reduce_add_sync(grp, (unsigned)step_bits(r, s));
+        if (lane == __ffs(grp) - 1) atomicAdd(w.hist + dgt, (unsigned long long)tot);
+      }
     }
   }
 }
 
-// One block: find the largest digit d with above + sum_{d' >= d} hist[d'] > budget.
+// One block: find the largest digit d with above + sum_{d' >= d} hist[d'] > budget.  Two
+// levels, every load coalesced: warp w sums its 2048 digits (lane-strided), warp 0 finds
+// the warp whose range holds the cut from the suffix sums of the 32 warp totals, then the
+// block scans that range's digits in pairs.
 __global__ void __launch_bounds__(1024) k_alloc_scan(AllocWs w, long long budget, int shift, int last) {
+  constexpr int kPerW = kDigits / 32;
+  __shared__ unsigned long long wtot[32];
   __shared__ unsigned long long part[1024];
-  __shared__ int found;
+  __shared__ unsigned long long wabove;
+  __shared__ int cutw, found;
   AllocState& st = *w.st;
-  const int t = threadIdx.x;
-  constexpr int per = kDigits / 1024;
+  const int t = threadIdx.x, lane = t & 31, wid = t >> 5;
   const bool skip = st.all_fit != 0;
-  // thread t owns digits [t * per, t * per + per); suffix sums run from the top digit down
-  unsigned long long mine = 0;
-  for (int i = 0; i < per; ++i) mine += w.hist[t * per + i];
-  part[t] = mine;
-  if (t == 0) found = 0;
-  __syncthreads();
-  // inclusive suffix scan over threads (Hillis-Steele, from high t to low t)
-  for (int o = 1; o < 1024; o <<= 1) {
-    const unsigned long long v = t + o < 1024 ? part[t + o] : 0ull;
-    __syncthreads();
-    part[t] += v;
-    __syncthreads();
-  }
   const unsigned long long above = st.above;
   const unsigned long long bud = (unsigned long long)budget;
-  if (!skip) {
-    unsigned long long run = (t + 1 < 1024 ? part[t + 1] : 0ull);   // digits above this thread's range
-    if (above + run + mine > bud && above + run <= bud) {
-      for (int i = per - 1; i >= 0; --i) {
-        const unsigned long long h = w.hist[t * per + i];
-        if (above + run + h > bud) {
-          const int dgt = t * per + i;
-          st.prefix |= (unsigned long long)dgt << shift;
-          st.above = above + run;
-          found = 1;
-          break;
-        }
-        run += h;
+  {
+    const unsigned long long* hw = w.hist + (size_t)wid * kPerW;
+    unsigned long long sum = 0;
+#pragma unroll 8
+    for (int i = 0; i < kPerW / 32; ++i) sum += hw[i * 32 + lane];
+#pragma unroll
+    for (int o = 16; o; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
+    if (lane == 0) wtot[wid] = sum;
+  }
+  if (t == 0) {
+    cutw = -1;
+    found = 0;
+  }
+  __syncthreads();
+  if (wid == 0 && !skip) {
+    const unsigned long long mine = wtot[lane];
+    unsigned long long sfx = mine;   // sum of the warps at or above this one
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const unsigned long long v = __shfl_down_sync(0xFFFFFFFFu, sfx, o);
+      if (lane + o < 32) sfx += v;
+    }
+    if (above + sfx > bud && above + sfx - mine <= bud) {
+      cutw = lane;
+      wabove = sfx - mine;
+    }
+  }
+  __syncthreads();
+  const int cw = cutw;
+  if (cw >= 0) {
+    // the cut warp's digits, two per thread (d0 = 2t, d1 = 2t + 1 of its range)
+    const unsigned long long* hc = w.hist + (size_t)cw * kPerW;
+    const unsigned long long h0 = hc[2 * t], h1 = hc[2 * t + 1];
+    part[t] = h0 + h1;
+    __syncthreads();
+    for (int o = 1; o < 1024; o <<= 1) {   // inclusive suffix scan over the pairs
+      const unsigned long long v = t + o < 1024 ? part[t + o] : 0ull;
+      __syncthreads();
+      part[t] += v;
+      __syncthreads();
+    }
+    const unsigned long long run = above + wabove + (t + 1 < 1024 ? part[t + 1] : 0ull);
+    if (run + h0 + h1 > bud && run <= bud) {
+      const int d1 = cw * kPerW + 2 * t + 1;
+      if (run + h1 > bud) {
+        st.prefix |= (unsigned long long)d1 << shift;
+        st.above = run;
+      } else {
+        st.prefix |= (unsigned long long)(d1 - 1) << shift;
+        st.above = run + h1;
       }
+      found = 1;
     }
   }
   __syncthreads();
@@ -305,7 +351,7 @@ __global__ void __launch_bounds__(1024) k_alloc_scan(AllocWs w, long long budget
       st.kstar = st.prefix;
     }
   }
-  for (int i = 0; i < per; ++i) w.hist[t * per + i] = 0ull;   // ready for the next pass
+  for (int i = t; i < kDigits; i += 1024) w.hist[i] = 0ull;   // ready for the next pass
 }
 
 // Step 3 for every unit, and its next increment for the fill.

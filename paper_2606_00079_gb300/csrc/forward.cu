@@ -2088,6 +2088,15 @@ int bitsmoe_moe_block_forward(float* h, const void* w_router, float eps, int T, 
                       ws_bytes, st, nullptr, true, &a);
 }
 
+int bitsmoe_block_norm_outputs(const bitsmoe_layer* L, int T, int top_k, size_t* x_offset, size_t* logits_offset) {
+  if (!L || T < 1 || top_k < 1 || top_k > std::min(L->hd().E, 32) || !x_offset || !logits_offset)
+    return BITSMOE_ERR_INVALID_ARG;
+  const WsLayout w = ws_layout(L->hd(), T, top_k);
+  *x_offset = w.x_stage;
+  *logits_offset = w.logits_stage;
+  return BITSMOE_OK;
+}
+
 int bitsmoe_last_device_status(void* ws, void* stream) {
   if (!ws) return BITSMOE_ERR_INVALID_ARG;
   cudaStream_t st = static_cast<cudaStream_t>(stream);

@@ -421,6 +421,8 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
         u32 = (u32 + 0x7FFFu + ((u32 >> 16) & 1u)) & 0xFFFF0000u;
       }
       xs[d] = (uint16_t)(u32 >> 16);
+      // block 0 leaves x in the workspace, where the separate norm/router step would put it
+      if (blk == 0 && d < p.D) const_cast<uint16_t*>(p.x)[d] = (uint16_t)(u32 >> 16);
     }
     __syncthreads();
   }

@@ -72,6 +72,15 @@ def test_stack_layer_local_parity(stack, T):
                                      ws.nbytes, st)
         if l in SAMPLED:
             torch.cuda.synchronize()
+            # the x and logits the block itself used (computed inside the fused kernel at one
+            # token) are the same bits as the separate norm/router step's
+            xo, lo = bm.bitsmoe_block_norm_outputs(layers[l], T, k)
+            wsb = ws.buf.view(torch.uint8)
+            d0 = ws.ptr - ws.buf.data_ptr()   # the workspace starts at the buffer's 256-byte boundary
+            xb = wsb[d0 + xo:d0 + xo + T * spec.D * 2].view(torch.int16).view(T, spec.D)
+            lb = wsb[d0 + lo:d0 + lo + T * spec.E * 4].view(torch.float32).view(T, spec.E)
+            assert torch.equal(xb, x), l
+            assert torch.equal(lb.view(torch.int32), lg.view(torch.int32)), l
             saved[l] = (h_in.cpu().numpy().astype(np.float64), x.cpu().numpy().view(np.uint16).copy(),
                         lg.cpu().numpy().copy(), h.cpu().numpy().astype(np.float64))
     torch.cuda.synchronize()
