@@ -35,6 +35,22 @@
 #include "fused_common.cuh"
 
 namespace {
+
+// Phase timestamps of each block (%globaltimer), compiled in only with -DBITSMOE_F2_TRACE
+// for timing studies; without it F1_MARK is empty.
+#ifdef BITSMOE_F2_TRACE
+__device__ unsigned long long g_f1_trace[1024][16];
+#define F1_MARK(i)                                                                    \
+  do {                                                                                \
+    unsigned long long t_;                                                            \
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t_));                            \
+    g_f1_trace[blockIdx.x & 1023][(i)] = t_;                                          \
+  } while (0)
+#else
+#define F1_MARK(i) \
+  do {             \
+  } while (0)
+#endif
 // Copy of a gate/up staging record into shared memory (its per-bucket arrays
 // are read with runtime indices, so it is used from there).
 __device__ __forceinline__ void copy_crec(CStage* dst, const CStage* src) {
@@ -360,6 +376,7 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
     }
   };
   if (tid == 0) {
+    F1_MARK(0);
     for (int i = 0; i < kMaxBStages + 1 + 2 * kFWarps; ++i) mbar_init(bar_b + i);
     seen[0] = seen[1] = seen[2] = seen[3] = 0;
     issue_b(0, nst_pre);
@@ -375,6 +392,7 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
   if (wid >= kBW) route_token(nullptr, p.E, p.k, keys, sel_e, sel_w, tid - kBW * 32);   // code warm-up
   __syncthreads();
   pdl_wait();   // x, logits, y and the workspace belong to earlier kernels until here
+  if (threadIdx.x == 0) F1_MARK(1);
 
   // the workspace's barrier counters must be zero (only counter 0 can move before
   // every block has passed this check)
@@ -489,6 +507,7 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
     }
     // the block's z rows are written: arrive at barrier 1 without waiting for the control warps
     asm volatile("bar.sync 3, %0;" ::"r"(kBW * 32) : "memory");
+    if (tid == 0) F1_MARK(5);
     if (tid == 0 && !((f.dbg & 1) && blk == 0)) grid_arrive(f.cnt + 0);
   } else {
     const int ct = tid - kBW * 32;
@@ -528,6 +547,7 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
     }
     // ---- routing of the token
     route_token(p.logits, p.E, p.k, keys, sel_e, sel_w, ct);
+    if (ct == 0) F1_MARK(3);
     // ---- staging: control thread s < nslot_c stages gate/up slot s; 32 + s < 32 + nslot_d prefetches down slot s
     const int A = p.k;
     const int nci = A * 2 * p.NRB * p.nseg;
@@ -554,7 +574,9 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
       }
     }
   }
+  if (tid == 0) F1_MARK(4);
   grid_wait(f.cnt + 0, nb, p.status, seen + 0, f.spin);
+  if (tid == 0) F1_MARK(6);
   // The projection rows are consumed; their buffer receives the first down tiles
   // (each staged by its slot's warp once that warp's gate/up items are done, so
   // that the copies do not delay the latency-bound z gathers) and, once the
@@ -595,7 +617,9 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
     fence_proxy_async();   // generic reads of the projection rows (before barrier 1), then async writes
     d_stage(p, f, drec[wid], dslots + (size_t)wid * f.slot_d, bar_d + wid);
   }
+  if (tid == 0) F1_MARK(7);
   grid_barrier(f.cnt + 1, nb, p.status, seen + 1, f.spin);
+  if (tid == 0) F1_MARK(8);
 
   // ---- D: down tiles, s += w * alpha * P_dn^T h.  Warp w works on slot w % nslot_d
   // over row blocks w / nslot_d, + nsub, ...; the slot's partial sums meet in shared memory.
@@ -660,7 +684,9 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
       __syncthreads();
     }
   }
+  if (tid == 0) F1_MARK(9);
   grid_barrier(f.cnt + 2, nb, p.status, seen + 2, f.spin);
+  if (tid == 0) F1_MARK(10);
   pdl_trigger();   // every block is past its last wait on other blocks
 
   // ---- E: y = Phi_dn s for rows [e0, e1)
@@ -694,6 +720,7 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
       }
     }
   }
+  if (tid == 0) F1_MARK(11);
   // the last block to finish resets the barrier counters for the next call
   if (tid == 0) {
     const uint32_t old = atomicAdd(f.cnt + 3, 1u);
@@ -856,3 +883,9 @@ cudaError_t launch_fused(const Fwd& p, const FusedArgs& f, int sms, cudaStream_t
 }
 
 }  // namespace bmoe
+
+#ifdef BITSMOE_F2_TRACE
+extern "C" int bitsmoe_f1_trace_read(void* dst) {
+  return (int)cudaMemcpyFromSymbol(dst, g_f1_trace, sizeof(g_f1_trace));
+}
+#endif
