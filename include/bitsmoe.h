@@ -419,6 +419,58 @@ int bitsmoe_importance(const void* x, const float* logits, int64_t T, int D, int
                        const float* const basis[2], const float* const alpha[2], const float* const factor[3],
                        float* beta, void* ws, size_t ws_bytes, void* stream);
 
+/* Shared-basis spectral decomposition of one projection type over its E experts
+ * (Sec. "Shared-basis Spectral Decomposition": Eq. shared_basis_input_proj and
+ * Eq. app_cat_svd_absorbed for gate/up, the concatenation along input channels
+ * of Eq. app_down_cat_svd_absorbed for down; alpha and P by Definitions
+ * spectral_energy_matrix / spectral_matrix):
+ *   side 0 ("in", gate/up): W is E x d x D (W_e = d x D), W_cat = [W_1; ...; W_E]
+ *                           = U S Phi^T, P~_cat = U S split into E row blocks
+ *   side 1 ("out", down):   W is E x D x d (W_e = D x d), W_cat = [W_1 ... W_E]
+ *                           = Phi S V^T, P~_cat = V S split by input channels
+ *   alpha[e][k] = ||P~_e[:, k]||_2, P_e = P~_e / alpha_e (P~_e where alpha = 0).
+ * Computed as the eigendecomposition of G = W_cat^T W_cat (side 0) or W_cat W_cat^T
+ * (side 1), D x D, in fp32 (cyclic two-sided Jacobi), then P~ = W_cat Phi (side 0)
+ * or W_cat^T Phi (side 1).  n = min(D, E d) columns, by descending singular
+ * value (ties: the lower eigenvector index); each basis column's largest
+ * |component| is positive (the first one on ties).  Singular values and
+ * vectors are those of W_cat up to fp32 rounding; a vector whose singular value
+ * is repeated is any orthonormal basis of its space.
+ *   W       device, fp32, 16-byte aligned, finite
+ *   E, d, D experts, their intermediate size, the feature dimension
+ *           (2 <= D <= BITSMOE_DECOMPOSE_MAX_D)
+ *   phi     device, D x n fp32 (column k = phi_k) (written)
+ *   sigma   device, n fp32 singular values, descending (written)
+ *   alpha   device, E x n fp32 (written)
+ *   P       device, E x n x d fp32, unit-major: P[e][k][:] = p_{e,k}, the row
+ *           layout bitsmoe_quantize_units takes (written)
+ *   ws      device workspace of >= bitsmoe_decompose_workspace_bytes(side, E, d, D)
+ *           bytes, 256-byte aligned
+ *   max_sweeps  Jacobi sweeps at most (>= 1; the solver stops earlier after a
+ *           sweep in which no rotation was needed: every |g_pq| <= 1e-7
+ *           sqrt(|g_pp g_qq|) or <= 4e-7 max_j |g_jj|)
+ *   sweeps  device int or NULL: the sweeps run (written)
+ *   status  device int: BITSMOE_ERR_TIMEOUT is written there if a bounded
+ *           grid-barrier wait of the solver ran out (the call then leaves its
+ *           outputs undefined); it is not cleared by the call
+ * Host-side checks (INVALID_ARG, WORKSPACE_TOO_SMALL, ALIGNMENT, SHAPE when the
+ * solver's block cannot be resident); never allocates, never synchronises.  Six
+ * kernel launches (one cooperative). */
+#define BITSMOE_DECOMPOSE_MAX_D 8192
+size_t bitsmoe_decompose_workspace_bytes(int side, int E, int d, int D);
+int bitsmoe_shared_basis(int side, const float* W, int E, int d, int D, float* phi, float* sigma, float* alpha,
+                         float* P, void* ws, size_t ws_bytes, int max_sweeps, int* sweeps, int* status,
+                         void* stream);
+
+/* Calibration Gram H = X^T Diag(g) X = sum_t g_t x_t x_t^T (appendix,
+ * Eq. app_affinity_gram: the activation metric of one expert with the routing
+ * affinities g of its tokens), fp32.
+ *   x   device, T x D bf16 (row t = x_t)
+ *   g   device, T fp32 weights, or NULL (all 1)
+ *   H   device, D x D fp32 (written; symmetric)
+ * T == 0 writes zeros.  Never allocates, never synchronises; one launch. */
+int bitsmoe_calibration_gram(const void* x, const float* g, int64_t T, int D, float* H, void* stream);
+
 /* Where bitsmoe_moe_block_forward(T, top_k) leaves the block's normalised
  * activations x (T x D bf16) and router logits (T x E fp32) in its workspace:
  * byte offsets from the workspace start, valid after the call completes (the

@@ -75,6 +75,9 @@ SIGNATURES = {
     "bitsmoe_importance_workspace_bytes": (_SZ, [ctypes.c_int64, _I, _I, _I, _I]),
     "bitsmoe_importance": (_I, [_P, _P, ctypes.c_int64, _I, _I, _I, _I, _I, ctypes.POINTER(_P), ctypes.POINTER(_P),
                                 ctypes.POINTER(_P), _P, _P, _SZ, _P]),
+    "bitsmoe_decompose_workspace_bytes": (_SZ, [_I, _I, _I, _I]),
+    "bitsmoe_shared_basis": (_I, [_I, _P, _I, _I, _I, _P, _P, _P, _P, _P, _SZ, _I, _P, _P, _P]),
+    "bitsmoe_calibration_gram": (_I, [_P, _P, ctypes.c_int64, _I, _P, _P]),
     "bitsmoe_block_norm_outputs": (_I, [_P, _I, _I, ctypes.POINTER(_SZ), ctypes.POINTER(_SZ)]),
     "bitsmoe_last_device_status": (_I, [_P, _P]),
     "bitsmoe_free": (None, [_P]),
@@ -469,6 +472,45 @@ def importance(x, logits, top_k: int, basis, alpha, factor, stream=None):
            "bitsmoe_importance")
     ws.record_stream(st)
     return beta
+
+
+def shared_basis(W, side: str, max_sweeps: int = 30, stream=None):
+    """Shared-basis decomposition of one projection type (torch fp32 on the device): side "in"
+    takes W = E x d x D (gate/up, W_e = d x D), side "out" W = E x D x d (down, W_e = D x d).
+    Returns (phi D x n, sigma n, alpha E x n, P E x n x d unit-major, sweeps, status) with
+    n = min(D, E d); sweeps and status are device int tensors (one element each)."""
+    import torch
+    sd = {"in": 0, "out": 1}[side]
+    E = int(W.shape[0])
+    d, D = (int(W.shape[1]), int(W.shape[2])) if sd == 0 else (int(W.shape[2]), int(W.shape[1]))
+    n = min(D, E * d)
+    dev = W.device
+    phi = torch.empty((D, n), dtype=torch.float32, device=dev)
+    sigma = torch.empty((n,), dtype=torch.float32, device=dev)
+    alpha = torch.empty((E, n), dtype=torch.float32, device=dev)
+    P = torch.empty((E, n, d), dtype=torch.float32, device=dev)
+    info = torch.zeros((2,), dtype=torch.int32, device=dev)   # sweeps, status
+    nb = int(_lib().bitsmoe_decompose_workspace_bytes(sd, E, d, D))
+    ws = torch.empty(nb + 256, dtype=torch.uint8, device=dev)
+    st = stream if stream is not None else torch.cuda.current_stream(dev)
+    _check(_lib().bitsmoe_shared_basis(sd, W.data_ptr(), E, d, D, phi.data_ptr(), sigma.data_ptr(), alpha.data_ptr(),
+                                       P.data_ptr(), (ws.data_ptr() + 255) // 256 * 256, nb, max_sweeps,
+                                       info.data_ptr(), info.data_ptr() + 4, st.cuda_stream),
+           "bitsmoe_shared_basis")
+    ws.record_stream(st)
+    return phi, sigma, alpha, P, info[0:1], info[1:2]
+
+
+def calibration_gram(x, g=None, stream=None):
+    """H = sum_t g_t x_t x_t^T (torch fp32 D x D) from x (torch int16 bf16 bit patterns, T x D)
+    and optional per-token weights g (fp32, T), on the device."""
+    import torch
+    T, D = int(x.shape[0]), int(x.shape[1])
+    H = torch.empty((D, D), dtype=torch.float32, device=x.device)
+    st = stream if stream is not None else torch.cuda.current_stream(x.device)
+    _check(_lib().bitsmoe_calibration_gram(x.data_ptr(), g.data_ptr() if g is not None else None, T, D,
+                                           H.data_ptr(), st.cuda_stream), "bitsmoe_calibration_gram")
+    return H
 
 
 def bitsmoe_debug_single_token_kernel(which: int) -> None:

@@ -1,13 +1,14 @@
 """Build libbitsmoe.so in-tree with nvcc for sm_103a (GB300).
 
-Nine translation units, compiled in parallel: the host packer (pack.cpp,
+Ten translation units, compiled in parallel: the host packer (pack.cpp,
 plain C++), the CUDA kernel chain + C ABI (forward.cu), the two fused
 single-token decode kernels (fused.cu, and the clustered one in fused2.cu),
 the tensor-core projections (gemm.cu), the tensor-core expert factors
 (expert_tc.cu), the per-unit quantiser from float spectral vectors
 (quantize.cu), the per-projection bit allocation (allocate.cu) and the
 importance beta from calibration tokens that the allocation weighs its losses
-by (importance.cu).  The CUDA runtime is linked statically, so the library
+by (importance.cu), and the shared-basis decomposition with the calibration
+Gram (decompose.cu).  The CUDA runtime is linked statically, so the library
 loads on a machine without a GPU (the host-only entry points then work; the
 device ones return BITSMOE_ERR_CUDA).
 """
@@ -43,7 +44,7 @@ def _run(cmd):
 
 def sources():
     return [os.path.join(CSRC, f) for f in ("pack.cpp", "forward.cu", "fused.cu", "fused2.cu", "gemm.cu", "expert_tc.cu",
-                                              "quantize.cu", "allocate.cu", "importance.cu")]
+                                              "quantize.cu", "allocate.cu", "importance.cu", "decompose.cu")]
 
 
 def up_to_date() -> bool:
