@@ -77,7 +77,7 @@ __device__ __forceinline__ void tile_fma(const float (*As)[kTM + 4], const float
 // of 8 with the next step's loads in flight during the current step's FMAs.
 template <typename T>
 __global__ void __launch_bounds__(kGT) k_gram(const T* __restrict__ A, const float* __restrict__ w, int64_t R, int D,
-                                              int64_t lda, float* __restrict__ G, int ntile) {
+                                              int64_t lda, float* __restrict__ G, int64_t ldg, int ntile) {
   __shared__ __align__(16) float As[2][kTK][kTM + 4];
   __shared__ __align__(16) float Bs[2][kTK][kTN + 4];
   int t = blockIdx.x, ta = 0;
@@ -127,8 +127,8 @@ __global__ void __launch_bounds__(kGT) k_gram(const T* __restrict__ A, const flo
     for (int j = 0; j < 8; ++j) {
       const int b = b0 + tx * 8 + j;
       if (a < D && b < D && (ta != tb || a <= b)) {   // exactly symmetric: one value per pair
-        G[(size_t)a * D + b] = acc[i][j];
-        G[(size_t)b * D + a] = acc[i][j];
+        G[(size_t)a * ldg + b] = acc[i][j];
+        G[(size_t)b * ldg + a] = acc[i][j];
       }
     }
   }
@@ -220,10 +220,12 @@ __global__ void k_transpose_out(const float* __restrict__ W, int E, int D, int d
 // one grid barrier per round suffices.
 // ---------------------------------------------------------------------------
 struct JacobiArgs {
-  float* G;          // n x n, symmetric, overwritten (diagonal: the eigenvalues)
-  float* Vt;         // n x n: row j = eigenvector j (set to the identity here)
+  float* G;          // n x ld (row stride ld), symmetric, overwritten (diagonal: the eigenvalues);
+                     // columns n .. ld - 1 zero
+  float* Vt;         // n x ld: row j = eigenvector j (set to the identity here)
   float2* tab;       // [2][m]: (a_jj, a_j,partner) of each index for a round
-  int n;
+  int n, ld;
+  int batch;         // pairs whose rows are in shared memory at once
   int max_sweeps;
   float tol;
   uint32_t* bar;     // grid-barrier counter (zero at launch)
@@ -231,6 +233,29 @@ struct JacobiArgs {
   int* sweeps;       // sweeps run (written by block 0)
   long long spin;    // bound of each barrier wait, in SM clocks
 };
+
+constexpr int kJBatch = 16;
+
+// Clock totals of the solver's phases per block, compiled in only with -DBITSMOE_JACOBI_TRACE
+// (timing studies): [0] rotations, [1] rows of G in, [2] rotations of G's rows, [3] rows of
+// V^T, [4] barrier.
+#ifdef BITSMOE_JACOBI_TRACE
+__device__ unsigned long long g_jacobi_trace[1024][8];
+#define JT_START() long long jt_ = clock64()
+#define JT_MARK(i)                                                            \
+  do {                                                                        \
+    const long long jn_ = clock64();                                          \
+    if (threadIdx.x == 0) g_jacobi_trace[blockIdx.x & 1023][(i)] += jn_ - jt_; \
+    jt_ = jn_;                                                                \
+  } while (0)
+#else
+#define JT_START() \
+  do {             \
+  } while (0)
+#define JT_MARK(i) \
+  do {             \
+  } while (0)
+#endif
 
 __device__ __forceinline__ int jacobi_player(int pos, int r, int m) { return pos == 0 ? 0 : 1 + (pos - 1 + r) % (m - 1); }
 __device__ __forceinline__ int jacobi_partner(int x, int r, int m) {
@@ -263,26 +288,72 @@ __device__ __forceinline__ bool grid_sync_bounded(uint32_t* bar, uint32_t target
   return *ok != 0;
 }
 
+__device__ __forceinline__ void cp16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+
+// Rows (lo, hi) of the batch's pairs of M (row stride ld) into X[2j], X[2j + 1] by 16-byte
+// copies of every thread, all in flight at once; only the rotated pairs when `only_rot`.
+__device__ __forceinline__ void jacobi_rows_in(const float* M, int ld, int bn, const int* blo, const int* bhi,
+                                              const float* sj, bool only_rot, int n, float* X) {
+  const int q4 = ld / 4;
+  for (int row = 0; row < 2 * bn; ++row) {
+    const int jj = row >> 1, x = (row & 1) ? bhi[jj] : blo[jj];
+    if (x >= n || (only_rot && sj[bhi[jj]] == 0.f)) continue;
+    for (int c4 = threadIdx.x; c4 < q4; c4 += blockDim.x)
+      cp16(X + (size_t)row * ld + 4 * c4, M + (size_t)x * ld + 4 * c4);
+  }
+  asm volatile("cp.async.wait_all;" ::: "memory");
+  __syncthreads();
+}
+// ... and back (16-byte stores through L2).
+__device__ __forceinline__ void jacobi_rows_out(float* M, int ld, int bn, const int* blo, const int* bhi,
+                                               const float* sj, bool only_rot, int n, const float* X) {
+  const int q4 = ld / 4;
+  for (int row = 0; row < 2 * bn; ++row) {
+    const int jj = row >> 1, x = (row & 1) ? bhi[jj] : blo[jj];
+    if (x >= n || (only_rot && sj[bhi[jj]] == 0.f)) continue;
+    for (int c4 = threadIdx.x; c4 < q4; c4 += blockDim.x)
+      __stcg(reinterpret_cast<float4*>(M + (size_t)x * ld) + c4,
+             *reinterpret_cast<const float4*>(X + (size_t)row * ld + 4 * c4));
+  }
+}
+// Row rotation of the batch's row pairs in place (16 bytes a thread at a time).
+__device__ __forceinline__ void jacobi_rotate_rows(int ld, int bn, const int* blo, const int* bhi, const float* cj,
+                                                   const float* sj, bool only_rot, float* X) {
+  const int q4 = ld / 4;
+  for (int jj = 0; jj < bn; ++jj) {
+    const int lo = blo[jj], hi = bhi[jj];
+    const float c = cj[lo], s_lo = sj[lo], s_hi = sj[hi];
+    if (only_rot && s_hi == 0.f) continue;
+    float4* xl = reinterpret_cast<float4*>(X + (size_t)(2 * jj) * ld);
+    float4* xh = reinterpret_cast<float4*>(X + (size_t)(2 * jj + 1) * ld);
+    for (int c4 = threadIdx.x; c4 < q4; c4 += blockDim.x) {
+      const float4 a = xl[c4], b = xh[c4];
+      xl[c4] = make_float4(c * a.x + s_lo * b.x, c * a.y + s_lo * b.y, c * a.z + s_lo * b.z, c * a.w + s_lo * b.w);
+      xh[c4] = make_float4(c * b.x + s_hi * a.x, c * b.y + s_hi * a.y, c * b.z + s_hi * a.z, c * b.w + s_hi * a.w);
+    }
+  }
+}
+
 __global__ void __launch_bounds__(512, 1) k_jacobi(JacobiArgs ja) {
   extern __shared__ __align__(16) uint8_t jsm[];
-  const int n = ja.n, m = n + (n & 1), half = m / 2;
-  int* partner = reinterpret_cast<int*>(jsm);             // [m]
-  float* cj = reinterpret_cast<float*>(partner + m);      // [m]
-  float* sj = cj + m;                                     // [m]
-  float* xp = sj + m;                                     // [m] lower row of a pair after the row rotation
-  float* xq = xp + m;                                     // [m] upper row
+  const int n = ja.n, ld = ja.ld, m = n + (n & 1), half = m / 2;
+  float* X = reinterpret_cast<float*>(jsm);                           // [2 batch][ld] a batch's rows
+  int* partner = reinterpret_cast<int*>(X + (size_t)2 * ja.batch * ld);   // [m]
+  float* cj = reinterpret_cast<float*>(partner + m);                  // [m]
+  float* sj = cj + m;                                                 // [m]
   __shared__ int active, ok;
+  // a batch's pairs: lower and upper index, first player, next partners, rotated diagonal
+  __shared__ int blo[kJBatch], bhi[kJBatch], bp[kJBatch], bnl[kJBatch], bnh[kJBatch];
+  __shared__ float bdl[kJBatch], bdh[kJBatch];
   const int tid = threadIdx.x, nt = blockDim.x, blk = blockIdx.x, nb = gridDim.x;
-  if (tid == 0) {   // the dummy column (odd n) reads as 0
-    xp[m - 1] = 0.f;
-    xq[m - 1] = 0.f;
-  }
-  // V^T = I; the table of round 0
-  for (size_t i = (size_t)blk * nt + tid; i < (size_t)n * n; i += (size_t)nb * nt)
-    ja.Vt[i] = (i / n == i % n) ? 1.f : 0.f;
+  // V^T = I (padding columns 0); the table of round 0
+  for (size_t i = (size_t)blk * nt + tid; i < (size_t)n * ld; i += (size_t)nb * nt)
+    ja.Vt[i] = (i / ld == i % ld) ? 1.f : 0.f;
   for (int x = blk * nt + tid; x < m; x += nb * nt) {
     const int y = jacobi_partner(x, 0, m);
-    ja.tab[x] = x < n ? make_float2(ja.G[(size_t)x * n + x], y < n ? ja.G[(size_t)x * n + y] : 0.f)
+    ja.tab[x] = x < n ? make_float2(ja.G[(size_t)x * ld + x], y < n ? ja.G[(size_t)x * ld + y] : 0.f)
                       : make_float2(0.f, 0.f);
   }
   uint32_t target = nb;
@@ -292,7 +363,7 @@ __global__ void __launch_bounds__(512, 1) k_jacobi(JacobiArgs ja) {
   __shared__ float dmax_s;
   {
     float dm = 0.f;
-    for (int x = tid; x < n; x += nt) dm = fmaxf(dm, fabsf(__ldcg(ja.G + (size_t)x * n + x)));
+    for (int x = tid; x < n; x += nt) dm = fmaxf(dm, fabsf(__ldcg(ja.G + (size_t)x * ld + x)));
     for (int o = 16; o; o >>= 1) dm = fmaxf(dm, __shfl_xor_sync(0xFFFFFFFFu, dm, o));
     if (tid == 0) dmax_s = 0.f;
     __syncthreads();
@@ -304,11 +375,13 @@ __global__ void __launch_bounds__(512, 1) k_jacobi(JacobiArgs ja) {
   for (; sweep < ja.max_sweeps; ++sweep) {
     int rotated = 0;
     for (int r = 0; r < m - 1; ++r, ++g) {
+      JT_START();
       const float2* tin = ja.tab + (size_t)(g & 1) * m;
       float2* tout = ja.tab + (size_t)((g + 1) & 1) * m;
       const int rn = r + 1 < m - 1 ? r + 1 : 0;   // the next round (of this sweep or the next)
       if (tid == 0) active = 0;
       __syncthreads();
+      // every rotation of the round, from the table
       int my_active = 0;
       for (int i = tid; i < half; i += nt) {
         const int p = jacobi_player(i, r, m), q = jacobi_player(m - 1 - i, r, m);
@@ -334,66 +407,84 @@ __global__ void __launch_bounds__(512, 1) k_jacobi(JacobiArgs ja) {
       if (my_active) atomicAdd(&active, my_active);
       __syncthreads();
       rotated += active;
-      for (int i = blk; i < half; i += nb) {
-        const int p = jacobi_player(i, r, m), q = jacobi_player(m - 1 - i, r, m);
-        const int lo = p < q ? p : q, hi = p < q ? q : p;   // hi may be the dummy
-        const float c = cj[lo], s_lo = sj[lo], s_hi = sj[hi];
-        const bool rot = s_hi != 0.f;
-        // the rotated 2 x 2 block: off-diagonal 0, diagonal a_xx + (s_x / c) a_pq (Golub &
-        // Van Loan's update, which keeps a_pp + a_qq to one rounding per element)
-        float dlo = 0.f, dhi = 0.f;
-        if (rot) {
-          const float2 tl = __ldcg(tin + lo), th = __ldcg(tin + hi);
-          const float apq = __ldcg(tin + p).y;
-          dlo = tl.x + (s_lo / c) * apq;
-          dhi = th.x + (s_hi / c) * apq;
-        }
-        float* gl = ja.G + (size_t)lo * n;
-        float* gh = hi < n ? ja.G + (size_t)hi * n : nullptr;
-        for (int k = tid; k < n; k += nt) {
-          const float vl = __ldcg(gl + k), vh = gh ? __ldcg(gh + k) : 0.f;
-          xp[k] = c * vl + s_lo * vh;
-          xq[k] = c * vh + s_hi * vl;
+      JT_MARK(0);
+      // this block's pairs i = blk, blk + nb, ..., in batches of ja.batch
+      const int npairs = blk < half ? (half - 1 - blk) / nb + 1 : 0;
+      for (int b0 = 0; b0 < npairs; b0 += ja.batch) {
+        const int bn = min(ja.batch, npairs - b0);
+        if (tid < bn) {   // the batch's pairs and the next round's partners of their rows
+          const int ii = blk + (b0 + tid) * nb;
+          const int p = jacobi_player(ii, r, m), q = jacobi_player(m - 1 - ii, r, m);
+          const int lo = p < q ? p : q, hi = p < q ? q : p;
+          blo[tid] = lo;
+          bhi[tid] = hi;
+          bp[tid] = p;
+          bnl[tid] = jacobi_partner(lo, rn, m);
+          bnh[tid] = hi < n ? jacobi_partner(hi, rn, m) : n;
+          if (sj[hi] != 0.f) {   // the rotated 2 x 2 block: off-diagonal 0, diagonal a_xx + (s_x / c) a_pq
+            // (Golub & Van Loan's update, which keeps a_pp + a_qq to one rounding per element)
+            const float apq = __ldcg(tin + p).y, cc = cj[lo];
+            bdl[tid] = __ldcg(tin + lo).x + (sj[lo] / cc) * apq;
+            bdh[tid] = hi < n ? __ldcg(tin + hi).x + (sj[hi] / cc) * apq : 0.f;
+          }
         }
         __syncthreads();
-        for (int k = tid; k < n; k += nt) {
+        // the rows of G (a dummy row reads as zeros)
+        for (int jj = 0; jj < bn; ++jj)
+          if (bhi[jj] >= n)
+            for (int k = tid; k < ld; k += nt) X[(size_t)(2 * jj + 1) * ld + k] = 0.f;
+        jacobi_rows_in(ja.G, ld, bn, blo, bhi, sj, false, n, X);
+        JT_MARK(1);
+        // row rotation in place, then the column rotation in place (index k with its partner:
+        // the lower of the two updates both), the rotated 2 x 2 blocks, the next table entries
+        jacobi_rotate_rows(ld, bn, blo, bhi, cj, sj, false, X);
+        __syncthreads();
+        for (int k = tid; k < m; k += nt) {
           const int pk = partner[k];
-          const float ck = cj[k], sk = sj[k];
-          float ol = ck * xp[k] + sk * xp[pk], oh = ck * xq[k] + sk * xq[pk];
-          if (rot && (k == hi || k == lo)) {
-            ol = k == hi ? 0.f : dlo;
-            oh = k == lo ? 0.f : dhi;
-          }
-          __stcg(gl + k, ol);
-          if (gh) __stcg(gh + k, oh);
-          // the next round's table entries of the two rows
-          const int nl = jacobi_partner(lo, rn, m);
-          if (k == lo) tout[lo].x = ol;
-          if (k == nl) tout[lo].y = ol;
-          if (gh) {
-            const int nh = jacobi_partner(hi, rn, m);
-            if (k == hi) tout[hi].x = oh;
-            if (k == nh) tout[hi].y = oh;
-          }
-        }
-        if (tid == 0) {   // a next partner past the matrix (the dummy) has no entry in the rows
-          if (jacobi_partner(lo, rn, m) >= n) tout[lo].y = 0.f;
-          if (gh && jacobi_partner(hi, rn, m) >= n) tout[hi].y = 0.f;
-          if (!gh) tout[hi] = make_float2(0.f, 0.f);
-        }
-        if (rot) {
-          float* vl_ = ja.Vt + (size_t)lo * n;
-          float* vh_ = ja.Vt + (size_t)hi * n;
-          for (int k = tid; k < n; k += nt) {
-            const float a = __ldcg(vl_ + k), b = __ldcg(vh_ + k);
-            __stcg(vl_ + k, c * a + s_lo * b);
-            __stcg(vh_ + k, c * b + s_hi * a);
+          if (pk < k) continue;   // the pair (k, pk) is updated once, by its lower index
+          const float ck = cj[k], sk = sj[k], cp = cj[pk], sp = sj[pk];
+          for (int row = 0; row < 2 * bn; ++row) {
+            float* xr = X + (size_t)row * ld;
+            const float a = xr[k], b = xr[pk];
+            xr[k] = ck * a + sk * b;
+            xr[pk] = cp * b + sp * a;
           }
         }
         __syncthreads();
+        if (tid < bn) {
+          const int lo = blo[tid], hi = bhi[tid];
+          float* xl = X + (size_t)(2 * tid) * ld;
+          float* xh = xl + ld;
+          if (sj[hi] != 0.f) {
+            xl[hi] = 0.f;
+            xl[lo] = bdl[tid];
+            if (hi < n) {
+              xh[lo] = 0.f;
+              xh[hi] = bdh[tid];
+            }
+          }
+          if (n & 1) {   // the dummy column stays 0
+            xl[m - 1] = 0.f;
+            xh[m - 1] = 0.f;
+          }
+          tout[lo] = make_float2(xl[lo], bnl[tid] < n ? xl[bnl[tid]] : 0.f);
+          tout[hi] = hi < n ? make_float2(xh[hi], bnh[tid] < n ? xh[bnh[tid]] : 0.f) : make_float2(0.f, 0.f);
+        }
+        __syncthreads();
+        jacobi_rows_out(ja.G, ld, bn, blo, bhi, sj, false, n, X);
+        __syncthreads();
+        JT_MARK(2);
+        // the rows of V^T of the batch's rotated pairs: row rotation only
+        jacobi_rows_in(ja.Vt, ld, bn, blo, bhi, sj, true, n, X);
+        jacobi_rotate_rows(ld, bn, blo, bhi, cj, sj, true, X);
+        __syncthreads();
+        jacobi_rows_out(ja.Vt, ld, bn, blo, bhi, sj, true, n, X);
+        __syncthreads();
+        JT_MARK(3);
       }
       target += nb;
       if (!grid_sync_bounded(ja.bar, target, ja.spin, ja.status, &ok)) return;
+      JT_MARK(4);
     }
     if (rotated == 0) break;
   }
@@ -404,7 +495,7 @@ __global__ void __launch_bounds__(512, 1) k_jacobi(JacobiArgs ja) {
 // each eigenvector (its largest |component| made positive, the first one on
 // ties), then Phi[:, rank] = sign * V^T[j, :] and sigma[rank] = sqrt(max(lambda, 0))
 // for the n_out leading ones.
-__global__ void k_order(const float* __restrict__ G, const float* __restrict__ Vt, int n, int n_out,
+__global__ void k_order(const float* __restrict__ G, const float* __restrict__ Vt, int n, int ld, int n_out,
                         float* __restrict__ phi, float* __restrict__ sigma) {
   const int j = blockIdx.x;   // one block per eigenvector
   __shared__ float red_v[32];
@@ -412,17 +503,17 @@ __global__ void k_order(const float* __restrict__ G, const float* __restrict__ V
   __shared__ float red_n[32];
   __shared__ int rank_s;
   __shared__ float scale_s;
-  const float lj = __ldg(G + (size_t)j * n + j);
+  const float lj = __ldg(G + (size_t)j * ld + j);
   int cnt = 0;
   for (int i = threadIdx.x; i < n; i += blockDim.x) {
-    const float li = __ldg(G + (size_t)i * n + i);
+    const float li = __ldg(G + (size_t)i * ld + i);
     cnt += (li > lj) | ((li == lj) & (i < j));
   }
   // largest |component| of V^T[j, :] (first on ties) and its squared norm (the vector is
   // rescaled to unit length: the rotations' rounding moves it by a few units in the last place)
   float bv = -1.f, nn = 0.f;
   int bi = 0x7FFFFFFF;
-  const float* vr = Vt + (size_t)j * n;
+  const float* vr = Vt + (size_t)j * ld;
   for (int i = threadIdx.x; i < n; i += blockDim.x) {
     const float v = vr[i], a = fabsf(v);
     nn = fmaf(v, v, nn);
@@ -528,8 +619,9 @@ DecLayout dec_layout(int side, int E, int d, int D) {
     return o;
   };
   l.A = take(side == 1 ? R * D * 4 : 0);
-  l.G = take((size_t)D * D * 4);
-  l.Vt = take((size_t)D * D * 4);
+  const size_t ld = (size_t)(D + (D & 1) + 3) / 4 * 4;   // row stride of G and V^T: 16-byte rows with the dummy column
+  l.G = take((size_t)D * ld * 4);
+  l.Vt = take((size_t)D * ld * 4);
   l.Pt = take(R * n * 4);
   l.tab = take((size_t)2 * (D + 1) * 8);
   l.sync = take(256);
@@ -563,7 +655,9 @@ extern "C" int bitsmoe_shared_basis(int side, const float* W, int E, int d, int 
   float* Pt = reinterpret_cast<float*>(wb + l.Pt);
   uint32_t* bar = reinterpret_cast<uint32_t*>(wb + l.sync);
   const float* A = W;
+  const size_t ld = (size_t)(D + (D & 1) + 3) / 4 * 4;
   BM_CK(cudaMemsetAsync(bar, 0, 256, st));
+  BM_CK(cudaMemsetAsync(G, 0, (size_t)D * ld * 4, st));   // the padding columns stay 0
   if (side == 1) {
     float* At = reinterpret_cast<float*>(wb + l.A);
     k_transpose_out<<<dim3((d + 31) / 32, (D + 31) / 32, E), dim3(32, 8), 0, st>>>(W, E, D, d, At);
@@ -571,24 +665,29 @@ extern "C" int bitsmoe_shared_basis(int side, const float* W, int E, int d, int 
     A = At;
   }
   const int ntile = (D + kTM - 1) / kTM;
-  k_gram<float><<<ntile * (ntile + 1) / 2, kGT, 0, st>>>(A, nullptr, R, D, D, G, ntile);
+  k_gram<float><<<ntile * (ntile + 1) / 2, kGT, 0, st>>>(A, nullptr, R, D, D, G, ld, ntile);
   BM_CK(cudaGetLastError());
   // the eigensolver: one block per SM, all resident (cooperative launch)
   int dev = 0, sms = 0;
   BM_CK(cudaGetDevice(&dev));
   BM_CK(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
   const int m = D + (D & 1);
-  const size_t smem = (size_t)m * 20;
+  const int nb = std::min(sms, m / 2);
+  const int per_block = (m / 2 + nb - 1) / nb;
+  const size_t room = 220 * 1024 - (size_t)m * 12;
+  const int batch = std::max(1, std::min({per_block, kJBatch, (int)(room / ((size_t)ld * 8))}));
+  const size_t smem = (size_t)m * 12 + (size_t)batch * ld * 8;
   BM_CK(cudaFuncSetAttribute(k_jacobi, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
   int per_sm = 0;
   BM_CK(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_jacobi, 512, smem));
   if (per_sm < 1) return BITSMOE_ERR_SHAPE;
-  const int nb = std::min(sms, m / 2);
   JacobiArgs ja;
   ja.G = G;
   ja.Vt = Vt;
   ja.tab = reinterpret_cast<float2*>(wb + l.tab);
   ja.n = D;
+  ja.ld = (int)ld;
+  ja.batch = batch;
   ja.max_sweeps = max_sweeps;
   ja.tol = 1e-7f;
   ja.bar = bar;
@@ -597,7 +696,7 @@ extern "C" int bitsmoe_shared_basis(int side, const float* W, int E, int d, int 
   ja.spin = 2ll << 30;
   void* args[] = {&ja};
   BM_CK(cudaLaunchCooperativeKernel(reinterpret_cast<void*>(k_jacobi), dim3(nb), dim3(512), args, smem, st));
-  k_order<<<D, 256, 0, st>>>(G, Vt, D, n, phi, sigma);
+  k_order<<<D, 256, 0, st>>>(G, Vt, D, ld, n, phi, sigma);
   BM_CK(cudaGetLastError());
   k_project<<<dim3((n + kTN - 1) / kTN, (unsigned)((R + kTM - 1) / kTM)), kGT, 0, st>>>(A, phi, R, D, n, Pt);
   BM_CK(cudaGetLastError());
@@ -615,7 +714,13 @@ extern "C" int bitsmoe_calibration_gram(const void* x, const float* g, int64_t T
     BM_CK(cudaMemsetAsync(H, 0, (size_t)D * D * 4, st));
     return BITSMOE_OK;
   }
-  k_gram<uint16_t><<<ntile * (ntile + 1) / 2, kGT, 0, st>>>(static_cast<const uint16_t*>(x), g, T, D, D, H, ntile);
+  k_gram<uint16_t><<<ntile * (ntile + 1) / 2, kGT, 0, st>>>(static_cast<const uint16_t*>(x), g, T, D, D, H, D, ntile);
   BM_CK(cudaGetLastError());
   return BITSMOE_OK;
 }
+
+#ifdef BITSMOE_JACOBI_TRACE
+extern "C" int bitsmoe_jacobi_trace_read(void* dst) {
+  return (int)cudaMemcpyFromSymbol(dst, g_jacobi_trace, sizeof(g_jacobi_trace));
+}
+#endif
