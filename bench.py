@@ -485,6 +485,19 @@ def run_reference_task(args, spec):
         }
         print(json.dumps(line), flush=True)
         return
+    if args.task == "decompose":
+        cpu = dec_oracle_rate(spec, budget_s=min(60.0, float(os.environ.get("BITSMOE_REF_BUDGET_S", "90"))))
+        n = min(spec.D, spec.E * spec.I)
+        line = {
+            "impl": "reference", "metric": DEC_METRIC, "value": cpu["value"], "unit": "units/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1000.0 * spec.E * n / cpu["value"], "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": dec_config(spec),
+            "cpu_baseline": cpu,
+            "e2e": {"value": cpu["value"], "unit": "units/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        }
+        print(json.dumps(line), flush=True)
+        return
     if args.task == "quantize":
         from oracle import quantizer as Q
         U = args.units or 3 * spec.E * spec.n
@@ -765,6 +778,135 @@ def imp_oracle_rate(spec, budget_s=12.0):
     return {"value": n_done / secs * (E / spec.E), "unit": "tokens/s", "cores": cpu_cores(), "kind": "oracle",
             "sample": f"{n_done} tokens through factor_importance on a layer with {E} experts of the workload's dims "
                       f"({secs:.1f} s), scaled to {spec.E} experts by the per-expert work"}
+
+
+DEC_METRIC = ("spectral units/s (shared-basis decomposition of one projection: Gram, Jacobi eigensolver, "
+              "basis, spectral energies and vectors)")
+
+
+def dec_config(spec):
+    return {"workload": f"shared-basis decomposition: the gate projection of a {spec.name} layer ({spec.E} experts "
+                        f"of {spec.I} x {spec.D} fp32 weights, rank {min(spec.D, spec.E * spec.I)})",
+            "experts": spec.E, "intermediate": spec.I, "hidden": spec.D, "side": "in",
+            "l2": f"weights {spec.E * spec.I * spec.D * 4 / 1e9:.2f} GB per step (129 MB L2)"}
+
+
+def dec_oracle_rate(spec, budget_s=20.0):
+    """The decomposition oracle (fp64 numpy SVD) on the host cores, on a bounded sample: the
+    workload's feature dimension with fewer experts (spectral units/s of the sample)."""
+    import oracle
+    rng = np.random.default_rng(6)
+    E = 8
+    W = [(rng.standard_normal((spec.I, spec.D)) / np.sqrt(spec.D)).astype(np.float32) for _ in range(E)]
+    n_units, secs, calls = 0, 0.0, 0
+    while secs < budget_s and calls < 4:
+        t0 = time.perf_counter()
+        oracle.shared_basis_decompose(W, "in")
+        secs += time.perf_counter() - t0
+        n_units += E * min(spec.D, E * spec.I)
+        calls += 1
+    return {"value": n_units / secs, "unit": "units/s", "cores": cpu_cores(), "kind": "oracle",
+            "sample": f"{calls} decompositions of {E} experts of {spec.I} x {spec.D} (oracle.shared_basis_decompose, "
+                      f"numpy SVD in fp64, {secs:.1f} s); the full workload has {spec.E} experts"}
+
+
+def run_decompose(args, spec, rank, world, local):
+    """Shared-basis decomposition of one Qwen3-shaped projection (gate: E experts of I x D fp32
+    weights, N(0, 1/D)) per step: bitsmoe_shared_basis, all of its launches timed."""
+    import torch
+    import paper_2606_00079_gb300 as bm
+    dev = torch.device("cuda", local)
+    E, I, D = spec.E, spec.I, spec.D
+    n = min(D, E * I)
+    g = torch.Generator(device=dev)
+    g.manual_seed(5000 + rank)
+    W = (torch.randn((E, I, D), generator=g, device=dev) / float(np.sqrt(D))).contiguous()
+    stream = torch.cuda.Stream(device=dev)
+    phi = torch.empty((D, n), dtype=torch.float32, device=dev)
+    sig = torch.empty((n,), dtype=torch.float32, device=dev)
+    alpha = torch.empty((E, n), dtype=torch.float32, device=dev)
+    P = torch.empty((E, n, I), dtype=torch.float32, device=dev)
+    info = torch.zeros((2,), dtype=torch.int32, device=dev)
+    nb = int(bm._lib().bitsmoe_decompose_workspace_bytes(0, E, I, D))
+    ws = torch.empty(nb + 256, dtype=torch.uint8, device=dev)
+    wsp = (ws.data_ptr() + 255) // 256 * 256
+
+    def step():
+        bm._check(bm._lib().bitsmoe_shared_basis(0, W.data_ptr(), E, I, D, phi.data_ptr(), sig.data_ptr(),
+                                                alpha.data_ptr(), P.data_ptr(), wsp, nb, 30, info.data_ptr(),
+                                                info.data_ptr() + 4, stream.cuda_stream), "bitsmoe_shared_basis")
+
+    with torch.cuda.stream(stream):
+        for _ in range(max(3, min(args.warmup, 3))):
+            step()
+    stream.synchronize()
+    clk = ClockSampler(local)
+    clk.start()
+    rank_barrier(world)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clk.mark("t0")
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    e1.synchronize()
+    clk.mark("t1")
+    torch.cuda.synchronize()
+    rank_barrier(world)
+    ms_own = e0.elapsed_time(e1)
+    ms = max_over_ranks(ms_own, world, dev)
+    clocks = clk.stop()
+    sweeps, status = int(info[0].item()), int(info[1].item())
+    if status != 0:
+        raise RuntimeError(f"bitsmoe_shared_basis device status {status}")
+    value = world * args.steps * E * n / (ms / 1e3)
+    sec = ms_own / args.steps / 1e3
+    # the dominant kernel is the Jacobi solver (its share: the launch list under profiles/); its
+    # arithmetic per round: 8 flops per element of G (row and column rotations) and 4 per element
+    # of V^T, D^2 elements each, (D - 1) rounds a sweep, sweeps + 1 sweeps (the last one checks)
+    m = D + (D & 1)
+    jac_flops = 12.0 * D * D * (m - 1) * (sweeps + 1 if sweeps < 30 else 30)
+    peaks, _ = measured_peaks()
+    sm_mhz = clocks.get("sm_mhz") or float(peaks.get("sm_max_mhz", 2070.0))
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    peak = sms * FP32_FLOPS_PER_SM_CLK * sm_mhz * 1e6 / 1e12
+    roofline = {"bound": "alu", "kernel": "k_jacobi (cyclic Jacobi eigensolver of the D x D Gram matrix, fp32)",
+                "achieved": jac_flops / sec / 1e12, "peak": peak, "unit": "TFLOP/s",
+                "frac": jac_flops / sec / 1e12 / peak,
+                "peak_source": f"{sms} SMs x 128 fp32 lanes x 2 flops x {sm_mhz:.0f} MHz (median SM clock under load)",
+                "note": "the whole call's time in the denominator; the solver is bound by its rounds (one grid "
+                        "barrier and a pass over its rows of G and V^T each), not by arithmetic",
+                "traffic": None, "flops_per_launch": jac_flops, "duration_us": sec * 1e6, "sweeps": sweeps}
+    # e2e: weights in from pinned host memory, basis + energies + spectral vectors back, every step
+    ne = 2
+    Wh = W.cpu().pin_memory()
+    Ph = torch.empty_like(P, device="cpu").pin_memory()
+    phih = torch.empty_like(phi, device="cpu").pin_memory()
+    ah = torch.empty_like(alpha, device="cpu").pin_memory()
+    t0 = time.perf_counter()
+    for _ in range(ne):
+        with torch.cuda.stream(stream):
+            W.copy_(Wh, non_blocking=True)
+            step()
+            Ph.copy_(P, non_blocking=True)
+            phih.copy_(phi, non_blocking=True)
+            ah.copy_(alpha, non_blocking=True)
+        stream.synchronize()
+    e2e_s = time.perf_counter() - t0
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = dec_oracle_rate(spec, budget_s=20.0)
+    if rank == 0:
+        line = {
+            "metric": DEC_METRIC, "value": value, "unit": "units/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": dec_config(spec),
+            "roofline": roofline, "cpu_baseline": cpu, "clocks": clocks, "gpu_launches": 6 * args.steps,
+            "e2e": {"value": world * ne * E * n / e2e_s, "unit": "units/s", "steps": ne,
+                    "h2d_bytes_per_step": E * I * D * 4, "d2h_bytes_per_step": (E * n * I + D * n + E * n) * 4},
+        }
+        print(json.dumps(line), flush=True)
 
 
 ALLOC_METRIC = "spectral units allocated/s (per-projection bit allocation: costs, Lagrangian cut, greedy fill)"
@@ -1109,10 +1251,12 @@ def main():
     ap.add_argument("--inputs", type=int, default=64)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--graph", type=int, default=256, help="forwards per captured CUDA graph")
-    ap.add_argument("--task", default="forward", choices=["forward", "quantize", "allocate", "importance"],
+    ap.add_argument("--task", default="forward",
+                    choices=["forward", "quantize", "allocate", "importance", "decompose"],
                     help="forward: the MoE-layer forward (default); quantize: the per-unit quantiser; "
                          "allocate: the per-projection bit allocation; importance: the importance beta of "
-                         "every unit from calibration tokens")
+                         "every unit from calibration tokens; decompose: the shared-basis decomposition of "
+                         "one projection")
     ap.add_argument("--calib-tokens", type=int, default=4096,
                     help="calibration tokens per step of --task importance")
     ap.add_argument("--grid", type=int, default=256, help="scale candidates of the quantiser (--task quantize)")
@@ -1126,7 +1270,7 @@ def main():
     spec = synth.WORKLOADS[args.workload]
     T = args.tokens or spec.tokens[0]
     if args.steps is None and not args.all:
-        args.steps = 20 if args.task != "forward" else (20000 if spec.layers == 1 else 400)
+        args.steps = {"forward": 20000 if spec.layers == 1 else 400, "decompose": 3}.get(args.task, 20)
     if args.impl == "reference":
         if args.task == "forward":
             run_reference(args, spec, T)
@@ -1146,8 +1290,8 @@ def main():
     dev = torch.device("cuda", local)
 
     if args.task != "forward":
-        {"quantize": run_quantize, "allocate": run_allocate,
-         "importance": run_importance}[args.task](args, spec, rank, world, local)
+        {"quantize": run_quantize, "allocate": run_allocate, "importance": run_importance,
+         "decompose": run_decompose}[args.task](args, spec, rank, world, local)
         if world > 1:
             torch.distributed.barrier()
             torch.distributed.destroy_process_group()
