@@ -184,6 +184,25 @@ int bitsmoe_debug_wait_limit(int skip_arrival, long long spin_clocks);
  * BITSMOE_OK, or BITSMOE_ERR_INVALID_ARG for another value. */
 int bitsmoe_debug_single_token_kernel(int which);
 
+/* Testing hook (no counterpart in the paper; the stand-in for a memory checker,
+ * which this environment does not run): with on = 1 the single-token kernels
+ * (both fused kernels) check every staging record before they copy from the
+ * packed image -- each gate/up item's code, unit-index, alpha and scale/zero
+ * ranges and each down tile's, against the image's size -- and a record that
+ * fails is skipped (its item contributes nothing) and reported as
+ * BITSMOE_ERR_DEVICE_BOUNDS in the workspace status word (the call's output is
+ * then undefined).  Layers packed or loaded while it is on are given a
+ * zero-filled slack of the image's own size after the image.  Applies to calls
+ * issued after it; on = 0 turns the checks off.  Returns BITSMOE_OK. */
+int bitsmoe_debug_bounds(int on);
+
+/* Testing hook (no counterpart in the paper): add `delta` bytes to the code
+ * offset of every gate/up staging record of expert e (both fused kernels'
+ * tables), so that a test can make those records point outside the image
+ * (into the slack of a layer loaded under bitsmoe_debug_bounds(1)) and shift
+ * them back.  Synchronous.  Errors: INVALID_ARG, CUDA. */
+int bitsmoe_debug_shift_expert_records(const bitsmoe_layer* layer, int e, long long delta);
+
 /* Kernels one bitsmoe_moe_block_forward call launches: 1 a token when the
  * fused single-token kernel runs (it computes the pre-norm and router too),
  * otherwise the norm/router kernel plus bitsmoe_forward_launches. */

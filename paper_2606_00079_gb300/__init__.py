@@ -85,6 +85,8 @@ SIGNATURES = {
     "bitsmoe_last_cuda_error": (_I, []),
     "bitsmoe_debug_wait_limit": (_I, [_I, ctypes.c_longlong]),
     "bitsmoe_debug_single_token_kernel": (_I, [_I]),
+    "bitsmoe_debug_bounds": (_I, [_I]),
+    "bitsmoe_debug_shift_expert_records": (_I, [_P, _I, ctypes.c_longlong]),
 }
 
 
@@ -517,6 +519,17 @@ def bitsmoe_debug_single_token_kernel(which: int) -> None:
     """Testing hook: 1 keeps single-token forwards on the fused kernel without clusters, 2 takes the
     clustered one wherever it fits, 0 restores the automatic choice."""
     _check(_lib().bitsmoe_debug_single_token_kernel(which), "bitsmoe_debug_single_token_kernel")
+
+
+def bitsmoe_debug_bounds(on: int) -> None:
+    """Testing hook: debug bounds checks of the single-token kernels' staging records (and a
+    zero-filled slack after the image of layers packed while it is on)."""
+    _check(_lib().bitsmoe_debug_bounds(on), "bitsmoe_debug_bounds")
+
+
+def bitsmoe_debug_shift_expert_records(layer, e: int, delta: int) -> None:
+    """Testing hook: shift the code offsets of expert e's gate/up staging records by delta bytes."""
+    _check(_lib().bitsmoe_debug_shift_expert_records(layer.handle, e, delta), "bitsmoe_debug_shift_expert_records")
 
 
 def bitsmoe_debug_wait_limit(skip_arrival: int, spin_clocks: int) -> None:

@@ -15,6 +15,7 @@ namespace bmoe {
 
 struct Fwd {
   const uint8_t* img;
+  uint64_t img_bytes;   // size of the packed image (the bounds of the debug checks)
   const ExpertDesc* desc;
   const int32_t* seg;
   const ItemRec* items;
@@ -94,7 +95,8 @@ struct FusedArgs {
   int nslot_c, slot_c, nslot_d, slot_d; // gate/up and down staging slots (count, bytes)
   int off_route, off_xs, off_r1, off_d, off_rc, off_cq, off_rec, off_part, smem;
   int smax, s16, seg_al, ul_max_tiles, d_code_bytes, d_h_bytes;
-  int dbg;             // bit 0: block 0 skips its arrival at grid barrier 1 (tests of the bounded waits)
+  int dbg;             // bit 0: block 0 skips its arrival at grid barrier 1 (tests of the bounded waits);
+                       // bit 1: every staging record is checked against the image before its copies
   long long spin;      // bound of the grid-barrier waits, in SM clocks
 };
 
@@ -169,7 +171,8 @@ struct F2Args {
   int b_stage, b_nst;       // input-basis rows per stage, stages
   int s16;                 // int16 activation table row (elements) per warp and group
   int off_rec, off_route, off_xs, off_cq, off_pw, off_xch, off_h, off_r1, off_d, off_r2, off_ss, smem;
-  int dbg;                 // bit 0: block 0 skips its arrival at grid barrier 1 (tests of the bounded waits)
+  int dbg;                 // bit 0: block 0 skips its arrival at grid barrier 1 (tests of the bounded waits);
+                           // bit 1: every staging record is checked against the image before its copies
   int prefetch_io;         // x and the logits are device memory: prefetch them into L2 before the wait
   int rec_smem;            // this rank's record table fits the gate/up staging area (copied there first)
   long long spin;          // bound of every wait, in SM clocks

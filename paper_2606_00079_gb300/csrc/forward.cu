@@ -89,6 +89,10 @@ std::atomic<int> g_dbg_skip{0};
 // Testing hook (bitsmoe_debug_single_token_kernel): 1 keeps single-token forwards on the
 // kernel without clusters, 2 takes the clustered one wherever it fits.
 std::atomic<int> g_dbg_kernel{0};
+// testing hook: debug bounds checks in the single-token kernels; layers uploaded while it is
+// on get a zero-filled slack of the image's own size after it (so that a record shifted past
+// the image, as the tests do, still reads mapped memory)
+std::atomic<int> g_dbg_bounds{0};
 
 thread_local int g_last_cuda = 0;
 int cuda_fail(cudaError_t e) {
@@ -1506,6 +1510,7 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
   Fwd p;
   std::memset(&p, 0, sizeof(p));
   p.img = L->d_img;
+  p.img_bytes = L->bytes;
   p.desc = reinterpret_cast<const ExpertDesc*>(L->d_img + hd.off_desc);
   p.seg = reinterpret_cast<const int32_t*>(L->d_img + hd.off_seg);
   p.items = reinterpret_cast<const ItemRec*>(L->d_img + hd.off_items);
@@ -1559,7 +1564,7 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
     if (ci >= 0) {
       f2.cnt = reinterpret_cast<uint32_t*>(wb + w.sync);
       f2.tab = L->d_f2 + L->f2_off[ci];
-      f2.dbg = g_dbg_skip.load();
+      f2.dbg = g_dbg_skip.load() | (g_dbg_bounds.load() ? 2 : 0);
       f2.prefetch_io = host_io ? 0 : 1;   // no L2 prefetch of host memory mapped into the address space
       const long long sp = g_dbg_spin.load();
       if (sp > 0) f2.spin = sp;
@@ -1575,7 +1580,7 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
   if (p.decode && fused_plan(hd, T, top_k, L->seg_bytes, L->ul_max_chunks, p.s16, sms, &fa)) {
     // one token: the whole layer in one persistent kernel
     fa.cnt = reinterpret_cast<uint32_t*>(wb + w.sync);
-    fa.dbg = g_dbg_skip.load();
+    fa.dbg = g_dbg_skip.load() | (g_dbg_bounds.load() ? 2 : 0);
     if (g_dbg_spin.load() > 0) fa.spin = g_dbg_spin.load();
     fa.cst = L->d_cst;
     fa.dst = L->d_dst;
@@ -1719,8 +1724,10 @@ int upload(std::vector<uint8_t>&& img, int device, bitsmoe_layer** out) {
   uint8_t* d = nullptr;
   uint8_t* ds = nullptr;
   uint8_t* df2 = nullptr;
-  if (e == cudaSuccess) e = cudaMalloc(&d, img.size());
+  const size_t slack = g_dbg_bounds.load() ? img.size() : 0;
+  if (e == cudaSuccess) e = cudaMalloc(&d, img.size() + slack);
   if (e == cudaSuccess) e = cudaMemcpy(d, img.data(), img.size(), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess && slack) e = cudaMemset(d + img.size(), 0, slack);
   if (e == cudaSuccess) e = cudaMalloc(&ds, cst_bytes + dst_bytes + 16);
   if (e == cudaSuccess && cst_bytes) e = cudaMemcpy(ds, cst.data(), cst_bytes, cudaMemcpyHostToDevice);
   if (e == cudaSuccess && dst_bytes) e = cudaMemcpy(ds + cst_bytes, dst.data(), dst_bytes, cudaMemcpyHostToDevice);
@@ -2136,6 +2143,42 @@ int bitsmoe_debug_wait_limit(int skip_arrival, long long spin_clocks) {
   g_dbg_skip.store(skip_arrival ? 1 : 0);
   g_dbg_spin.store(spin_clocks > 0 ? spin_clocks : 0);
   return BITSMOE_OK;
+}
+
+int bitsmoe_debug_bounds(int on) {
+  g_dbg_bounds.store(on ? 1 : 0);
+  return BITSMOE_OK;
+}
+
+int bitsmoe_debug_shift_expert_records(const bitsmoe_layer* L, int e, long long delta) {
+  if (!L || e < 0) return BITSMOE_ERR_INVALID_ARG;
+  const ImageHeader& hd = L->hd();
+  if (e >= hd.E) return BITSMOE_ERR_INVALID_ARG;
+  int prev = 0;
+  BM_CK(cudaGetDevice(&prev));
+  BM_CK(cudaSetDevice(L->device));
+  auto shift = [&](uint8_t* rec) -> cudaError_t {   // the record's first field: its code offset
+    uint64_t v = 0;
+    cudaError_t r = cudaMemcpy(&v, rec, 8, cudaMemcpyDeviceToHost);
+    if (r != cudaSuccess) return r;
+    v += (uint64_t)delta;
+    return cudaMemcpy(rec, &v, 8, cudaMemcpyHostToDevice);
+  };
+  cudaError_t r = cudaSuccess;
+  // the kernel without clusters: CStage [2][E][nseg]
+  for (int h = 0; h < 2 && r == cudaSuccess; ++h)
+    for (int q = 0; q < hd.nseg && r == cudaSuccess; ++q)
+      r = shift(L->d_stage + (((size_t)h * hd.E + e) * hd.nseg + q) * sizeof(CStage));
+  // the clustered kernel: per cluster size, per rank [gate E][up E][down E]
+  const size_t rank_bytes = (size_t)hd.E * (2 * sizeof(F2Gu) + sizeof(F2Dn));
+  for (int i = 0; i < 5 && r == cudaSuccess; ++i) {
+    if (!L->f2_nc[i]) continue;
+    for (int rk = 0; rk < kF2Sizes[i] && r == cudaSuccess; ++rk)
+      for (int h = 0; h < 2 && r == cudaSuccess; ++h)
+        r = shift(L->d_f2 + L->f2_off[i] + rk * rank_bytes + ((size_t)h * hd.E + e) * sizeof(F2Gu));
+  }
+  cudaSetDevice(prev);
+  return r == cudaSuccess ? BITSMOE_OK : cuda_fail(r);
 }
 
 }  // extern "C"

@@ -159,6 +159,18 @@ __device__ float ul_tile_rt(int b, const uint8_t* code, int NRB, int rb0, int st
   return accf;
 }
 
+// The copies of a gate/up item of row block rb and of a down tile lie inside the image.
+template <int G>
+__device__ bool crec_ok(const Fwd& p, const CStage& r, int rb) {
+  const int g_base = (rb * kRows) / p.group;
+  return in_image(p, r.code0 + (uint64_t)rb * r.rb_stride, r.bytes) && in_image(p, r.unit0, r.mb) &&
+         in_image(p, r.alpha0, r.mb) && in_image(p, r.sz0 + (uint64_t)(g_base + G - 1) * r.sz_row, r.mb);
+}
+__device__ bool drec_ok(const Fwd& p, const DStage& r) {
+  return in_image(p, r.code, (uint64_t)p.NRB * ul_chunks((int)r.bits) * kChunkBytes) && in_image(p, r.unit, 128) &&
+         in_image(p, r.alpha, 128) && in_image(p, r.sz + (uint64_t)(p.NG - 1) * r.sz_row, 128);
+}
+
 // Copies of one gate/up item into a slot: [codes seg_al][unit smax][alpha smax][scale/zero G x smax].
 template <int G>
 __device__ void c_stage(const Fwd& p, const FusedArgs& f, const CStage& r, int rb, uint8_t* slot, uint64_t* bar) {
@@ -558,17 +570,26 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
         const CStage* g = f.cst + ((size_t)ci.h * p.E + sel_e[ci.a]) * p.nseg + ci.sg;
         if (m == ct) {
           copy_crec(crec + ct, g);
+          if ((f.dbg & 2) && crec[ct].bytes && !crec_ok<G>(p, crec[ct], ci.rb)) {
+            crec[ct].bytes = 0;
+            report_bounds(p.status);
+          }
           if (crec[ct].bytes) c_stage<G>(p, f, crec[ct], ci.rb, rc + (size_t)ct * f.slot_c, bar_c + ct);
         } else {
           const uint32_t bytes = __ldg(&g->bytes);
-          if (bytes) prefetch_run(p.img + __ldg(&g->code0) + (uint64_t)ci.rb * __ldg(&g->rb_stride), bytes);
+          const uint64_t o = __ldg(&g->code0) + (uint64_t)ci.rb * __ldg(&g->rb_stride);
+          if (bytes && (!(f.dbg & 2) || in_image(p, o, bytes))) prefetch_run(p.img + o, bytes);
         }
       }
     } else if (ct >= 32 && ct < 32 + f.nslot_d) {
       const int s = ct - 32;
       for (int m = s; m < md; m += f.nslot_d) {
         const int i = d_item(blk, m, nb), a = i % p.k, tile = f.ul_max_tiles - 1 - i / p.k;
-        const DStage r = load_drec(f.dst + (size_t)sel_e[a] * f.ul_max_tiles + tile);
+        DStage r = load_drec(f.dst + (size_t)sel_e[a] * f.ul_max_tiles + tile);
+        if ((f.dbg & 2) && r.bits && !drec_ok(p, r)) {
+          r.bits = 0;
+          report_bounds(p.status);
+        }
         if (m == s) drec[s] = r;
         else if (r.bits) prefetch_run(p.img + r.code, (uint64_t)p.NRB * ul_chunks((int)r.bits) * kChunkBytes);
       }
@@ -597,7 +618,13 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
       const CStage& r = crec[wid];
       if (m != wid) {   // a later item of this slot: its record replaces the previous one
         __syncwarp();
-        if (lane == 0) copy_crec(crec + wid, f.cst + ((size_t)ci.h * p.E + sel_e[ci.a]) * p.nseg + ci.sg);
+        if (lane == 0) {
+          copy_crec(crec + wid, f.cst + ((size_t)ci.h * p.E + sel_e[ci.a]) * p.nseg + ci.sg);
+          if ((f.dbg & 2) && crec[wid].bytes && !crec_ok<G>(p, crec[wid], ci.rb)) {
+            crec[wid].bytes = 0;
+            report_bounds(p.status);
+          }
+        }
         __syncwarp();
       }
       if (!r.bytes) continue;
@@ -651,6 +678,10 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
         const int i = d_item(blk, m, nb), tile = f.ul_max_tiles - 1 - i / p.k;
         a = i % p.k;
         r = rd == 0 ? drec[sl] : load_drec(f.dst + (size_t)sel_e[a] * f.ul_max_tiles + tile);
+        if (rd > 0 && (f.dbg & 2) && r.bits && !drec_ok(p, r)) {
+          r.bits = 0;
+          if (sub == 0 && lane == 0) report_bounds(p.status);
+        }
       }
       if (r.bits && rd > 0 && sub == 0 && lane == 0) {   // refill: the slot's previous tile is done
         fence_proxy_async();

@@ -526,6 +526,31 @@ __global__ void __launch_bounds__(kFThreads, 1) k_f2(Fwd p, F2Args f) {
       else if (lane < 10) copy_rec_words(ru, tr + ((size_t)p.E + e) * sizeof(F2Gu), 5, lane - 5);
       else if (lane < 17) copy_rec_words(rd, tr + (size_t)2 * p.E * sizeof(F2Gu) + (size_t)e * sizeof(F2Dn), 7, lane - 10);
       __syncwarp();
+      if ((f.dbg & 2) && lane == 0) {   // debug bounds checks of the three records
+        const int g_base = (rb * kRows) / p.group;
+        for (int h = 0; h < 2; ++h) {
+          F2Gu* r = h ? ru : rg;
+          const uint64_t ms = (uint64_t)r->nslot * 4;
+          if (r->bytes && !(in_image(p, r->code0 + (uint64_t)rb * r->rb_stride, r->bytes) &&
+                            in_image(p, r->unit0, ms) && in_image(p, r->alpha0, ms) &&
+                            in_image(p, r->sz0 + (uint64_t)(g_base + G - 1) * r->sz_row, ms))) {
+            r->bytes = 0;
+            report_bounds(p.status);
+          }
+        }
+        if (rd->nslot) {
+          const uint64_t ms = (uint64_t)rd->nslot * 4;
+          bool ok = in_image(p, rd->unit0, ms) && in_image(p, rd->alpha0, ms) &&
+                    in_image(p, rd->sz0 + (uint64_t)(g_base + G - 1) * rd->sz_row, ms);
+          for (int k = 0; k < rd->nr; ++k)
+            ok = ok && in_image(p, rd->code[k], (uint64_t)rd->ntl[k] * p.NRB * ul_chunks(rd->bits[k]) * kChunkBytes);
+          if (!ok) {
+            rd->nslot = 0;
+            report_bounds(p.status);
+          }
+        }
+      }
+      __syncwarp();
       fence_proxy_async();   // the table's generic reads before the copies that overwrite it
       if (rg->bytes) stage_gu<G>(p, *rg, rb, r2, 0, bar_g, lane);
       if (ru->bytes) stage_gu<G>(p, *ru, rb, r2, gu_lay(*rg, 0, G).end, bar_u, lane - 8);

@@ -84,6 +84,13 @@ __device__ __forceinline__ void prefetch_run(const uint8_t* p, uint64_t bytes) {
   }
 }
 
+// Debug bounds checks (dbg bit 1): a staging record's copies must lie inside the packed
+// image; a record that fails is reported as BITSMOE_ERR_DEVICE_BOUNDS and its item skipped.
+__device__ __forceinline__ bool in_image(const Fwd& p, uint64_t off, uint64_t len) {
+  return off <= p.img_bytes && len <= p.img_bytes - off;
+}
+__device__ __forceinline__ void report_bounds(int* status) { atomicCAS(status, 0, BITSMOE_ERR_DEVICE_BOUNDS); }
+
 // Issue `bytes` (16-byte multiple, 16-byte aligned) into shared memory on an
 // mbarrier whose transaction count the caller has set.
 __device__ __forceinline__ void bulk_run(void* dst, const uint8_t* src, uint32_t bytes, uint64_t* bar) {

@@ -306,6 +306,38 @@ def test_bounded_wait_runs_out_and_is_reported(env):
     check(env, layer, x, logits, spec.top_k, L=L, ws=ws)       # the counters were left at zero
 
 
+def test_debug_bounds_check_reports_and_skips(env):
+    """Debug bounds mode (the stand-in for a memory checker): the gate/up staging records of
+    the token's first-ranked expert are shifted by the image's size, past its end.  The layer
+    was loaded in that mode, so a zero-filled slack of the image's own size follows it, and the
+    shifted copies would read mapped zeros even if a check were missing.  The kernel reports
+    BITSMOE_ERR_DEVICE_BOUNDS and returns; with the records shifted back the next call on the
+    same workspace matches the oracle."""
+    torch, bm, kern = env
+    spec = small(E=8, top_k=2, n=72)
+    layer = synth.make_layer(spec, seed=45)
+    bm.bitsmoe_debug_bounds(1)
+    try:
+        L = bm.bitsmoe_pack(layer, device=0)
+        img = int(L.bytes()["total"])
+        ws = bm.Workspace(L, 1, spec.top_k)
+        x, logits = synth.make_inputs(spec, 1, seed=45)
+        e = int(np.argmax(logits[0]))
+        check(env, layer, x, logits, spec.top_k, L=L, ws=ws)       # in bounds: no report
+        assert bm.bitsmoe_last_device_status(ws.ptr) == 0
+        bm.bitsmoe_debug_shift_expert_records(L, e, img)
+        xd = torch.from_numpy(x.view(np.int16)).cuda()
+        ld = torch.from_numpy(logits).cuda()
+        bm.moe_forward(L, xd, ld, spec.top_k, ws=ws)
+        torch.cuda.synchronize()
+        assert bm.bitsmoe_last_device_status(ws.ptr) == bm.ERR_CODE["DEVICE_BOUNDS"]
+        bm.bitsmoe_debug_shift_expert_records(L, e, -img)
+        check(env, layer, x, logits, spec.top_k, L=L, ws=ws)
+        assert bm.bitsmoe_last_device_status(ws.ptr) == 0
+    finally:
+        bm.bitsmoe_debug_bounds(0)
+
+
 def test_clustered_plan_for_qw3_dims(env):
     """The Qwen3-shaped layer (full dims, top-8) runs on the clustered kernel at one token when
     it is forced (the device holds a cluster per (routing slot, row block) pair) and on the
