@@ -767,11 +767,11 @@ __device__ __forceinline__ void ul_tile(const Fwd& p, const uint8_t* code, int r
 // ---------------------------------------------------------------------------
 constexpr int kK2DecWarps = 4;
 constexpr int kDecMaxT = 8;        // decode mode: at most this many tokens
-constexpr int kZ = 4;              // item slots per lane whose z values are gathered at once (larger items loop)
+constexpr int kZ = 12;             // item slots per lane whose z values are gathered at once
 constexpr int kK3DecWarps = 4;
 
 template <int G, int TB>
-__global__ void __launch_bounds__(kK2DecWarps * 32, 3) k_gateup_dec(Fwd p) {
+__global__ void __launch_bounds__(kK2DecWarps * 32) k_gateup_dec(Fwd p) {
   pdl_trigger();
   extern __shared__ int4 smem_k2d[];
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
