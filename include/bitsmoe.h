@@ -242,6 +242,18 @@ int bitsmoe_moe_forward_host(const void* x_host, const float* logits_host, int T
                              const bitsmoe_layer* layer, float* y_host,
                              void* ws, size_t ws_bytes, void* stream);
 
+/* The same without the final synchronisation (no counterpart in the paper: for
+ * a serving loop that keeps several steps in flight): every copy and kernel is
+ * enqueued on `stream` and the call returns.  The caller synchronises the
+ * stream (or an event recorded after the call) before it reads y_host or
+ * writes x_host / logits_host again; with pageable buffers the copies are
+ * synchronous as in cudaMemcpyAsync.  Consecutive single-token calls on the
+ * fused kernel overlap each other's prologue (programmatic dependent launch),
+ * as bitsmoe_moe_forward does. */
+int bitsmoe_moe_forward_host_async(const void* x_host, const float* logits_host, int T, int top_k,
+                                   const bitsmoe_layer* layer, float* y_host,
+                                   void* ws, size_t ws_bytes, void* stream);
+
 /* Pre-norm of one MoE block of a decoder stack (the 48-layer MoE FFN stack
  * workload; attention is outside this library):
  *   r = h / sqrt(mean_d h^2 + eps)  (RMSNorm with unit weight), x = bf16(r),

@@ -60,6 +60,7 @@ SIGNATURES = {
     "bitsmoe_forward_plan": (_I, [_P, _I, _I]),
     "bitsmoe_moe_forward": (_I, [_P, _P, _I, _I, _P, _P, _P, _SZ, _P]),
     "bitsmoe_moe_forward_host": (_I, [_P, _P, _I, _I, _P, _P, _P, _SZ, _P]),
+    "bitsmoe_moe_forward_host_async": (_I, [_P, _P, _I, _I, _P, _P, _P, _SZ, _P]),
     "bitsmoe_moe_forward_noalloc": (_I, [_P, _P, _I, _I, _P, _P, _P]),
     "bitsmoe_noalloc_last_status": (_I, [_P]),
     "bitsmoe_rmsnorm_router": (_I, [_P, _P, ctypes.c_float, _I, _I, _I, _P, _P, _P]),

@@ -1989,8 +1989,8 @@ int bitsmoe_moe_forward(const void* x, const float* logits, int T, int top_k, co
   return forward_impl(x, logits, T, top_k, L, y, ws, ws_bytes, static_cast<cudaStream_t>(stream));
 }
 
-int bitsmoe_moe_forward_host(const void* x_host, const float* logits_host, int T, int top_k,
-                             const bitsmoe_layer* L, float* y_host, void* ws, size_t ws_bytes, void* stream) {
+static int forward_host(const void* x_host, const float* logits_host, int T, int top_k, const bitsmoe_layer* L,
+                        float* y_host, void* ws, size_t ws_bytes, void* stream, bool sync) {
   if (!L || T < 0) return BITSMOE_ERR_INVALID_ARG;
   const ImageHeader& hd = L->hd();
   if (top_k < 1 || top_k > std::min(hd.E, 32)) return BITSMOE_ERR_INVALID_ARG;
@@ -2015,7 +2015,7 @@ int bitsmoe_moe_forward_host(const void* x_host, const float* logits_host, int T
       rc = forward_impl(xd, static_cast<const float*>(ld), T, top_k, L, static_cast<float*>(yd), ws, ws_bytes, st,
                         nullptr, false, nullptr, true);
       if (rc) return rc;
-      BM_CK(cudaStreamSynchronize(st));
+      if (sync) BM_CK(cudaStreamSynchronize(st));
       return BITSMOE_OK;
     }
   }
@@ -2025,8 +2025,18 @@ int bitsmoe_moe_forward_host(const void* x_host, const float* logits_host, int T
                     reinterpret_cast<float*>(wb + w.y_stage), ws, ws_bytes, st);
   if (rc) return rc;
   BM_CK(cudaMemcpyAsync(y_host, wb + w.y_stage, (size_t)T * hd.D * 4, cudaMemcpyDeviceToHost, st));
-  BM_CK(cudaStreamSynchronize(st));
+  if (sync) BM_CK(cudaStreamSynchronize(st));
   return BITSMOE_OK;
+}
+
+int bitsmoe_moe_forward_host(const void* x_host, const float* logits_host, int T, int top_k,
+                             const bitsmoe_layer* L, float* y_host, void* ws, size_t ws_bytes, void* stream) {
+  return forward_host(x_host, logits_host, T, top_k, L, y_host, ws, ws_bytes, stream, true);
+}
+
+int bitsmoe_moe_forward_host_async(const void* x_host, const float* logits_host, int T, int top_k,
+                                   const bitsmoe_layer* L, float* y_host, void* ws, size_t ws_bytes, void* stream) {
+  return forward_host(x_host, logits_host, T, top_k, L, y_host, ws, ws_bytes, stream, false);
 }
 
 int bitsmoe_profile_forward(const void* x, const float* logits, int T, int top_k, const bitsmoe_layer* L,

@@ -189,6 +189,35 @@ def test_host_buffer_single_token_pinned_and_pageable(env):
     assert bm.bitsmoe_last_device_status(ws.ptr, 0) == 0
 
 
+@pytest.mark.parametrize("T", [1, 3])
+def test_host_buffer_async_steps_in_flight(env, T):
+    """The asynchronous host-buffer entry point: six steps enqueued back to back on one
+    stream and workspace, each with its own pinned input and output buffers (for T = 1 the
+    fused kernel reads and writes them in place), one synchronisation at the end; every
+    step's output matches the oracle."""
+    torch, bm = env
+    spec = small()
+    layer = synth.make_layer(spec, seed=13, alpha_scale=3.0)
+    L = bm.bitsmoe_pack(layer, device=0)
+    ws = bm.Workspace(L, T, spec.top_k)
+    st = torch.cuda.Stream()
+    steps = []
+    for step in range(6):
+        x, logits = synth.make_inputs(spec, T, seed=13, step=step)
+        xp = torch.from_numpy(x.view(np.int16).copy()).pin_memory()
+        lp = torch.from_numpy(logits.copy()).pin_memory()
+        yp = torch.full((T, spec.D), float("nan"), dtype=torch.float32).pin_memory()
+        rc = bm._lib().bitsmoe_moe_forward_host_async(xp.data_ptr(), lp.data_ptr(), T, spec.top_k, L.handle,
+                                                      yp.data_ptr(), ws.ptr, ws.nbytes, st.cuda_stream)
+        assert rc == 0
+        steps.append((x, logits, xp, lp, yp))
+    st.synchronize()
+    for x, logits, _, _, yp in steps:
+        ref = oracle.moe_forward_factored(layer, x, logits, spec.top_k)
+        assert rel_err(yp.numpy().astype(np.float64), ref) <= TOL
+    assert bm.bitsmoe_last_device_status(ws.ptr, 0) == 0
+
+
 def test_blob_upload_and_device_unpack_roundtrip(env):
     torch, bm = env
     spec = small()
