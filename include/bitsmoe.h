@@ -171,7 +171,7 @@ int bitsmoe_forward_plan(const bitsmoe_layer* layer, int T, int top_k);
  * second), and when skip_arrival is 1 let block 0 skip its arrival at the
  * first grid barrier, so that every other block's bounded wait runs out.  The
  * calls after it report BITSMOE_ERR_TIMEOUT through the device status word and
- * return; the workspace is left zeroed for the next call.  Applies to calls
+ * return; the workspace is left ready for the next call.  Applies to calls
  * issued after it on any host thread; skip_arrival = 0 with spin_clocks = 0
  * restores the normal behaviour.  Returns BITSMOE_OK. */
 int bitsmoe_debug_wait_limit(int skip_arrival, long long spin_clocks);
@@ -219,10 +219,11 @@ int bitsmoe_block_forward_launches(const bitsmoe_layer* layer, int T, int top_k)
  *   ws      device workspace of >= bitsmoe_workspace_bytes(layer, T, top_k)
  *           bytes, 256-byte aligned, owned by the caller; must not be used by
  *           another call in flight.  Zero-fill it once before its first use
- *           (the single-token kernel keeps grid-barrier counters in its first
- *           bytes, and every call leaves them at zero again); it may then be
- *           reused across calls, layers and token counts.  A workspace whose
- *           counters are not zero is reported as BITSMOE_ERR_WORKSPACE_STATE
+ *           (the single-token kernel keeps a call count and two sets of
+ *           grid-barrier counters in its first 64 bytes; each call uses one set
+ *           and clears the other for the next call); it may then be reused
+ *           across calls, layers and token counts.  A workspace whose counters
+ *           are not in that state is reported as BITSMOE_ERR_WORKSPACE_STATE
  *           by bitsmoe_last_device_status and the call computes nothing.
  * Host-side argument checks only: never allocates, never synchronises. */
 int bitsmoe_moe_forward(const void* x, const float* logits, int T, int top_k,

@@ -83,7 +83,7 @@ static_assert(sizeof(DStage) == 48, "DStage layout");
 // Fused single-token decode kernel (fused.cu): workspace pointers and the
 // shared-memory plan chosen on the host.
 struct FusedArgs {
-  uint32_t* cnt;     // [4] grid-barrier counters
+  uint32_t* sync;    // [kSyncWords] epoch and two sets of barrier counters (fused_common.cuh)
   const CStage* cst; // [2][E][nseg]
   const DStage* dst; // [E][ul_max_tiles] (directly after cst)
   uint64_t tab_bytes;  // bytes of both tables
@@ -162,7 +162,7 @@ __host__ __device__ inline int rl_split_at(const uint8_t* bits, const uint16_t* 
 
 // Launch plan of the clustered kernel (fused2.cu).
 struct F2Args {
-  uint32_t* cnt;           // grid-barrier counters (workspace)
+  uint32_t* sync;          // [kSyncWords] epoch and two sets of barrier counters (workspace)
   const uint8_t* tab;      // records of this cluster size: per rank [gate E][up E][down E]
   uint32_t rank_bytes;     // bytes of one rank's records
   int CL, npairs;          // cluster size; (routing slot, row block) pairs, one per cluster

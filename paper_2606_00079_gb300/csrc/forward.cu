@@ -1213,7 +1213,7 @@ WsLayout ws_layout(const ImageHeader& hd, int T, int k) {
     return o;
   };
   const size_t P = (size_t)T * k;
-  w.status = take(64);   // [0] status, [1] routing flag; bytes 32..47: fused-kernel barrier counters
+  w.status = take(64);   // [0] status, [1] routing flag, [2] router block count; bytes 16..63: single-token kernels' sync words
   w.pair_expert = take(P * 4);
   w.pair_weight = take(P * 4);
   w.expert_count = take((size_t)hd.E * 4);
@@ -1230,7 +1230,7 @@ WsLayout ws_layout(const ImageHeader& hd, int T, int k) {
   w.x_stage = take((size_t)T * hd.D * 2);
   w.logits_stage = take((size_t)T * hd.E * 4);
   w.y_stage = take((size_t)T * hd.D * 4);
-  w.sync = w.status + 32;   // fixed offset: no other layout of the workspace writes there
+  w.sync = w.status + 16;   // fixed offset: no other layout of the workspace writes there (12 words)
   w.total = off;
   return w;
 }
@@ -1562,7 +1562,7 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
     F2Args f2;
     const int ci = f2_choose(L, top_k, &f2);
     if (ci >= 0) {
-      f2.cnt = reinterpret_cast<uint32_t*>(wb + w.sync);
+      f2.sync = reinterpret_cast<uint32_t*>(wb + w.sync);
       f2.tab = L->d_f2 + L->f2_off[ci];
       f2.dbg = g_dbg_skip.load() | (g_dbg_bounds.load() ? 2 : 0);
       f2.prefetch_io = host_io ? 0 : 1;   // no L2 prefetch of host memory mapped into the address space
@@ -1579,7 +1579,7 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
   FusedArgs fa;
   if (p.decode && fused_plan(hd, T, top_k, L->seg_bytes, L->ul_max_chunks, p.s16, sms, &fa)) {
     // one token: the whole layer in one persistent kernel
-    fa.cnt = reinterpret_cast<uint32_t*>(wb + w.sync);
+    fa.sync = reinterpret_cast<uint32_t*>(wb + w.sync);
     fa.dbg = g_dbg_skip.load() | (g_dbg_bounds.load() ? 2 : 0);
     if (g_dbg_spin.load() > 0) fa.spin = g_dbg_spin.load();
     fa.cst = L->d_cst;

@@ -401,20 +401,26 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
     if (o < f.tab_bytes)
       prefetch_run(reinterpret_cast<const uint8_t*>(f.cst) + o, min(per, f.tab_bytes - o));
   }
-  if (wid >= kBW) route_token(nullptr, p.E, p.k, keys, sel_e, sel_w, tid - kBW * 32);   // code warm-up
   __syncthreads();
-  pdl_wait();   // x, logits, y and the workspace belong to earlier kernels until here
+  pdl_trigger();   // the next call's blocks may take SMs as soon as this call's leave
+  pdl_wait();      // x, logits, y and the workspace belong to earlier kernels until here
   if (threadIdx.x == 0) F1_MARK(1);
+  const uint32_t epoch = __ldcg(f.sync);
+  uint32_t* cnt = sync_set(f.sync, epoch);
 
-  // the workspace's barrier counters must be zero (only counter 0 can move before
+  // counters 1 and 2 of this call's set must be zero (counters 0 and 3 can move before
   // every block has passed this check)
   {
     int* bad = reinterpret_cast<int*>(part);
     if (tid == 0) {
-      const int v = (__ldcg(f.cnt + 1) | __ldcg(f.cnt + 2) | __ldcg(f.cnt + 3)) != 0u;
+      const int v = (__ldcg(cnt + 1) | __ldcg(cnt + 2)) != 0u;
       *bad = v;
-      if (v) atomicExch(p.status, BITSMOE_ERR_WORKSPACE_STATE);
-      else if (blk == 0) p.status[0] = 0;
+      if (v) {
+        atomicExch(p.status, BITSMOE_ERR_WORKSPACE_STATE);
+      } else if (blk == 0) {
+        p.status[0] = 0;
+        sync_clear_next(f.sync, epoch);
+      }
     }
     __syncthreads();
     if (*bad) {   // compute nothing; the projection rows already requested land before the block exits
@@ -520,7 +526,7 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
     // the block's z rows are written: arrive at barrier 1 without waiting for the control warps
     asm volatile("bar.sync 3, %0;" ::"r"(kBW * 32) : "memory");
     if (tid == 0) F1_MARK(5);
-    if (tid == 0 && !((f.dbg & 1) && blk == 0)) grid_arrive(f.cnt + 0);
+    if (tid == 0 && !((f.dbg & 1) && blk == 0)) grid_arrive(cnt + 0);
   } else {
     const int ct = tid - kBW * 32;
     if (f.norm) {
@@ -554,8 +560,8 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
         if (lane == 0) const_cast<float*>(p.logits)[e] = acc;
       }
       asm volatile("bar.sync 2, %0;" ::"r"(kCT) : "memory");
-      if (ct == 0) grid_arrive(f.cnt + 4);
-      grid_wait_ctl(f.cnt + 4, nb, p.status, seen + 3, cw, kCT, f.spin);
+      if (ct == 0) grid_arrive(cnt + 3);
+      grid_wait_ctl(cnt + 3, nb, p.status, seen + 3, cw, kCT, f.spin);
     }
     // ---- routing of the token
     route_token(p.logits, p.E, p.k, keys, sel_e, sel_w, ct);
@@ -596,7 +602,7 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
     }
   }
   if (tid == 0) F1_MARK(4);
-  grid_wait(f.cnt + 0, nb, p.status, seen + 0, f.spin);
+  grid_wait(cnt + 0, nb, p.status, seen + 0, f.spin);
   if (tid == 0) F1_MARK(6);
   // The projection rows are consumed; their buffer receives the first down tiles
   // (each staged by its slot's warp once that warp's gate/up items are done, so
@@ -645,7 +651,7 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
     d_stage(p, f, drec[wid], dslots + (size_t)wid * f.slot_d, bar_d + wid);
   }
   if (tid == 0) F1_MARK(7);
-  grid_barrier(f.cnt + 1, nb, p.status, seen + 1, f.spin);
+  grid_barrier(cnt + 1, nb, p.status, seen + 1, f.spin);
   if (tid == 0) F1_MARK(8);
 
   // ---- D: down tiles, s += w * alpha * P_dn^T h.  Warp w works on slot w % nslot_d
@@ -716,9 +722,9 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
     }
   }
   if (tid == 0) F1_MARK(9);
-  grid_barrier(f.cnt + 2, nb, p.status, seen + 2, f.spin);
+  grid_barrier(cnt + 2, nb, p.status, seen + 2, f.spin);
   if (tid == 0) F1_MARK(10);
-  pdl_trigger();   // every block is past its last wait on other blocks
+  if (tid == 0 && blk == 0) sync_finish(f.sync);   // every block has read the epoch
 
   // ---- E: y = Phi_dn s for rows [e0, e1)
   float* ss = reinterpret_cast<float*>(rc);
@@ -752,18 +758,6 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
     }
   }
   if (tid == 0) F1_MARK(11);
-  // the last block to finish resets the barrier counters for the next call
-  if (tid == 0) {
-    const uint32_t old = atomicAdd(f.cnt + 3, 1u);
-    if (old == (uint32_t)nb - 1) {
-      f.cnt[0] = 0u;
-      f.cnt[1] = 0u;
-      f.cnt[2] = 0u;
-      f.cnt[4] = 0u;
-      __threadfence();
-      f.cnt[3] = 0u;
-    }
-  }
 }
 
 }  // namespace

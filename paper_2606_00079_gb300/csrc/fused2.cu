@@ -469,13 +469,19 @@ __global__ void __launch_bounds__(kFThreads, 1) k_f2(Fwd p, F2Args f) {
   pdl_wait();      // x, logits, y and the workspace belong to earlier kernels until here
   if (tid == 0) F2_MARK(1);
 
-  // the workspace's barrier counters must be zero (counter 0 is the only one that can
-  // move before every block has passed this check)
+  const uint32_t epoch = __ldcg(f.sync);
+  uint32_t* cnt = sync_set(f.sync, epoch);
+  // counters 1 and 2 of this call's set must be zero (counter 0 is the only one of this
+  // kernel's that can move before every block has passed this check)
   if (tid == 0) {
-    const int v = (__ldcg(f.cnt + 1) | __ldcg(f.cnt + 2) | __ldcg(f.cnt + 3)) != 0u;
+    const int v = (__ldcg(cnt + 1) | __ldcg(cnt + 2)) != 0u;
     flags[2] = v;
-    if (v) atomicExch(p.status, BITSMOE_ERR_WORKSPACE_STATE);
-    else if (blk == 0) p.status[0] = 0;
+    if (v) {
+      atomicExch(p.status, BITSMOE_ERR_WORKSPACE_STATE);
+    } else if (blk == 0) {
+      p.status[0] = 0;
+      sync_clear_next(f.sync, epoch);
+    }
   }
   // x into shared memory (a token row inside a batch starts at 2*D*t bytes: 16-byte loads
   // only when x is 16-byte aligned), s cleared
@@ -589,7 +595,7 @@ __global__ void __launch_bounds__(kFThreads, 1) k_f2(Fwd p, F2Args f) {
   __syncthreads();   // z rows and the cleared s are written; the projection rows are consumed
   if (tid == 0) {
     F2_MARK(5);
-    if (!((f.dbg & 1) && blk == 0)) grid_arrive(f.cnt + 0);
+    if (!((f.dbg & 1) && blk == 0)) grid_arrive(cnt + 0);
     // the freed buffer: a pair block's down part now and its output-basis rows after the
     // z gathers of the next phase; a free block's output-basis rows now
     fence_proxy_async();
@@ -599,7 +605,7 @@ __global__ void __launch_bounds__(kFThreads, 1) k_f2(Fwd p, F2Args f) {
                bar_e);
     }
   }
-  grid_wait(f.cnt + 0, nb, p.status, flags + 0, f.spin);
+  grid_wait(cnt + 0, nb, p.status, flags + 0, f.spin);
   if (tid == 0) F2_MARK(6);
 
   // ---- C: gate (warps 0-7) and up (warps 8-15) of the cluster's row block over this
@@ -737,8 +743,9 @@ __global__ void __launch_bounds__(kFThreads, 1) k_f2(Fwd p, F2Args f) {
     if (ru->bytes) mbar_wait_for(bar_u, 0, f.spin);
   }
   if (tid == 0) F2_MARK(10);
-  grid_barrier(f.cnt + 1, nb, p.status, flags + 1, f.spin);
+  grid_barrier(cnt + 1, nb, p.status, flags + 1, f.spin);
   if (tid == 0) F2_MARK(11);
+  if (tid == 0 && blk == 0) sync_finish(f.sync);   // every block has read the epoch
 
   // ---- E: y = Phi_dn s for rows [e0, e1)
   float* ss = reinterpret_cast<float*>(fsm + f.off_ss);
@@ -774,16 +781,6 @@ __global__ void __launch_bounds__(kFThreads, 1) k_f2(Fwd p, F2Args f) {
   if (tid == 0) F2_MARK(12);
   // every copy into shared memory has landed before the block leaves
   cp_async_wait_all();
-  // the last block to finish resets the barrier counters for the next call
-  if (tid == 0) {
-    const uint32_t old = atomicAdd(f.cnt + 3, 1u);
-    if (old == (uint32_t)nb - 1) {
-      f.cnt[0] = 0u;
-      f.cnt[1] = 0u;
-      __threadfence();
-      f.cnt[3] = 0u;
-    }
-  }
 }
 
 }  // namespace

@@ -75,6 +75,24 @@ __device__ __forceinline__ void grid_barrier(uint32_t* cnt, uint32_t nblocks, in
   grid_wait(cnt, nblocks, status, seen, spin);
 }
 
+// Barrier counters of the single-token kernels: kSyncWords words at a fixed workspace
+// offset.  Word 0 counts the calls that have completed (the epoch); two sets of four
+// counters follow (words 4-7 and 8-11; in each: grid barriers 1-3, then the norm mode's
+// logits).  Call E uses set E & 1 and clears set (E + 1) & 1 for call E + 1: that set's
+// last user, call E - 1, completed before this call's PDL wait returned.  Block 0 adds 1
+// to the epoch after the last grid barrier, when every block has read it.  So nothing is
+// reset at the end of a call (no block waits for an atomic's return before it exits), and
+// a call whose waits ran out still leaves a clean set to the next call.  A zero-filled
+// workspace is a valid start (epoch 0, both sets clear).
+constexpr int kSyncWords = 12;
+__device__ __forceinline__ uint32_t* sync_set(uint32_t* sync, uint32_t epoch) { return sync + 4 + 4 * (epoch & 1u); }
+__device__ __forceinline__ void sync_clear_next(uint32_t* sync, uint32_t epoch) {
+  *reinterpret_cast<uint4*>(sync_set(sync, epoch + 1u)) = make_uint4(0u, 0u, 0u, 0u);
+}
+__device__ __forceinline__ void sync_finish(uint32_t* sync) {
+  asm volatile("red.relaxed.gpu.global.add.u32 [%0], 1;" ::"l"(sync) : "memory");
+}
+
 __device__ __forceinline__ void prefetch_run(const uint8_t* p, uint64_t bytes) {
   while (bytes > 0) {
     const uint32_t c = bytes > 65536 ? 65536u : (uint32_t)bytes;

@@ -151,7 +151,7 @@ def test_fused_consecutive_calls_layers_and_workspace_state(env):
     torch.cuda.synchronize()
     assert bm.bitsmoe_last_device_status(ws.ptr) == bm.ERR_CODE["WORKSPACE_STATE"]
     assert bool((y == 7.0).all())
-    # zero-filled: consecutive calls on two layers share it (the kernel leaves its counters at zero)
+    # zero-filled: consecutive calls on two layers share it (each call leaves the next one's counters clear)
     ws.buf.zero_()
     for step in range(6):
         i = step % 2
@@ -303,7 +303,7 @@ def test_bounded_wait_runs_out_and_is_reported(env):
         bm.bitsmoe_debug_wait_limit(0, 0)
     assert bm.bitsmoe_last_device_status(ws.ptr) == bm.ERR_CODE["TIMEOUT"]
     assert bm.bitsmoe_last_device_status(ws.ptr) == 0          # read and cleared
-    check(env, layer, x, logits, spec.top_k, L=L, ws=ws)       # the counters were left at zero
+    check(env, layer, x, logits, spec.top_k, L=L, ws=ws)       # the next call's counters were cleared
 
 
 def test_debug_bounds_check_reports_and_skips(env):
