@@ -66,7 +66,8 @@ struct CStage {            // one per gate/up item (h < 2, e, segment)
   uint8_t nr;              // buckets the item touches
   uint8_t bits[kNumBk];    // their bit-widths
   uint16_t ntl[kNumBk];    // tiles per touched bucket
-  uint8_t pad_[8];
+  uint32_t meta0;          // offset in the metadata mirror of row block 0's [unit | alpha | scale/zero G rows]
+  uint8_t pad_[4];
 };
 static_assert(sizeof(CStage) == 80, "CStage layout");
 
@@ -76,7 +77,8 @@ struct DStage {            // one per down tile (e, tile < ul_max_tiles)
   uint64_t sz;             // image offset of its first slot's scale/zero in group row 0
   uint32_t sz_row;         // bytes between group rows
   uint32_t bits;           // 0: the expert has no tile of this index
-  uint32_t pad_[2];
+  uint32_t meta;           // offset in the metadata mirror of [unit 32 | alpha 32 | scale/zero NG rows of 32]
+  uint32_t pad_;
 };
 static_assert(sizeof(DStage) == 48, "DStage layout");
 
@@ -85,6 +87,8 @@ static_assert(sizeof(DStage) == 48, "DStage layout");
 struct FusedArgs {
   uint32_t* sync;    // [kSyncWords] epoch and two sets of barrier counters (fused_common.cuh)
   const CStage* cst; // [2][E][nseg]
+  const uint8_t* meta;   // metadata mirror: each staging item's unit indices, alphas and scale/zero rows
+  uint64_t meta_bytes;   //   contiguous, so that one copy stages them
   const DStage* dst; // [E][ul_max_tiles] (directly after cst)
   uint64_t tab_bytes;  // bytes of both tables
   const float* hn;     // norm mode (pre-norm block): hidden state h [D] to normalise; y = h accumulates
@@ -207,7 +211,8 @@ cudaError_t launch_dn_tc(const Fwd& p, int ul_max_tiles, cudaStream_t st, bool p
 // h of the pairs of the tensor-core down kernel, as its bf16 pair and group sums.
 cudaError_t launch_h_pack(const Fwd& p, cudaStream_t st, bool pdl);
 // Staging records of a packed image (host side, at upload).
-void build_stage_tables(const uint8_t* img, std::vector<CStage>& cst, std::vector<DStage>& dst);
+bool build_stage_tables(const uint8_t* img, std::vector<CStage>& cst, std::vector<DStage>& dst,
+                        std::vector<uint8_t>& meta);
 // Records of the clustered kernel for cluster size CL (host side, at upload):
 // per rank r, [F2Gu gate E][F2Gu up E][F2Dn E]; and the largest staged sizes.
 // False when a record would reach outside the image (the kernel is then not used).

@@ -49,6 +49,9 @@ struct bitsmoe_layer {
   const CStage* d_cst = nullptr;
   const DStage* d_dst = nullptr;
   uint64_t stage_bytes = 0;
+  const uint8_t* d_meta = nullptr;   // metadata mirror of the staging items (inside d_stage's allocation)
+  uint64_t meta_bytes = 0;
+  bool meta_ok = false;              // the mirror was built (the fused kernel needs it)
   alignas(64) uint8_t map_in[128];    // TMA maps of the two input bases and of the output basis
   alignas(64) uint8_t map_out[128];
   bool maps = false;
@@ -1453,7 +1456,8 @@ bool fused_fits(const bitsmoe_layer* L, int top_k) {
   const ImageHeader& hd = L->hd();
   FusedArgs fa;
   const int s16 = (int)align_up(std::max(hd.seg_max_slots, 8), 64) + 8;
-  return decode_mode(hd, 1) && fused_plan(hd, 1, top_k, L->seg_bytes, L->ul_max_chunks, s16, L->num_sms, &fa);
+  return decode_mode(hd, 1) && L->meta_ok &&
+         fused_plan(hd, 1, top_k, L->seg_bytes, L->ul_max_chunks, s16, L->num_sms, &fa);
 }
 
 // The clustered single-token plan for this layer and top_k: the index of its cluster
@@ -1577,7 +1581,7 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
     }
   }
   FusedArgs fa;
-  if (p.decode && fused_plan(hd, T, top_k, L->seg_bytes, L->ul_max_chunks, p.s16, sms, &fa)) {
+  if (p.decode && L->meta_ok && fused_plan(hd, T, top_k, L->seg_bytes, L->ul_max_chunks, p.s16, sms, &fa)) {
     // one token: the whole layer in one persistent kernel
     fa.sync = reinterpret_cast<uint32_t*>(wb + w.sync);
     fa.dbg = g_dbg_skip.load() | (g_dbg_bounds.load() ? 2 : 0);
@@ -1585,6 +1589,8 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
     fa.cst = L->d_cst;
     fa.dst = L->d_dst;
     fa.tab_bytes = L->stage_bytes;
+    fa.meta = L->d_meta;
+    fa.meta_bytes = L->meta_bytes;
     if (norm) {
       fa.norm = 1;
       fa.hn = norm->h;
@@ -1703,8 +1709,10 @@ int upload(std::vector<uint8_t>&& img, int device, bitsmoe_layer** out) {
   // staging records of the fused single-token kernel, derived from the image
   std::vector<CStage> cst;
   std::vector<DStage> dst;
-  build_stage_tables(img.data(), cst, dst);
+  std::vector<uint8_t> meta;
+  const bool meta_ok = build_stage_tables(img.data(), cst, dst, meta);
   const size_t cst_bytes = cst.size() * sizeof(CStage), dst_bytes = dst.size() * sizeof(DStage);
+  const size_t meta_at = align_up(cst_bytes + dst_bytes, 256);
   // records of the clustered single-token kernel for every cluster size, one buffer
   std::vector<uint8_t> f2all;
   uint64_t f2_off[5] = {};
@@ -1728,9 +1736,10 @@ int upload(std::vector<uint8_t>&& img, int device, bitsmoe_layer** out) {
   if (e == cudaSuccess) e = cudaMalloc(&d, img.size() + slack);
   if (e == cudaSuccess) e = cudaMemcpy(d, img.data(), img.size(), cudaMemcpyHostToDevice);
   if (e == cudaSuccess && slack) e = cudaMemset(d + img.size(), 0, slack);
-  if (e == cudaSuccess) e = cudaMalloc(&ds, cst_bytes + dst_bytes + 16);
+  if (e == cudaSuccess) e = cudaMalloc(&ds, meta_at + meta.size() + 16);
   if (e == cudaSuccess && cst_bytes) e = cudaMemcpy(ds, cst.data(), cst_bytes, cudaMemcpyHostToDevice);
   if (e == cudaSuccess && dst_bytes) e = cudaMemcpy(ds + cst_bytes, dst.data(), dst_bytes, cudaMemcpyHostToDevice);
+  if (e == cudaSuccess && !meta.empty()) e = cudaMemcpy(ds + meta_at, meta.data(), meta.size(), cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMalloc(&df2, f2all.size() + 16);
   if (e == cudaSuccess && !f2all.empty()) e = cudaMemcpy(df2, f2all.data(), f2all.size(), cudaMemcpyHostToDevice);
   cudaSetDevice(prev);
@@ -1757,6 +1766,9 @@ int upload(std::vector<uint8_t>&& img, int device, bitsmoe_layer** out) {
   L->d_cst = reinterpret_cast<const CStage*>(ds);
   L->d_dst = reinterpret_cast<const DStage*>(ds + cst_bytes);
   L->stage_bytes = cst_bytes + dst_bytes;
+  L->d_meta = ds + meta_at;
+  L->meta_bytes = meta.size();
+  L->meta_ok = meta_ok && !meta.empty();
   {
     const ImageHeader* h = header_of(img.data());
     L->maps = make_basis_map(L->map_in, d + h->off_basis_in, 2 * h->n, h->D_pad) &&
@@ -1941,7 +1953,7 @@ int forward_launches(const bitsmoe_layer* L, int T, int top_k, bool allow_f2) {
   const bool decode = decode_mode(hd, T);
   FusedArgs fa;
   const int s16 = (int)align_up(std::max(hd.seg_max_slots, 8), 64) + 8;
-  if (decode && fused_plan(hd, T, top_k, L->seg_bytes, L->ul_max_chunks, s16, L->num_sms, &fa)) return 1;
+  if (decode && L->meta_ok && fused_plan(hd, T, top_k, L->seg_bytes, L->ul_max_chunks, s16, L->num_sms, &fa)) return 1;
   if (T <= kFusedMaxTokens && fused_fits(L, top_k)) return T;   // one fused forward per token
   if (decode || !L->maps) return 5;
   return 3 + (L->tcx ? 2 : 1) + (L->tcd ? 3 : 1);   // router, projection, gate/up, [h pack,] down, output basis

@@ -73,7 +73,8 @@ __device__ __forceinline__ DStage load_drec(const DStage* src) {
   r.sz = u64_of(b.z, b.w);
   r.sz_row = c.x;
   r.bits = c.y;
-  r.pad_[0] = r.pad_[1] = 0;
+  r.meta = c.z;
+  r.pad_ = 0;
   return r;
 }
 
@@ -159,32 +160,27 @@ __device__ float ul_tile_rt(int b, const uint8_t* code, int NRB, int rb0, int st
   return accf;
 }
 
-// The copies of a gate/up item of row block rb and of a down tile lie inside the image.
+// The copies of a gate/up item of row block rb and of a down tile lie inside the image and
+// the metadata mirror.
 template <int G>
-__device__ bool crec_ok(const Fwd& p, const CStage& r, int rb) {
-  const int g_base = (rb * kRows) / p.group;
-  return in_image(p, r.code0 + (uint64_t)rb * r.rb_stride, r.bytes) && in_image(p, r.unit0, r.mb) &&
-         in_image(p, r.alpha0, r.mb) && in_image(p, r.sz0 + (uint64_t)(g_base + G - 1) * r.sz_row, r.mb);
+__device__ bool crec_ok(const Fwd& p, const FusedArgs& f, const CStage& r, int rb) {
+  const uint64_t mrow = (uint64_t)(2 + G) * r.mb;
+  return in_image(p, r.code0 + (uint64_t)rb * r.rb_stride, r.bytes) && r.meta0 + (rb + 1) * mrow <= f.meta_bytes;
 }
-__device__ bool drec_ok(const Fwd& p, const DStage& r) {
-  return in_image(p, r.code, (uint64_t)p.NRB * ul_chunks((int)r.bits) * kChunkBytes) && in_image(p, r.unit, 128) &&
-         in_image(p, r.alpha, 128) && in_image(p, r.sz + (uint64_t)(p.NG - 1) * r.sz_row, 128);
+__device__ bool drec_ok(const Fwd& p, const FusedArgs& f, const DStage& r) {
+  return in_image(p, r.code, (uint64_t)p.NRB * ul_chunks((int)r.bits) * kChunkBytes) &&
+         (uint64_t)r.meta + 256 + (uint64_t)p.NG * 128 <= f.meta_bytes;
 }
 
-// Copies of one gate/up item into a slot: [codes seg_al][unit smax][alpha smax][scale/zero G x smax].
+// Copies of one gate/up item into a slot: [codes seg_al][unit mb][alpha mb][scale/zero G x mb]
+// (mb = 4 bytes a slot of the item): the codes from the image, the rest from the metadata
+// mirror, where they lie together, in one copy.
 template <int G>
 __device__ void c_stage(const Fwd& p, const FusedArgs& f, const CStage& r, int rb, uint8_t* slot, uint64_t* bar) {
-  uint8_t* su = slot + f.seg_al;
-  uint8_t* sa = su + (size_t)f.smax * 4;
-  uint8_t* ssz = sa + (size_t)f.smax * 4;
-  const int g_base = (rb * kRows) / p.group;
-  mbar_expect_tx(bar, r.bytes + (2 + G) * r.mb);
+  const uint32_t mrow = (2 + G) * r.mb;
+  mbar_expect_tx(bar, r.bytes + mrow);
   bulk_run(slot, p.img + r.code0 + (uint64_t)rb * r.rb_stride, r.bytes, bar);
-  bulk_g2s(su, p.img + r.unit0, r.mb, bar);
-  bulk_g2s(sa, p.img + r.alpha0, r.mb, bar);
-#pragma unroll
-  for (int gl = 0; gl < G; ++gl)
-    bulk_g2s(ssz + (size_t)gl * f.smax * 4, p.img + r.sz0 + (uint64_t)(g_base + gl) * r.sz_row, r.mb, bar);
+  bulk_g2s(slot + f.seg_al, f.meta + r.meta0 + (uint64_t)rb * mrow, mrow, bar);
 }
 
 // One staged gate/up item for the single token: adds its partial rows of gate
@@ -192,9 +188,10 @@ __device__ void c_stage(const Fwd& p, const FusedArgs& f, const CStage& r, int r
 template <int G>
 __device__ void c_compute(const Fwd& p, const FusedArgs& f, const CStage& r, int h, int rb, const uint8_t* slot,
                           int16_t* cq, int pair, int lane) {
+  const int ms = (int)(r.mb / 4);   // the item's slots
   const int* su = reinterpret_cast<const int*>(slot + f.seg_al);
-  const float* sa = reinterpret_cast<const float*>(su + f.smax);
-  const uint32_t* ssz = reinterpret_cast<const uint32_t*>(sa + f.smax);
+  const float* sa = reinterpret_cast<const float*>(su + ms);
+  const uint32_t* ssz = reinterpret_cast<const uint32_t*>(sa + ms);
   const float* zrow = p.z + (size_t)h * p.n_pad;   // one token: z[h][0][:]
   const int nls = r.nls;
   // c = alpha * z * scale per (slot, group), int16 with one scale per item.
@@ -222,7 +219,7 @@ __device__ void c_compute(const Fwd& p, const FusedArgs& f, const CStage& r, int
       if (i < nls) {
 #pragma unroll
         for (int gl = 0; gl < G; ++gl) {
-          const float sc = __half2float(__ushort_as_half((unsigned short)(ssz[gl * f.smax + i] & 0xFFFFu)));
+          const float sc = __half2float(__ushort_as_half((unsigned short)(ssz[gl * ms + i] & 0xFFFFu)));
           mx = fmaxf(mx, fabsf(zr[m] * sc));
         }
       }
@@ -248,7 +245,7 @@ __device__ void c_compute(const Fwd& p, const FusedArgs& f, const CStage& r, int
       if (i < nls) {
 #pragma unroll
         for (int gl = 0; gl < G; ++gl) {
-          const uint32_t w = ssz[gl * f.smax + i];
+          const uint32_t w = ssz[gl * ms + i];
           const float sc = __half2float(__ushort_as_half((unsigned short)(w & 0xFFFFu)));
           const float zp = __half2float(__ushort_as_half((unsigned short)(w >> 16)));
           const int ci = __float2int_rn(zr[m] * sc * inv);
@@ -337,17 +334,14 @@ __device__ void h_rows(const Fwd& p, int pair, int rb0, int step, int16_t* hq, f
   }
 }
 
-// D slot layout: [codes NRB * ul_max_chunks * 512][unit 32 x 4][alpha 32 x 4][scale/zero NG x 32 x 4]
+// D slot layout: [codes NRB * ul_max_chunks * 512][unit 32 x 4][alpha 32 x 4][scale/zero NG x 32 x 4]:
+// the codes from the image, the rest from the metadata mirror in one copy.
 __device__ void d_stage(const Fwd& p, const FusedArgs& f, const DStage& r, uint8_t* slot, uint64_t* bar) {
   const uint32_t cb = (uint32_t)p.NRB * ul_chunks((int)r.bits) * kChunkBytes;
-  uint8_t* su = slot + f.d_code_bytes;
-  uint8_t* sa = su + 128;
-  uint8_t* ssz = sa + 128;
-  mbar_expect_tx(bar, cb + 256 + (uint32_t)p.NG * 128);
+  const uint32_t mt = 256 + (uint32_t)p.NG * 128;
+  mbar_expect_tx(bar, cb + mt);
   bulk_run(slot, p.img + r.code, cb, bar);
-  bulk_g2s(su, p.img + r.unit, 128, bar);
-  bulk_g2s(sa, p.img + r.alpha, 128, bar);
-  for (int g = 0; g < p.NG; ++g) bulk_g2s(ssz + g * 128, p.img + r.sz + (uint64_t)g * r.sz_row, 128, bar);
+  bulk_g2s(slot + f.d_code_bytes, f.meta + r.meta, mt, bar);
 }
 
 template <int G>
@@ -576,7 +570,7 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
         const CStage* g = f.cst + ((size_t)ci.h * p.E + sel_e[ci.a]) * p.nseg + ci.sg;
         if (m == ct) {
           copy_crec(crec + ct, g);
-          if ((f.dbg & 2) && crec[ct].bytes && !crec_ok<G>(p, crec[ct], ci.rb)) {
+          if ((f.dbg & 2) && crec[ct].bytes && !crec_ok<G>(p, f, crec[ct], ci.rb)) {
             crec[ct].bytes = 0;
             report_bounds(p.status);
           }
@@ -592,7 +586,7 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
       for (int m = s; m < md; m += f.nslot_d) {
         const int i = d_item(blk, m, nb), a = i % p.k, tile = f.ul_max_tiles - 1 - i / p.k;
         DStage r = load_drec(f.dst + (size_t)sel_e[a] * f.ul_max_tiles + tile);
-        if ((f.dbg & 2) && r.bits && !drec_ok(p, r)) {
+        if ((f.dbg & 2) && r.bits && !drec_ok(p, f, r)) {
           r.bits = 0;
           report_bounds(p.status);
         }
@@ -626,7 +620,7 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
         __syncwarp();
         if (lane == 0) {
           copy_crec(crec + wid, f.cst + ((size_t)ci.h * p.E + sel_e[ci.a]) * p.nseg + ci.sg);
-          if ((f.dbg & 2) && crec[wid].bytes && !crec_ok<G>(p, crec[wid], ci.rb)) {
+          if ((f.dbg & 2) && crec[wid].bytes && !crec_ok<G>(p, f, crec[wid], ci.rb)) {
             crec[wid].bytes = 0;
             report_bounds(p.status);
           }
@@ -684,7 +678,7 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
         const int i = d_item(blk, m, nb), tile = f.ul_max_tiles - 1 - i / p.k;
         a = i % p.k;
         r = rd == 0 ? drec[sl] : load_drec(f.dst + (size_t)sel_e[a] * f.ul_max_tiles + tile);
-        if (rd > 0 && (f.dbg & 2) && r.bits && !drec_ok(p, r)) {
+        if (rd > 0 && (f.dbg & 2) && r.bits && !drec_ok(p, f, r)) {
           r.bits = 0;
           if (sub == 0 && lane == 0) report_bounds(p.status);
         }
@@ -764,11 +758,22 @@ __global__ void __launch_bounds__(kFThreads, 1) k_fused(Fwd p, FusedArgs f) {
 
 namespace bmoe {
 
-void build_stage_tables(const uint8_t* img, std::vector<CStage>& cst, std::vector<DStage>& dst) {
+bool build_stage_tables(const uint8_t* img, std::vector<CStage>& cst, std::vector<DStage>& dst,
+                        std::vector<uint8_t>& meta) {
   const ImageHeader& hd = *header_of(img);
   const ExpertDesc* desc = desc_of(img);
   const ItemRec* items = reinterpret_cast<const ItemRec*>(img + hd.off_items);
   const int E = hd.E;
+  const int G = std::max(1, kRows / hd.group);
+  // the metadata mirror: per gate/up item and row block [unit | alpha | G scale/zero rows],
+  // per down tile [unit 32 | alpha 32 | NG scale/zero rows of 32], 16-byte multiples
+  meta.clear();
+  bool fits = true;
+  auto put = [&](uint64_t off, uint32_t bytes) { meta.insert(meta.end(), img + off, img + off + bytes); };
+  auto at = [&]() -> uint32_t {
+    if (meta.size() > 0xFFFFFFF0ull) fits = false;
+    return (uint32_t)meta.size();
+  };
   cst.assign(2 * (size_t)E * hd.nseg, CStage{});
   for (int pi = 0; pi < 2 * E; ++pi) {
     const ExpertDesc& x = desc[pi];
@@ -792,6 +797,13 @@ void build_stage_tables(const uint8_t* img, std::vector<CStage>& cst, std::vecto
         if (it.bits[k] < 16) nls += it.ntl[k] * rl_units(it.bits[k]);
       }
       r.nls = (uint16_t)nls;
+      r.meta0 = at();
+      for (int rb = 0; rb < hd.NRB && fits; ++rb) {
+        const int g_base = (rb * kRows) / hd.group;
+        put(r.unit0, r.mb);
+        put(r.alpha0, r.mb);
+        for (int gl = 0; gl < G; ++gl) put(r.sz0 + (uint64_t)(g_base + gl) * r.sz_row, r.mb);
+      }
     }
   }
   dst.assign((size_t)E * hd.ul_max_tiles, DStage{});
@@ -810,9 +822,17 @@ void build_stage_tables(const uint8_t* img, std::vector<CStage>& cst, std::vecto
         r.sz = x.sz_off + slot * 4;
         r.sz_row = (uint32_t)x.nslots * 4;
         r.bits = (uint32_t)bd.bits;
+        r.meta = at();
+        if (fits) {
+          put(r.unit, 128);
+          put(r.alpha, 128);
+          for (int g = 0; g < hd.NG; ++g) put(r.sz + (uint64_t)g * r.sz_row, 128);
+        }
       }
     }
   }
+  if (!fits) meta.clear();
+  return fits;
 }
 
 bool fused_plan(const ImageHeader& hd, int T, int top_k, int seg_bytes, int ul_max_chunks, int s16, int sms,
