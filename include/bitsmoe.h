@@ -144,8 +144,9 @@ size_t bitsmoe_workspace_bytes(const bitsmoe_layer* layer, int T, int top_k);
  * CUDA graph or count launches).  A single token runs as one fused persistent
  * kernel (1) when the layer's per-block shares of the bases and factors fit
  * in shared memory, and up to 4 tokens as one such kernel per token (T);
- * otherwise the forward is a chain of 5 to 8 kernels (see
- * bitsmoe_forward_plan).  Returns a negative error code for invalid arguments. */
+ * otherwise the forward is a chain of 5 kernels, 6 with the tensor-core expert
+ * factors (see bitsmoe_forward_plan).
+ * Returns a negative error code for invalid arguments. */
 int bitsmoe_forward_launches(const bitsmoe_layer* layer, int T, int top_k);
 
 /* How a forward of T tokens runs on this layer, as a bit set:
@@ -154,9 +155,10 @@ int bitsmoe_forward_launches(const bitsmoe_layer* layer, int T, int top_k);
  *      fused kernel, else 5 <= T <= 8)
  *   4  tensor-core (tcgen05) shared-basis projections (every T > 8; the decode
  *      chain from 4 tokens)
- *   8  tensor-core gate/up factors (layers without 16-bit gate/up units whose
- *      group is a multiple of 128 rows; otherwise the dp2a kernel)
- *  16  tensor-core down factor (the same condition on the down units)
+ *   8  tensor-core gate/up factors with SiLU(gate) * up fused (T > 8 on layers
+ *      without 16-bit units whose group is a multiple of 128 rows; otherwise
+ *      the dp2a kernel): the codes enter the MMA as fp16 bit patterns
+ *  16  tensor-core down factor (the same condition; always set with 8)
  *  32  with 1: the fused kernel is the clustered one, in which a thread-block
  *      cluster owns one (routing slot, 128-row block) pair of the token and
  *      its blocks exchange partial gate/up rows through distributed shared

@@ -44,11 +44,22 @@ struct Fwd {
   float* gu;        // [P][2][I_pad]
   float* s;         // [T][n_pad]
   float* zT;        // [2][n_pad][T]: z again, token fastest (written for the tensor-core gate/up kernel)
-  uint16_t* hh;     // [P][I_pad] bf16 hi of h = SiLU(gate) * up (pairs of the tensor-core down kernel)
-  uint16_t* hl;     // [P][I_pad] bf16 lo (the rounded remainder)
-  float* hsum;      // [P][NG] sums of h over each quantisation group (zeroed before)
-  int tc_gu_min;    // > 0: the tensor-core gate/up kernel takes the experts with at least this many
-  int tc_dn_min;    //      tokens and the dp2a kernel the rest (likewise for the down factor)
+};
+
+// Buffers and sizes of the multi-token tensor-core expert kernels (expert_tc.cu).
+struct XArgs {
+  int NT;                 // rows of a token tile (16, 32 or 64): an expert's tokens in tiles of NT
+  int max_tiles;          // bound on the call's token tiles
+  int A_max;              // bound on the call's routed experts
+  int Rtot;               // rows of the h buffers (multiple of 16)
+  uint32_t ring;          // bytes of a CTA's copy ring (set at launch)
+  const float* msa;       // [2][E] max over groups and slots of |scale * alpha| of gate/up (h, e)
+  const uint32_t* zmax;   // [2][T] max over j of |z_h[t][j]| (fp32 bits)
+  uint8_t* hb;            // [NRB][Rtot rows x 512 B]: h as an fp16 pair, a token tile of N rows at its first
+                          //   row R0 as the down kernel's B tile [half 2][piece 2][N rows][128 B] (swizzled)
+  float2* hs;             // [NRB][Rtot]: (sum of h over the row block's rows, 2^(24 - S) of its scaling)
+  float* zv;              // z gathered per (projection, token tile) in unit-slot order: [K-block][128 slots][N]
+  uint64_t zv_floats;     // its length
 };
 
 // Staging records of the fused single-token kernel, derived from the image
@@ -201,15 +212,16 @@ cudaError_t launch_fused(const Fwd& p, const FusedArgs& f, int sms, cudaStream_t
 // unless y carries a residual).
 bool make_basis_map(void* map_out, const void* base, int rows, int cols_pad);
 cudaError_t launch_gemm_tc(int mode, const void* map, const Fwd& p, int sms, cudaStream_t st, bool pdl,
-                           float* zT = nullptr, void* zero = nullptr, size_t zero_bytes = 0);
-// Tensor-core gate/up factors of every routed expert (reads zT); the
-// layer's most row-lane tiles and slots of any gate/up (h, e) size the shared memory.
-cudaError_t launch_gu_tc(const Fwd& p, int max_tiles, int max_slots, cudaStream_t st, bool pdl);
-// Tensor-core down factor of every routed expert into s (zeroed before); ul_max_tiles:
-// the layer's most unit-lane tiles of any expert.
-cudaError_t launch_dn_tc(const Fwd& p, int ul_max_tiles, cudaStream_t st, bool pdl);
-// h of the pairs of the tensor-core down kernel, as its bf16 pair and group sums.
-cudaError_t launch_h_pack(const Fwd& p, cudaStream_t st, bool pdl);
+                           float* zT = nullptr, void* zero = nullptr, size_t zero_bytes = 0,
+                           uint32_t* zmax = nullptr);
+// Multi-token expert factors on tensor cores (expert_tc.cu): buffer sizes for T tokens,
+// z gathered per token tile in unit-slot order (reads zT), gate/up with h = SiLU(gate) up
+// into x.hb / x.hs (reads zmax), then the down factor of every routed expert into s
+// (zeroed before).  Persistent: `sms` CTAs.
+XArgs x_args(const ImageHeader& hd, int T, int k);
+cudaError_t launch_zgather(const Fwd& p, const XArgs& x, int sms, cudaStream_t st, bool pdl);
+cudaError_t launch_gu16(const Fwd& p, const XArgs& x, int sms, cudaStream_t st, bool pdl);
+cudaError_t launch_dn16(const Fwd& p, const XArgs& x, int sms, cudaStream_t st, bool pdl);
 // Staging records of a packed image (host side, at upload).
 bool build_stage_tables(const uint8_t* img, std::vector<CStage>& cst, std::vector<DStage>& dst,
                         std::vector<uint8_t>& meta);

@@ -30,8 +30,10 @@
 
 #include <algorithm>
 #include <atomic>
+#include <cmath>
 #include <cstring>
 #include <functional>
+#include <limits>
 #include <mutex>
 #include <vector>
 
@@ -55,10 +57,8 @@ struct bitsmoe_layer {
   alignas(64) uint8_t map_in[128];    // TMA maps of the two input bases and of the output basis
   alignas(64) uint8_t map_out[128];
   bool maps = false;
-  bool tcx = false;            // gate/up factors on tensor cores: no 16-bit units, groups of whole row blocks
-  bool tcd = false;            // down factor on tensor cores: the same conditions for the down units
-  int rl_max_tiles = 0;        // most row-lane tiles and slots of any gate/up (h, e)
-  int rl_max_slots = 0;
+  bool tcx = false;            // expert factors on tensor cores: no 16-bit units, groups of whole row blocks
+  const float* d_msa = nullptr;   // [2][E] max |scale * alpha| of each gate/up (h, e) (inside d_stage's allocation)
   std::vector<uint8_t> meta;   // host copy of header + descriptors + segment table
   int seg_bytes = 0;           // largest gate/up item: code bytes inside one row block
   int ul_max_chunks = 1;       // largest 16-byte chunks per row block of any down unit
@@ -811,7 +811,7 @@ __global__ void __launch_bounds__(kK2DecWarps * 32) k_gateup_dec(Fwd p) {
   const ExpertDesc& xd = p.desc[h * p.E + e];
   const ItemRec it = p.items[((size_t)h * p.E + e) * p.nseg + sg];
   const int ntok = p.expert_count[e], pst = p.expert_start[e];
-  if (it.nr == 0 || (p.tc_gu_min > 0 && ntok >= p.tc_gu_min)) {   // empty, or the tensor-core kernel's
+  if (it.nr == 0) {
     pdl_wait();
     return;
   }
@@ -1039,7 +1039,7 @@ __global__ void __launch_bounds__(kK3DecWarps * 32) k_down_dec(Fwd p) {
   const int r = item - a * ntg * nrc;
   const int tg = r / nrc, rc = r - tg * nrc;
   const ExpertDesc& xd = p.desc[2 * p.E + e];
-  if (tg * kK3DecWarps >= xd.ntiles || (p.tc_dn_min > 0 && p.expert_count[e] >= p.tc_dn_min)) {
+  if (tg * kK3DecWarps >= xd.ntiles) {
     pdl_wait();
     return;
   }
@@ -1200,8 +1200,18 @@ __global__ void __launch_bounds__(kK3DecWarps * 32) k_down_dec(Fwd p) {
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
+#ifndef BITSMOE_DECODE_MAX_TOKENS
+#define BITSMOE_DECODE_MAX_TOKENS 8
+#endif
+
+// Small batches run the decode chain (every kernel routes all tokens itself; the
+// single token also the fused kernel), larger ones the tensor-core chain.
+inline bool decode_mode(const ImageHeader& hd, int T) {
+  return T <= BITSMOE_DECODE_MAX_TOKENS && T * hd.E <= 4096;
+}
+
 struct WsLayout {
-  size_t status, pair_expert, pair_weight, expert_count, expert_start, pair_list, active, z, gu, s, zt, hsum, hh, hl;
+  size_t status, pair_expert, pair_weight, expert_count, expert_start, pair_list, active, z, gu, s, zmax, zt, hb, hs, zv;
   size_t x_stage, logits_stage, y_stage;
   size_t sync;   // fused single-token kernel: grid-barrier counters
   size_t total;
@@ -1226,10 +1236,15 @@ WsLayout ws_layout(const ImageHeader& hd, int T, int k) {
   w.z = take(2 * (size_t)T * hd.n_pad * 4);
   w.gu = take(P * 2 * hd.I_pad * 4);
   w.s = take((size_t)T * hd.n_pad * 4);
-  w.zt = take(2 * (size_t)T * hd.n_pad * 4);   // z again, token fastest (tensor-core gate/up)
-  w.hsum = take(P * hd.NG * 4);                 // group sums of h (tensor-core down)
-  w.hh = take(P * hd.I_pad * 2);                // h as a bf16 pair (tensor-core down)
-  w.hl = take(P * hd.I_pad * 2);
+  // tensor-core expert factors (calls past the decode chain): max |z| per token (directly after
+  // s: one clear for both), z token fastest, h tiles and their row-block sums and scales
+  const bool tcx = !decode_mode(hd, T);
+  const XArgs xa = tcx ? x_args(hd, T, k) : XArgs{};
+  w.zmax = take(tcx ? 2 * (size_t)T * 4 : 0);
+  w.zt = take(tcx ? 2 * (size_t)T * hd.n_pad * 4 : 0);
+  w.hb = take(tcx ? (size_t)hd.NRB * xa.Rtot * 512 : 0);
+  w.hs = take(tcx ? (size_t)hd.NRB * xa.Rtot * 8 : 0);
+  w.zv = take(tcx ? (size_t)xa.zv_floats * 4 : 0);
   w.x_stage = take((size_t)T * hd.D * 2);
   w.logits_stage = take((size_t)T * hd.E * 4);
   w.y_stage = take((size_t)T * hd.D * 4);
@@ -1434,19 +1449,6 @@ int num_sms_current(int* sms) {
 
 // norm != nullptr: a pre-norm block (y = h accumulates); x and logits are the workspace buffers that
 // the norm/router step fills, either as its own kernel or inside the one-token fused kernel.
-#ifndef BITSMOE_DECODE_MAX_TOKENS
-#define BITSMOE_DECODE_MAX_TOKENS 8
-#endif
-// Small batches run the decode chain (every kernel routes all tokens itself; the
-// single token also the fused kernel), larger ones the tensor-core chain.
-inline bool decode_mode(const ImageHeader& hd, int T) {
-  return T <= BITSMOE_DECODE_MAX_TOKENS && T * hd.E <= 4096;
-}
-
-#ifndef BITSMOE_TC_MIN_TOKENS
-#define BITSMOE_TC_MIN_TOKENS 8
-#endif
-constexpr int kTcMinTokens = BITSMOE_TC_MIN_TOKENS;   // tokens from which an expert's factors use tensor cores
 
 // Up to this many tokens run as one fused single-token forward per token when the layer
 // fits the fused kernel (T fused forwards beat the decode chain there).
@@ -1552,9 +1554,6 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
   p.gu = reinterpret_cast<float*>(wb + w.gu);
   p.s = reinterpret_cast<float*>(wb + w.s);
   p.zT = reinterpret_cast<float*>(wb + w.zt);
-  p.hsum = reinterpret_cast<float*>(wb + w.hsum);
-  p.hh = reinterpret_cast<uint16_t*>(wb + w.hh);
-  p.hl = reinterpret_cast<uint16_t*>(wb + w.hl);
   const int sms = L->num_sms;
   int rc;
   auto mark = [&](int i) -> int {
@@ -1645,50 +1644,73 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
   if ((rc = set_smem(k_router, router_smem))) return rc;
   if ((rc = launch(k_router, dim3((T + tpb - 1) / tpb), dim3(1024), router_smem, st, false, p))) return rc;
   if ((rc = mark(1))) return rc;
-  const bool tc = L->maps;   // tensor-core projections for multi-token calls
-  const bool tcx = tc && L->tcx;   // and tensor-core gate/up factors (z then stored token-fastest)
-  if (tc) {
-    // the gate/up and down kernels add into gu and s (cleared here with z and zT, which lie
-    // next to them); the projection stores z (and zT), the output basis stores y (or adds
-    // into it, when it holds the residual)
-    BM_CK(cudaMemsetAsync(p.z, 0,
-                          (size_t)(reinterpret_cast<uint8_t*>(p.hsum) - reinterpret_cast<uint8_t*>(p.z)) +
-                              (size_t)T * top_k * hd.NG * 4,
-                          st));
-    BM_CK(launch_gemm_tc(0, L->map_in, p, sms, st, false, tcx ? p.zT : nullptr));
-  } else if ((rc = launch_gemv_any(true, p, sms, st, pdl))) {
-    return rc;
-  }
-  if ((rc = mark(2))) return rc;
-  {   // gate/up factors (tensor cores, or the staged dp2a kernel over batches of 4 tokens), then down
-    std::function<int()> between = ev ? std::function<int()>([&]() { return mark(3); }) : std::function<int()>();
-    const int A_max = std::min(hd.E, p.P);
-    // Experts with at least kTcMinTokens tokens go to the tensor-core kernels (their codes
-    // are decoded once for all tokens), the others to the dp2a kernels (whose cost follows
-    // the tokens): each kernel skips the other's experts.
-    const bool tcd = tc && L->tcd;
-    p.tc_gu_min = tcx ? kTcMinTokens : 0;
-    p.tc_dn_min = tcd ? kTcMinTokens : 0;
-    if (G == 1) rc = launch_k2k3_dec<1, 4>(p, A_max, sms, st, pdl, std::function<int()>(), 1);
-    else if (G == 2) rc = launch_k2k3_dec<2, 4>(p, A_max, sms, st, pdl, std::function<int()>(), 1);
-    else rc = launch_k2k3_dec<4, 4>(p, A_max, sms, st, pdl, std::function<int()>(), 1);
-    if (rc) return rc;
-    if (tcx) BM_CK(launch_gu_tc(p, L->rl_max_tiles, L->rl_max_slots, st, pdl));
-    if (between && (rc = between())) return rc;
-    if (G == 1) rc = launch_k2k3_dec<1, 4>(p, A_max, sms, st, pdl, std::function<int()>(), 2);
-    else if (G == 2) rc = launch_k2k3_dec<2, 4>(p, A_max, sms, st, pdl, std::function<int()>(), 2);
-    else rc = launch_k2k3_dec<4, 4>(p, A_max, sms, st, pdl, std::function<int()>(), 2);
-    if (rc) return rc;
-    if (tcd) {
-      BM_CK(launch_h_pack(p, st, pdl));
-      BM_CK(launch_dn_tc(p, hd.ul_max_tiles, st, pdl));
+  const bool tc = L->maps;          // tensor-core projections for multi-token calls
+  const bool tcx = tc && L->tcx;    // and the expert factors on tensor cores
+  const int A_max = std::min(hd.E, p.P);
+  if (tcx) {
+    // expert factors on tensor cores: the down kernel adds into s and the projection takes
+    // the max |z| of each token (both cleared here; zmax lies right after s); the projection
+    // also stores z token-fastest for the gate/up kernel
+    XArgs xa = x_args(hd, T, top_k);
+    xa.msa = L->d_msa;
+    xa.zmax = reinterpret_cast<const uint32_t*>(wb + w.zmax);
+    xa.hb = wb + w.hb;
+    xa.hs = reinterpret_cast<float2*>(wb + w.hs);
+    xa.zv = reinterpret_cast<float*>(wb + w.zv);
+    BM_CK(cudaMemsetAsync(p.s, 0, w.zmax + 2 * (size_t)T * 4 - w.s, st));
+    BM_CK(launch_gemm_tc(0, L->map_in, p, sms, st, false, p.zT, nullptr, 0, reinterpret_cast<uint32_t*>(wb + w.zmax)));
+    if ((rc = mark(2))) return rc;
+    BM_CK(launch_zgather(p, xa, sms, st, pdl));
+    BM_CK(launch_gu16(p, xa, sms, st, pdl));
+    if ((rc = mark(3))) return rc;
+    BM_CK(launch_dn16(p, xa, sms, st, pdl));
+  } else {
+    if (tc) {
+      // the dp2a gate/up and down kernels add into gu and s (cleared here with z, which lies
+      // before them); the projection stores z, the output basis stores y (or adds into it,
+      // when it holds the residual)
+      BM_CK(cudaMemsetAsync(p.z, 0, w.s + (size_t)T * hd.n_pad * 4 - w.z, st));
+      BM_CK(launch_gemm_tc(0, L->map_in, p, sms, st, false));
+    } else if ((rc = launch_gemv_any(true, p, sms, st, pdl))) {
+      return rc;
     }
+    if ((rc = mark(2))) return rc;
+    // gate/up factors (the staged dp2a kernel over batches of 4 tokens), then down
+    std::function<int()> between = ev ? std::function<int()>([&]() { return mark(3); }) : std::function<int()>();
+    if (G == 1) rc = launch_k2k3_dec<1, 4>(p, A_max, sms, st, pdl, between);
+    else if (G == 2) rc = launch_k2k3_dec<2, 4>(p, A_max, sms, st, pdl, between);
+    else rc = launch_k2k3_dec<4, 4>(p, A_max, sms, st, pdl, between);
   }
   if (rc) return rc;
   if ((rc = mark(4))) return rc;
   if (tc) BM_CK(launch_gemm_tc(1, L->map_out, p, sms, st, pdl));
   else if ((rc = launch_gemv_any(false, p, sms, st, pdl))) return rc;
   return mark(5);
+}
+
+// Per gate/up (h, e): the largest |scale * alpha| over its groups and slots, in the fp32
+// arithmetic of the tensor-core gate/up kernel (which bounds its operand by it).
+std::vector<float> gate_up_scale_bounds(const uint8_t* img) {
+  const ImageHeader& hd = *header_of(img);
+  const ExpertDesc* xd = desc_of(img);
+  std::vector<float> out(2 * (size_t)hd.E, 0.f);
+  auto f16 = [](uint32_t b) {   // IEEE binary16 bits -> float
+    const int s = (b >> 15) & 1, e = (b >> 10) & 31, m = b & 1023;
+    const float v = e == 0 ? std::ldexp((float)m, -24)
+                    : e == 31 ? (m ? std::numeric_limits<float>::quiet_NaN() : std::numeric_limits<float>::infinity())
+                              : std::ldexp((float)(m | 1024), e - 25);
+    return s ? -v : v;
+  };
+  for (int i = 0; i < 2 * hd.E; ++i) {
+    const ExpertDesc& x = xd[i];
+    const float* al = reinterpret_cast<const float*>(img + x.alpha_off);
+    const uint32_t* sz = reinterpret_cast<const uint32_t*>(img + x.sz_off);
+    float m = 0.f;
+    for (int g = 0; g < hd.NG; ++g)
+      for (int j = 0; j < x.nslots; ++j) m = std::max(m, std::fabs(f16(sz[(size_t)g * x.nslots + j] & 0xFFFFu) * al[j]));
+    out[i] = m;
+  }
+  return out;
 }
 
 int check_device(const bitsmoe_layer* L) {
@@ -1713,6 +1735,8 @@ int upload(std::vector<uint8_t>&& img, int device, bitsmoe_layer** out) {
   const bool meta_ok = build_stage_tables(img.data(), cst, dst, meta);
   const size_t cst_bytes = cst.size() * sizeof(CStage), dst_bytes = dst.size() * sizeof(DStage);
   const size_t meta_at = align_up(cst_bytes + dst_bytes, 256);
+  const std::vector<float> msa = gate_up_scale_bounds(img.data());
+  const size_t msa_at = align_up(meta_at + meta.size(), 256);
   // records of the clustered single-token kernel for every cluster size, one buffer
   std::vector<uint8_t> f2all;
   uint64_t f2_off[5] = {};
@@ -1736,7 +1760,8 @@ int upload(std::vector<uint8_t>&& img, int device, bitsmoe_layer** out) {
   if (e == cudaSuccess) e = cudaMalloc(&d, img.size() + slack);
   if (e == cudaSuccess) e = cudaMemcpy(d, img.data(), img.size(), cudaMemcpyHostToDevice);
   if (e == cudaSuccess && slack) e = cudaMemset(d + img.size(), 0, slack);
-  if (e == cudaSuccess) e = cudaMalloc(&ds, meta_at + meta.size() + 16);
+  if (e == cudaSuccess) e = cudaMalloc(&ds, msa_at + msa.size() * 4 + 16);
+  if (e == cudaSuccess) e = cudaMemcpy(ds + msa_at, msa.data(), msa.size() * 4, cudaMemcpyHostToDevice);
   if (e == cudaSuccess && cst_bytes) e = cudaMemcpy(ds, cst.data(), cst_bytes, cudaMemcpyHostToDevice);
   if (e == cudaSuccess && dst_bytes) e = cudaMemcpy(ds + cst_bytes, dst.data(), dst_bytes, cudaMemcpyHostToDevice);
   if (e == cudaSuccess && !meta.empty()) e = cudaMemcpy(ds + meta_at, meta.data(), meta.size(), cudaMemcpyHostToDevice);
@@ -1769,6 +1794,7 @@ int upload(std::vector<uint8_t>&& img, int device, bitsmoe_layer** out) {
   L->d_meta = ds + meta_at;
   L->meta_bytes = meta.size();
   L->meta_ok = meta_ok && !meta.empty();
+  L->d_msa = reinterpret_cast<const float*>(ds + msa_at);
   {
     const ImageHeader* h = header_of(img.data());
     L->maps = make_basis_map(L->map_in, d + h->off_basis_in, 2 * h->n, h->D_pad) &&
@@ -1778,15 +1804,11 @@ int upload(std::vector<uint8_t>&& img, int device, bitsmoe_layer** out) {
     for (int i = 0; i < 2 * h->E; ++i) {
       for (int k = 0; k < xd[i].nbk; ++k)
         if (xd[i].bk[k].bits >= 16) ok16 = false;
-      L->rl_max_tiles = std::max(L->rl_max_tiles, (int)xd[i].ntiles);
-      L->rl_max_slots = std::max(L->rl_max_slots, (int)xd[i].nslots);
     }
-    L->tcx = ok16;
-    bool okd = h->group % kRows == 0;
     for (int i = 2 * h->E; i < 3 * h->E; ++i)
       for (int k = 0; k < xd[i].nbk; ++k)
-        if (xd[i].bk[k].bits >= 16) okd = false;
-    L->tcd = okd;
+        if (xd[i].bk[k].bits >= 16) ok16 = false;
+    L->tcx = ok16;
   }
   const ImageHeader* hd = header_of(img.data());
   const size_t meta_end = hd->off_basis_in;   // header + descriptors + segments
@@ -1956,7 +1978,7 @@ int forward_launches(const bitsmoe_layer* L, int T, int top_k, bool allow_f2) {
   if (decode && L->meta_ok && fused_plan(hd, T, top_k, L->seg_bytes, L->ul_max_chunks, s16, L->num_sms, &fa)) return 1;
   if (T <= kFusedMaxTokens && fused_fits(L, top_k)) return T;   // one fused forward per token
   if (decode || !L->maps) return 5;
-  return 3 + (L->tcx ? 2 : 1) + (L->tcd ? 3 : 1);   // router, projection, gate/up, [h pack,] down, output basis
+  return L->tcx ? 6 : 5;   // router, projection, [z gather,] gate/up, down, output basis
 }
 }  // namespace
 
@@ -1972,7 +1994,7 @@ int bitsmoe_forward_plan(const bitsmoe_layer* L, int T, int top_k) {
   if (T <= kFusedMaxTokens && fused_fits(L, top_k)) return 1;
   const ImageHeader& hd = L->hd();
   if (decode_mode(hd, T)) return 2 | (L->maps && T >= 4 ? 4 : 0);
-  return L->maps ? 4 | (L->tcx ? 8 : 0) | (L->tcd ? 16 : 0) : 0;
+  return L->maps ? 4 | (L->tcx ? 8 | 16 : 0) : 0;
 }
 
 int bitsmoe_block_forward_launches(const bitsmoe_layer* L, int T, int top_k) {

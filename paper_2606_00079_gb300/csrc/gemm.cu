@@ -59,6 +59,7 @@ struct GemmArgs {
   const float* s;    // mode 1: [T][n_pad]
   float* z;          // mode 0: [2][T][n_pad]
   float* zT;         // mode 0: null, or [2][n_pad][T] (token fastest): also written
+  uint32_t* zmax;    // mode 0: null, or [2][T] max_j |z_h[t][j]| as fp32 bits (zeroed before)
   float* y;          // mode 1: [T][D]
   float4* zero;      // null, or a buffer of later kernels to clear (after the PDL wait)
   size_t zero_n;     // its length in float4
@@ -281,7 +282,8 @@ __global__ void __launch_bounds__(kGThreads, 1) k_gemm_tc(const __grid_constant_
         const int c = e / rs, rr = rbeg + (e - c * rs);
         const float sum = (v[b][0] + v[b][1]) + (v[b][2] + v[b][3]);
         const int m = m0 + rr, t = g.t0 + c;
-        if (m < g.M && t < g.T) {
+        const bool in = m < g.M && t < g.T;
+        if (in) {
           if (g.mode == 0) {
             const int h = m >= g.n, j = m - h * g.n;
             g.z[((size_t)h * g.T + t) * g.n_pad + j] = sum;
@@ -289,6 +291,18 @@ __global__ void __launch_bounds__(kGThreads, 1) k_gemm_tc(const __grid_constant_
           } else {
             float* yp = g.y + (size_t)t * g.D + m;
             *yp = g.accum ? *yp + sum : sum;
+          }
+        }
+        if (g.mode == 0 && g.zmax) {   // max |z| per (h, token): one atomic per warp where its lanes agree
+          const int key = in ? (m >= g.n ? g.T : 0) + t : -1;
+          const uint32_t am = in ? __float_as_uint(fabsf(sum)) : 0u;
+          const unsigned act = __activemask();
+          const int k0 = __shfl_sync(act, key, __ffs(act) - 1);
+          if (__all_sync(act, key == k0)) {
+            const uint32_t wm = __reduce_max_sync(act, am);
+            if (key >= 0 && lane == __ffs(act) - 1) atomicMax(g.zmax + key, wm);
+          } else if (key >= 0) {
+            atomicMax(g.zmax + key, am);
           }
         }
       }
@@ -343,7 +357,7 @@ bool make_basis_map(void* map_out, const void* base, int rows, int cols_pad) {
 // mode 0: z = Phi_{g,u}^T x (and zT, when given) for all T tokens; mode 1:
 // y = Phi_dn s, or y += Phi_dn s when p.accum.  Plain stores: nothing to clear.
 cudaError_t launch_gemm_tc(int mode, const void* map, const Fwd& p, int sms, cudaStream_t st, bool pdl, float* zT,
-                           void* zero, size_t zero_bytes) {
+                           void* zero, size_t zero_bytes, uint32_t* zmax) {
   static_assert(sizeof(CUtensorMap) == 128, "tensor map size");
   GemmArgs g;
   std::memset(&g, 0, sizeof(g));
@@ -361,6 +375,7 @@ cudaError_t launch_gemm_tc(int mode, const void* map, const Fwd& p, int sms, cud
   g.s = p.s;
   g.z = p.z;
   g.zT = zT;
+  g.zmax = zmax;
   g.zero = static_cast<float4*>(zero);
   g.zero_n = zero_bytes / 16;
   g.y = p.y;

@@ -66,9 +66,10 @@ TC_BITS = {0: 0.1, 1: 0.15, 2: 0.2, 3: 0.15, 4: 0.15, 6: 0.15, 8: 0.1}
     (600, 4, 2, 64, 40, 256, 128),    # experts with more than 256 tokens: two token tiles
 ])
 def test_tensor_expert_factors(env, T, E, k, D, n, I, group):
-    """Gate/up and down factors on tcgen05 (codes decoded once into bf16 tiles; gate/up:
-    scale * alpha * z as a bf16 pair; down: h as a bf16 pair, group scales applied to the
-    per-group partial sums): every bit-width below 16."""
+    """Gate/up and down factors on tcgen05 (codes as fp16 bit patterns, decoded once per
+    row block; gate/up: scale * alpha * z as an fp16 pair with SiLU(gate) * up in the
+    epilogue; down: h as an fp16 pair, group scales applied to the per-row-block partial
+    sums): every bit-width below 16, token tiles split at 32 tokens."""
     torch, bm = env
     spec = synth.scaled_spec(synth.WORKLOADS["tiny"], D=D, E=E, I=I, n=n, group=group, top_k=k)
     layer = synth.make_layer(spec, seed=T + n, bits_dist=TC_BITS, alpha_scale=4.0)
@@ -83,9 +84,9 @@ def test_tensor_expert_factors(env, T, E, k, D, n, I, group):
     assert rel_err(y.cpu().numpy().astype(np.float64), ref) <= TOL
 
 
-def test_tensor_and_dp2a_experts_in_one_call(env):
-    """Experts with many tokens take the tensor-core factor kernels and the others the dp2a
-    kernels in the same call (a biased logit sends every token to expert 0)."""
+def test_tensor_experts_skewed_load(env):
+    """One expert holding every token (a biased logit sends all tokens to expert 0) next
+    to experts with a single token: full and partial token tiles in one call."""
     torch, bm = env
     spec = synth.scaled_spec(synth.WORKLOADS["tiny"], D=128, E=8, I=384, n=120, group=128, top_k=2)
     layer = synth.make_layer(spec, seed=81, bits_dist=TC_BITS, alpha_scale=4.0)
