@@ -56,7 +56,7 @@
 
 namespace {
 
-constexpr int kGuCW = 12;                      // compute warps of the gate/up kernel
+constexpr int kGuCW = 16;                      // compute warps of the gate/up kernel
 constexpr int kDnCW = 16;                      // compute warps of the down kernel
 constexpr int kGuThreads = kGuCW * 32 + 64;    // and a producer warp and an MMA warp
 constexpr int kDnThreads = kDnCW * 32 + 64;
