@@ -44,6 +44,8 @@ struct Fwd {
   float* gu;        // [P][2][I_pad]
   float* s;         // [T][n_pad]
   float* zT;        // [2][n_pad][T]: z again, token fastest (written for the tensor-core gate/up kernel)
+  int tc_min;       // > 0: experts with at least this many tokens take the tensor-core factor kernels,
+                    //      the dp2a kernels skip them (and the tensor-core kernels the others)
 };
 
 // Buffers and sizes of the multi-token tensor-core expert kernels (expert_tc.cu).
@@ -58,6 +60,7 @@ struct XArgs {
   uint8_t* hb;            // [NRB][Rtot rows x 512 B]: h as an fp16 pair, a token tile of N rows at its first
                           //   row R0 as the down kernel's B tile [half 2][piece 2][N rows][128 B] (swizzled)
   float2* hs;             // [NRB][Rtot]: (sum of h over the row block's rows, 2^(24 - S) of its scaling)
+  int tc_min;             // experts with fewer tokens are left to the dp2a kernels
   float* zv;              // z gathered per (projection, token tile) in unit-slot order: [K-block][128 slots][N]
   uint64_t zv_floats;     // its length
 };

@@ -147,7 +147,8 @@ __device__ void build_tiles(const Fwd& p, const XArgs& x, const Tiles& t) {
   for (int a = tid; a < na; a += (int)blockDim.x) {
     const int e = p.active[1 + a];
     t.a_e[a] = e;
-    t.a_cnt[a] = p.expert_count[e];
+    const int c = p.expert_count[e];
+    t.a_cnt[a] = c >= x.tc_min ? c : 0;   // fewer tokens: the dp2a kernels' expert (no tiles)
     t.a_pst[a] = p.expert_start[e];
   }
   __syncthreads();

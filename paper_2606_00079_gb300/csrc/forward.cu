@@ -811,7 +811,7 @@ __global__ void __launch_bounds__(kK2DecWarps * 32) k_gateup_dec(Fwd p) {
   const ExpertDesc& xd = p.desc[h * p.E + e];
   const ItemRec it = p.items[((size_t)h * p.E + e) * p.nseg + sg];
   const int ntok = p.expert_count[e], pst = p.expert_start[e];
-  if (it.nr == 0) {
+  if (it.nr == 0 || (p.tc_min > 0 && ntok >= p.tc_min)) {   // empty, or the tensor-core kernels' expert
     pdl_wait();
     return;
   }
@@ -1039,7 +1039,7 @@ __global__ void __launch_bounds__(kK3DecWarps * 32) k_down_dec(Fwd p) {
   const int r = item - a * ntg * nrc;
   const int tg = r / nrc, rc = r - tg * nrc;
   const ExpertDesc& xd = p.desc[2 * p.E + e];
-  if (tg * kK3DecWarps >= xd.ntiles) {
+  if (tg * kK3DecWarps >= xd.ntiles || (p.tc_min > 0 && p.expert_count[e] >= p.tc_min)) {
     pdl_wait();
     return;
   }
@@ -1202,6 +1202,17 @@ __global__ void __launch_bounds__(kK3DecWarps * 32) k_down_dec(Fwd p) {
 // ---------------------------------------------------------------------------
 #ifndef BITSMOE_DECODE_MAX_TOKENS
 #define BITSMOE_DECODE_MAX_TOKENS 8
+#endif
+// Tokens from which an expert's factors use the tensor-core kernels (their cost follows the
+// codes, the dp2a kernels' the tokens): measured crossovers on GB300 are about 8 tokens for
+// Qwen3-sized experts (768 x 2048 codes a matrix) and at most 4 for Mixtral-sized ones
+// (14336 x 4096), whose per-item costs amortise over far more codes.
+#ifndef BITSMOE_TC_MIN_TOKENS
+inline int tc_min_tokens(const ImageHeader& hd) {
+  return (uint64_t)hd.I_pad * (uint64_t)hd.n_pad >= (8ull << 20) ? 4 : 8;
+}
+#else
+inline int tc_min_tokens(const ImageHeader&) { return BITSMOE_TC_MIN_TOKENS; }
 #endif
 
 // Small batches run the decode chain (every kernel routes all tokens itself; the
@@ -1648,22 +1659,34 @@ int forward_impl(const void* x, const float* logits, int T, int top_k, const bit
   const bool tcx = tc && L->tcx;    // and the expert factors on tensor cores
   const int A_max = std::min(hd.E, p.P);
   if (tcx) {
-    // expert factors on tensor cores: the down kernel adds into s and the projection takes
-    // the max |z| of each token (both cleared here; zmax lies right after s); the projection
-    // also stores z token-fastest for the gate/up kernel
+    // Experts with at least tc_min_tokens tokens take the tensor-core factor kernels (their codes
+    // are decoded once for all their tokens), the others the dp2a kernels (whose cost follows
+    // the tokens); each kind skips the other's experts, both add into s.  Cleared here: gu
+    // (dp2a gate/up adds into it), s, and the max |z| per token that the projection takes;
+    // z lies before them, zmax right after s.  The projection also stores z token-fastest.
+    p.tc_min = tc_min_tokens(hd);
     XArgs xa = x_args(hd, T, top_k);
+    xa.tc_min = p.tc_min;
     xa.msa = L->d_msa;
     xa.zmax = reinterpret_cast<const uint32_t*>(wb + w.zmax);
     xa.hb = wb + w.hb;
     xa.hs = reinterpret_cast<float2*>(wb + w.hs);
     xa.zv = reinterpret_cast<float*>(wb + w.zv);
-    BM_CK(cudaMemsetAsync(p.s, 0, w.zmax + 2 * (size_t)T * 4 - w.s, st));
+    BM_CK(cudaMemsetAsync(p.z, 0, w.zmax + 2 * (size_t)T * 4 - w.z, st));
     BM_CK(launch_gemm_tc(0, L->map_in, p, sms, st, false, p.zT, nullptr, 0, reinterpret_cast<uint32_t*>(wb + w.zmax)));
     if ((rc = mark(2))) return rc;
     BM_CK(launch_zgather(p, xa, sms, st, pdl));
     BM_CK(launch_gu16(p, xa, sms, st, pdl));
+    if (G == 1) rc = launch_k2k3_dec<1, 4>(p, A_max, sms, st, pdl, std::function<int()>(), 1);
+    else if (G == 2) rc = launch_k2k3_dec<2, 4>(p, A_max, sms, st, pdl, std::function<int()>(), 1);
+    else rc = launch_k2k3_dec<4, 4>(p, A_max, sms, st, pdl, std::function<int()>(), 1);
+    if (rc) return rc;
     if ((rc = mark(3))) return rc;
     BM_CK(launch_dn16(p, xa, sms, st, pdl));
+    if (G == 1) rc = launch_k2k3_dec<1, 4>(p, A_max, sms, st, pdl, std::function<int()>(), 2);
+    else if (G == 2) rc = launch_k2k3_dec<2, 4>(p, A_max, sms, st, pdl, std::function<int()>(), 2);
+    else rc = launch_k2k3_dec<4, 4>(p, A_max, sms, st, pdl, std::function<int()>(), 2);
+    if (rc) return rc;
   } else {
     if (tc) {
       // the dp2a gate/up and down kernels add into gu and s (cleared here with z, which lies
@@ -1978,7 +2001,7 @@ int forward_launches(const bitsmoe_layer* L, int T, int top_k, bool allow_f2) {
   if (decode && L->meta_ok && fused_plan(hd, T, top_k, L->seg_bytes, L->ul_max_chunks, s16, L->num_sms, &fa)) return 1;
   if (T <= kFusedMaxTokens && fused_fits(L, top_k)) return T;   // one fused forward per token
   if (decode || !L->maps) return 5;
-  return L->tcx ? 6 : 5;   // router, projection, [z gather,] gate/up, down, output basis
+  return L->tcx ? 8 : 5;   // router, projection, [z gather, gate/up tc,] gate/up, [down tc,] down, output basis
 }
 }  // namespace
 
