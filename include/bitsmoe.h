@@ -144,8 +144,9 @@ size_t bitsmoe_workspace_bytes(const bitsmoe_layer* layer, int T, int top_k);
  * CUDA graph or count launches).  A single token runs as one fused persistent
  * kernel (1) when the layer's per-block shares of the bases and factors fit
  * in shared memory, and up to 4 tokens as one such kernel per token (T);
- * otherwise the forward is a chain of 5 kernels, 6 with the tensor-core expert
- * factors (see bitsmoe_forward_plan).
+ * otherwise the forward is a chain of 5 kernels, 8 with the tensor-core expert
+ * factors (z gather, gate/up and down on tensor cores beside the dp2a kernels;
+ * see bitsmoe_forward_plan).
  * Returns a negative error code for invalid arguments. */
 int bitsmoe_forward_launches(const bitsmoe_layer* layer, int T, int top_k);
 
@@ -157,7 +158,9 @@ int bitsmoe_forward_launches(const bitsmoe_layer* layer, int T, int top_k);
  *      chain from 4 tokens)
  *   8  tensor-core gate/up factors with SiLU(gate) * up fused (T > 8 on layers
  *      without 16-bit units whose group is a multiple of 128 rows; otherwise
- *      the dp2a kernel): the codes enter the MMA as fp16 bit patterns
+ *      the dp2a kernel) for the experts with at least 8 tokens (4 when a
+ *      factor matrix holds at least 8 M codes), the dp2a kernel for the
+ *      others: the codes enter the MMA as fp16 bit patterns
  *  16  tensor-core down factor (the same condition; always set with 8)
  *  32  with 1: the fused kernel is the clustered one, in which a thread-block
  *      cluster owns one (routing slot, 128-row block) pair of the token and
