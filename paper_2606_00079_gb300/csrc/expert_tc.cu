@@ -742,7 +742,7 @@ __global__ void __launch_bounds__(kGuThreads, 1) k_gu16(Fwd p, XArgs x) {
         for (int hf = 0; hf < kh; ++hf) {
 #pragma unroll
           for (int k16 = 0; k16 < 4; ++k16)
-            mma_bf16(acc, sw128_desc(a0 + hf * kAHalf + 32 * k16), sw128_desc(b0 + (uint32_t)hf * 2u * m.N * 128u + 32u * k16),
+            mma_f16(acc, sw128_desc(a0 + hf * kAHalf + 32 * k16), sw128_desc(b0 + (uint32_t)hf * 2u * m.N * 128u + 32u * k16),
                      idesc, ((m.flags & 2) && hf == 0 && k16 == 0) ? 0u : 1u);
         }
         mma_commit(mdone + ab);
@@ -1364,7 +1364,7 @@ __global__ void __launch_bounds__(kDnThreads, 1) k_dn16(Fwd p, XArgs x) {
         for (int kh = 0; kh < 2; ++kh) {
 #pragma unroll
           for (int k16 = 0; k16 < 4; ++k16)
-            mma_bf16(acc, sw128_desc(a0 + kh * kAHalf + 32 * k16),
+            mma_f16(acc, sw128_desc(a0 + kh * kAHalf + 32 * k16),
                      sw128_desc(b0 + (uint32_t)kh * 2u * mr.N * 128u + 32 * k16), idesc, (kh | k16) ? 1u : 0u);
         }
         mma_commit(mdone + ab);

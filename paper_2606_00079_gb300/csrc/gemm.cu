@@ -131,8 +131,8 @@ __global__ void __launch_bounds__(kGThreads, 1) k_gemm_tc(const __grid_constant_
 #pragma unroll
         for (int k16 = 0; k16 < kKB / 16; ++k16) {
           const uint64_t ad = sw128_desc(a0 + k16 * 32);
-          mma_bf16(tmem, ad, sw128_desc(b0 + k16 * 32), idesc, (i | k16) != 0);
-          if (g.mode == 1) mma_bf16(tmem, ad, sw128_desc(b0 + b_bytes + k16 * 32), idesc, 1u);
+          mma_f16(tmem, ad, sw128_desc(b0 + k16 * 32), idesc, (i | k16) != 0);
+          if (g.mode == 1) mma_f16(tmem, ad, sw128_desc(b0 + b_bytes + k16 * 32), idesc, 1u);
         }
         mma_commit(empty + st);
       }

@@ -1,6 +1,7 @@
 // tcgen05 building blocks shared by the tensor-core kernels (library-internal):
 // shared-memory matrix descriptors for 128-byte-swizzled K-major tiles, the
-// kind::f16 instruction descriptor, MMA issue and commit, TMEM allocation and loads.
+// kind::f16 instruction descriptor (bf16 operands), MMA issue and commit, TMEM
+// allocation and loads.
 #pragma once
 #include <stdint.h>
 
@@ -25,7 +26,8 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int n) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
 }
 
-__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+// One tcgen05.mma of kind::f16 (f16 or bf16 operands, as the instruction descriptor says).
+__device__ __forceinline__ void mma_f16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
   asm volatile(
       "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
       " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
